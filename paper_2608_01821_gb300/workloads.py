@@ -1,0 +1,258 @@
+"""Seeded synthetic workloads for the DAVET step-conditioning path.
+
+This module holds sizes, level schedules and seeded input generators only; it
+contains none of the method's arithmetic.  The tests feed the same generated
+tensors to the CUDA library and to the CPU oracle, and the benchmark uses it to
+build its inputs.
+
+Workloads (shapes of an 8B-class diffusion VLM backbone with 32 heads of
+dimension 128 and 384px tiles of 27x27 visual tokens):
+
+  tiny     1 request, 4x64 heads, one 12x12 tile, levels 12/6/3, prompt 16,
+           response 32, 8 steps with levels [0,0,1,1,2,2,1,0], vocab 1024,
+           top-4 per step, seed 0
+  single   1 request, one 27x27 tile, levels 27/14/7/4, prompt 64,
+           response 128, 64 steps, level floor(4t/64), vocab 126464, top-2,
+           seed 1
+  anyres   1 request, 5 tiles, prompt 128, response 256, 128 steps, level 0
+           for t < 32 then level 2, top-2, seed 2
+  highres  4 requests, 10 tiles each, prompt 256, response 512, 256 steps,
+           level 2 for t < 224 then level 0, top-2, seed 3
+  ragged   16 requests, tiles U{1..9}, prompt U{32..256}, response
+           U{64..512}, 128 steps, level drawn per (step, request) from
+           {0,1,2,3} with p = [0.25, 0.25, 0.30, 0.20], top-2, seed 4
+
+Per-token channel count C = 3*H*D: each visual and text row carries the
+packed [query | key | value] projections of its token, so a gathered row is
+exactly one row of the attention input (pooling commutes with the linear
+projection, so pooling the projected rows equals projecting pooled rows).
+
+Value recipe: features, text rows ~ N(0, 1); logits ~ N(0, 2) (variance 2);
+all rounded to bf16 (round to nearest even).  Each tensor has its own
+torch.Generator seeded from (workload seed, tensor kind, index) through
+splitmix64, so every tensor is reproducible on its own.  Integer workload
+parameters of the ragged mix come from one splitmix64 stream (seed 4): the
+per-request (tiles, prompt, response) triples first, request by request, then
+the level schedule in step-major order.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+
+import numpy as np
+
+MASK64 = (1 << 64) - 1
+VOCAB_8B = 126464
+
+
+def splitmix64(state: int) -> tuple[int, int]:
+    """One step of splitmix64 (Steele, Lea, Flood 2014): (new_state, output)."""
+    state = (state + 0x9E3779B97F4A7C15) & MASK64
+    z = state
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & MASK64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & MASK64
+    return state, z ^ (z >> 31)
+
+
+class SplitMix64:
+    def __init__(self, seed: int):
+        self.state = seed & MASK64
+
+    def next(self) -> int:
+        self.state, out = splitmix64(self.state)
+        return out
+
+    def uniform_int(self, lo: int, hi: int) -> int:
+        """Integer in [lo, hi] (modulo reduction; bias < 2^-50 here)."""
+        return lo + self.next() % (hi - lo + 1)
+
+    def uniform01(self) -> float:
+        return (self.next() >> 11) * (1.0 / (1 << 53))
+
+
+def derive_seed(*parts: int) -> int:
+    s = 0x5DEECE66D
+    for p in parts:
+        s, _ = splitmix64(s ^ (p & MASK64))
+        _, s = splitmix64(s)
+    return s & ((1 << 63) - 1)
+
+
+# tensor kinds for derive_seed
+KIND_FEAT, KIND_TEXT, KIND_LOGITS, KIND_QKV = 1, 2, 3, 4
+
+
+@dataclasses.dataclass
+class Workload:
+    name: str
+    batch: int
+    H: int
+    D: int
+    grid: int
+    n_levels: int
+    tiles: list[int]
+    prompt: list[int]
+    resp: list[int]
+    T: int
+    schedule: np.ndarray  # int32 [T, batch]
+    V: int
+    k: int
+    seed: int
+
+    @property
+    def C(self) -> int:
+        return 3 * self.H * self.D
+
+    @property
+    def scale(self) -> float:
+        return 1.0 / math.sqrt(self.D)
+
+    def level_sides(self) -> list[int]:
+        out, g = [], self.grid
+        for _ in range(self.n_levels):
+            out.append(g)
+            g = (g + 1) // 2
+        return out
+
+    def pyramid_rows(self, b: int) -> int:
+        return self.tiles[b] * sum(g * g for g in self.level_sides())
+
+    def seq_len(self, b: int, level: int) -> int:
+        g = self.level_sides()[level]
+        return self.tiles[b] * g * g + self.prompt[b] + self.resp[b]
+
+    def step_lengths(self, t: int) -> list[int]:
+        return [self.seq_len(b, int(self.schedule[t, b])) for b in range(self.batch)]
+
+    def max_total_rows(self) -> int:
+        return sum(self.seq_len(b, 0) for b in range(self.batch))
+
+    @property
+    def total_resp(self) -> int:
+        return sum(self.resp)
+
+    def cu_resp(self) -> np.ndarray:
+        return np.concatenate([[0], np.cumsum(self.resp)]).astype(np.int32)
+
+    def text_offsets(self) -> np.ndarray:
+        n = [p + r for p, r in zip(self.prompt, self.resp)]
+        return np.concatenate([[0], np.cumsum(n)[:-1]]).astype(np.int64)
+
+    def total_text(self) -> int:
+        return sum(p + r for p, r in zip(self.prompt, self.resp))
+
+    # ------------------------------------------------------ algorithmic work
+    def attention_flops(self, t: int) -> float:
+        """4 L^2 H D per request (two GEMMs of 2 L^2 D flops per head)."""
+        return float(sum(4.0 * L * L * self.H * self.D for L in self.step_lengths(t)))
+
+    def gather_bytes(self, t: int) -> float:
+        """Read + write of every packed row (bf16)."""
+        return 2.0 * sum(self.step_lengths(t)) * self.C * 2
+
+    def pyramid_bytes(self) -> float:
+        """Read level 0 + write levels >= 1 (bf16), all requests."""
+        sides = self.level_sides()
+        rows_in = sum(self.tiles) * sides[0] ** 2
+        rows_out = sum(self.tiles) * sum(g * g for g in sides[1:])
+        return float((rows_in + rows_out) * self.C * 2)
+
+    def masked_rows(self, t: int) -> int:
+        """|M_t| summed over requests when k positions are committed per step."""
+        return sum(max(r - self.k * t, 0) for r in self.resp)
+
+    def unmask_bytes(self, t: int) -> float:
+        """Logit bytes of the masked rows (bf16)."""
+        return float(self.masked_rows(t) * self.V * 2)
+
+
+def _sched_const(T, batch, fn):
+    s = np.empty((T, batch), dtype=np.int32)
+    for t in range(T):
+        s[t, :] = fn(t)
+    return s
+
+
+def make(name: str) -> Workload:
+    if name == "tiny":
+        return Workload("tiny", 1, 4, 64, 12, 3, [1], [16], [32], 8,
+                        np.array([[0], [0], [1], [1], [2], [2], [1], [0]], dtype=np.int32),
+                        1024, 4, 0)
+    if name == "single":
+        # level ramps 0 -> 3 linearly over 64 steps: 16 steps at each level
+        return Workload("single", 1, 32, 128, 27, 4, [1], [64], [128], 64,
+                        _sched_const(64, 1, lambda t: (4 * t) // 64), VOCAB_8B, 2, 1)
+    if name == "anyres":
+        return Workload("anyres", 1, 32, 128, 27, 4, [5], [128], [256], 128,
+                        _sched_const(128, 1, lambda t: 0 if t < 32 else 2), VOCAB_8B, 2, 2)
+    if name == "highres":
+        return Workload("highres", 4, 32, 128, 27, 4, [10] * 4, [256] * 4, [512] * 4, 256,
+                        _sched_const(256, 4, lambda t: 2 if t < 224 else 0), VOCAB_8B, 2, 3)
+    if name == "ragged":
+        rng = SplitMix64(4)
+        tiles, prompt, resp = [], [], []
+        for _ in range(16):
+            tiles.append(rng.uniform_int(1, 9))
+            prompt.append(rng.uniform_int(32, 256))
+            resp.append(rng.uniform_int(64, 512))
+        cum = [0.25, 0.50, 0.80, 1.00]
+        sched = np.empty((128, 16), dtype=np.int32)
+        for t in range(128):
+            for b in range(16):
+                u = rng.uniform01()
+                sched[t, b] = next(i for i, c in enumerate(cum) if u < c)
+        return Workload("ragged", 16, 32, 128, 27, 4, tiles, prompt, resp, 128, sched,
+                        VOCAB_8B, 2, 4)
+    raise ValueError(f"unknown workload {name!r}")
+
+
+NAMES = ("tiny", "single", "anyres", "highres", "ragged")
+
+
+# ------------------------------------------------------------ value sources
+def normal_bf16(shape, seed: int, sigma: float = 1.0):
+    """bf16 CPU tensor ~ N(0, sigma^2), reproducible from `seed`."""
+    import torch
+    g = torch.Generator(device="cpu")
+    g.manual_seed(int(seed))
+    x = torch.randn(tuple(shape), generator=g, dtype=torch.float32)
+    if sigma != 1.0:
+        x.mul_(sigma)
+    return x.to(torch.bfloat16)
+
+
+def features(w: Workload, b: int):
+    """Visual tokens of request b: bf16 [tiles, G, G, C] ~ N(0,1)."""
+    return normal_bf16((w.tiles[b], w.grid, w.grid, w.C), derive_seed(w.seed, KIND_FEAT, b))
+
+
+def text_rows(w: Workload):
+    """Prompt and response rows of all requests, request-major: bf16 [sum(P+R), C]."""
+    import torch
+    parts = [normal_bf16((w.prompt[b] + w.resp[b], w.C), derive_seed(w.seed, KIND_TEXT, b))
+             for b in range(w.batch)]
+    return torch.cat(parts, 0)
+
+
+def logits(w: Workload, t: int):
+    """Step-t logits of all answer rows: bf16 [sum(R), V] ~ N(0, 2)."""
+    return normal_bf16((w.total_resp, w.V), derive_seed(w.seed, KIND_LOGITS, t), math.sqrt(2.0))
+
+
+def logits_device(w: Workload, t: int, device, out=None):
+    """Device-generated step-t logits for timing runs (torch's device RNG,
+    seeded per step; not bit-identical to `logits`)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(derive_seed(w.seed, KIND_LOGITS, t))
+    if out is None:
+        out = torch.empty((w.total_resp, w.V), dtype=torch.bfloat16, device=device)
+    tmp = torch.randn(out.shape, generator=g, dtype=torch.float32, device=device)
+    out.copy_(tmp.mul_(math.sqrt(2.0)))
+    return out
+
+
+def qkv_rows(n_rows: int, H: int, D: int, seed: int):
+    """Stand-alone attention input bf16 [n_rows, 3, H, D] ~ N(0,1)."""
+    return normal_bf16((n_rows, 3, H, D), derive_seed(seed, KIND_QKV, n_rows))
