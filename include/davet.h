@@ -1,0 +1,221 @@
+/*
+ * davet.h -- C ABI of the GB300 (sm_103a) DAVET step-conditioning library.
+ *
+ * DAVET (Denoising-Aware Visual Evidence Trajectory allocation) conditions
+ * every denoising step of a diffusion vision-language model on one view of
+ * an ordered hierarchy of visual "evidence views" built once from a single
+ * visual encoding (Sec. 4.3).  This library implements the data-parallel
+ * path that the policy drives:
+ *
+ *   davet_build_pyramid   the evidence hierarchy (Sec. 4.3), once per request
+ *   davet_gather_view     the step input [view || prompt || answer] (Eq. 5)
+ *   davet_step_attention  bidirectional attention over it (Sec. 3.1, Eq. 1)
+ *   davet_unmask_topk     argmax, confidence and confidence-ranked commit
+ *                         (Sec. 3.1, Eq. 1-2) plus the mean confidence and
+ *                         churn that drive the trajectory risk (Eq. 7)
+ *
+ * Conventions shared by every entry point:
+ *  - Pointers named *_dev, and every tensor argument, are DEVICE pointers on
+ *    the device current to the calling thread.  The caller owns every buffer;
+ *    the library never allocates, frees or retains caller memory.
+ *  - bf16 tensors are IEEE bfloat16 bit patterns (uint16), row-major, with
+ *    the layout given per function.  Tensor base pointers must be 16-byte
+ *    aligned.
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
+ *    call only enqueues work on that stream and returns without waiting; no
+ *    call synchronizes the host, so calls can be captured in a CUDA graph
+ *    once each entry point has run at least once on the device outside of a
+ *    capture (the first call per device resolves a few device addresses).
+ *  - Host-visible argument checks run before anything is enqueued and return
+ *    DAVET_ERR_INVALID_ARG or DAVET_ERR_UNSUPPORTED.  A failed launch returns
+ *    DAVET_ERR_CUDA (the CUDA error code is kept for davet_last_cuda_error).
+ *  - Values that live on the device (lengths, levels) are checked by the
+ *    kernels: an out-of-range value never leads to an out-of-bounds access;
+ *    instead the kernel clamps, skips the offending item and sets a bit in a
+ *    per-device error word that davet_device_status() reads.  Device-side
+ *    waits are bounded; a wait that gives up sets the timeout bit and the
+ *    kernel returns early (its outputs are then undefined).
+ *  - No C++ exception crosses this interface.
+ */
+#ifndef DAVET_H_
+#define DAVET_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum davet_status {
+  DAVET_OK = 0,
+  DAVET_ERR_INVALID_ARG = 1, /* null pointer, bad size, misalignment */
+  DAVET_ERR_UNSUPPORTED = 2, /* valid request outside the supported shapes */
+  DAVET_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed */
+  DAVET_ERR_TIMEOUT = 4,     /* device error word: a bounded wait gave up */
+  DAVET_ERR_DEVICE = 5       /* device error word: capacity or argument bit set */
+} davet_status;
+
+/* Device error word bits (davet_device_status). */
+#define DAVET_DEV_TIMEOUT 0x1u  /* a kernel's bounded wait gave up */
+#define DAVET_DEV_CAPACITY 0x2u /* a device-side length exceeded a capacity */
+#define DAVET_DEV_ARG 0x4u      /* a device-side argument was out of range */
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int davet_version(void);
+
+/* Static, NUL-terminated description of a status code (never NULL). */
+const char* davet_status_string(int status);
+
+/* The cudaError_t recorded by the last call on this thread that returned
+ * DAVET_ERR_CUDA (0 if none). */
+int davet_last_cuda_error(void);
+
+/*
+ * Reads the device error word of the current device into *flags (bits
+ * DAVET_DEV_*), optionally clearing it.  This call SYNCHRONIZES the device
+ * (it copies the word to the host); call it outside stream capture.
+ * Returns DAVET_OK when no bit is set, DAVET_ERR_TIMEOUT when the timeout
+ * bit is set, DAVET_ERR_DEVICE when another bit is set.
+ */
+davet_status davet_device_status(unsigned* flags, int clear);
+
+/* --------------------------------------------------------- evidence views */
+
+/*
+ * Host-only layout helper for the evidence pyramid (Sec. 4.3: an ordered
+ * hierarchy of views built from one encoding by structured pooling; the
+ * finest view is the encoding itself).
+ *   grid       side G of each square tile of visual tokens (>= 1)
+ *   n_levels   number of levels, 1..5; level 0 is the unpooled grid and
+ *              G_l = ceil(G_{l-1} / 2)
+ *   n_tiles    tiles of the request (>= 0)
+ *   level_side[n_levels]         out (nullable): G_l
+ *   level_row_offset[n_levels+1] out (nullable): first row of each level in
+ *              the level-major pyramid layout; [n_levels] is the total row
+ *              count.  Within a level, rows are tile-major, then row-major
+ *              within a tile: row = offset[l] + t*G_l^2 + y*G_l + x.
+ */
+davet_status davet_pyramid_layout(int grid, int n_levels, int n_tiles, int* level_side,
+                                  int64_t* level_row_offset);
+
+/*
+ * Builds the evidence pyramid of one request (Sec. 4.3, "structured
+ * pooling", all views constructed once before denoising).  Level l >= 1
+ * cell (y, x) is the mean of the level l-1 cells (2y+i, 2x+j), i, j in
+ * {0, 1}, that lie inside the level l-1 grid (a 2x2 stride-2 cascade; edge
+ * cells of odd grids average their in-range children only).  Accumulation
+ * is fp32 from the level below held in fp32; each level is rounded to bf16
+ * once, on store.
+ *   feat     bf16 [n_tiles][grid][grid][C], the encoding (level 0)
+ *   pyr      bf16 [level_row_offset[n_levels]][C], level-major layout of
+ *            davet_pyramid_layout.  If pyr == feat, level 0 is already in
+ *            place and only levels >= 1 are written; otherwise feat must not
+ *            overlap pyr and level 0 is copied into pyr as well.
+ *   C        channels per token, a multiple of 8
+ *   pyr_f32  nullable fp32 [level_row_offset[n_levels]][C]: every level
+ *            before rounding (level 0 widened exactly)
+ * n_tiles == 0 is a no-op.
+ */
+davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C,
+                                 float* pyr_f32, void* stream);
+
+/*
+ * Packs the input of one denoising step for a batch of requests (Eq. 5:
+ * the step is conditioned on v_t = A(v; b_t), the view selected for the
+ * step, together with the query and the current answer state).  For request
+ * b the packed rows are
+ *     [ all rows of level level_dev[b] of its pyramid (tiles in order)
+ *       || its prompt_len_dev[b] prompt rows || its resp_len_dev[b] answer rows ]
+ * and requests follow one another in batch order.  Rows are copied bit for
+ * bit.  cu_seqlens_dev[b] receives the first packed row of request b and
+ * cu_seqlens_dev[batch] the total row count.
+ *   pyr_ptrs_dev     device array [batch] of device pointers to each
+ *                    request's bf16 pyramid (davet_build_pyramid layout)
+ *   tiles_dev        int32 [batch] tiles per request
+ *   text             bf16 [*][C]; request b's prompt and answer rows are
+ *                    contiguous from row text_off_dev[b] (int64 [batch])
+ *   prompt_len_dev, resp_len_dev, level_dev   int32 [batch]
+ *   grid, n_levels, C  as for davet_build_pyramid (shared by the batch)
+ *   packed           bf16 [max_total_rows][C] output
+ *   cu_seqlens_dev   int32 [batch+1] output
+ * Device-side checks: a level outside [0, n_levels) or a negative count sets
+ * DAVET_DEV_ARG and the request contributes no visual rows; a total above
+ * max_total_rows sets DAVET_DEV_CAPACITY, rows beyond the capacity are not
+ * written and cu_seqlens is clamped to max_total_rows.
+ */
+davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* tiles_dev, const void* text,
+                               const int64_t* text_off_dev, const int32_t* prompt_len_dev,
+                               const int32_t* resp_len_dev, const int32_t* level_dev, int batch, int grid,
+                               int n_levels, int C, void* packed, int32_t* cu_seqlens_dev,
+                               int64_t max_total_rows, void* stream);
+
+/* ------------------------------------------------------- step attention */
+
+/*
+ * Bidirectional multi-head attention of one denoising step (Sec. 3.1, Eq. 1:
+ * masked positions are predicted in parallel through bidirectional
+ * attention).  For every request b, every row i of the request and head h:
+ *     out[i][h] = sum_j softmax_j(scale * q_i,h . k_j,h) v_j,h
+ * over all rows j of the same request (no causal mask, no attention across
+ * requests).  tcgen05 tensor-core kernel; bf16 inputs, fp32 accumulation and
+ * softmax, bf16 output.
+ *   qkv             bf16 [max_total_rows][3][H][D]: per row the query, key
+ *                   and value of every head (the packed rows of
+ *                   davet_gather_view with C = 3*H*D)
+ *   cu_seqlens_dev  int32 [batch+1] request boundaries, non-decreasing,
+ *                   cu[0] = 0, cu[batch] <= max_total_rows
+ *   H >= 1, D in {64, 128}, scale > 0 (usually 1/sqrt(D))
+ *   out             bf16 [max_total_rows][H][D]; rows past cu[batch] are not
+ *                   written
+ * Device-side checks: boundaries outside [0, max_total_rows] or decreasing
+ * set DAVET_DEV_ARG and are clamped.
+ */
+davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev, int batch,
+                                  int64_t max_total_rows, int H, int D, float scale, void* out, void* stream);
+
+/* ------------------------------------------------------------ unmasking */
+
+/* Bytes of device workspace that davet_unmask_topk needs for these sizes. */
+davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, size_t* bytes);
+
+/*
+ * One confidence-ranked commitment step (Sec. 3.1, Eq. 1-2) for a batch of
+ * requests.  For every masked answer row i (masked_dev[i] != 0, the set M_t):
+ *     argmax_i = smallest w with logits[i][w] = max_w logits[i][w]
+ *     conf_i   = 1 / sum_w exp(logits[i][w] - max) (the largest softmax
+ *                probability)
+ * Then, per request, the min(k, |M_t|) masked rows with the highest conf
+ * (ties: lower position first) are committed: tokens_dev[i] = argmax_i and
+ * masked_dev[i] = 0; the rest stay masked.  Also returns the inputs of the
+ * trajectory risk (Eq. 7): the mean conf over M_t and the churn, the
+ * fraction of rows of M_t that had a previous prediction whose argmax
+ * changed.
+ *   logits        bf16 [total_rows][V]; only masked rows are read
+ *   V             vocabulary size, a multiple of 8
+ *   cu_resp_dev   int32 [batch+1]: request b owns rows cu[b]..cu[b+1]-1;
+ *                 cu[batch] <= total_rows
+ *   k             commits per request per step, 1..1024
+ *   masked_dev    uint8 [total_rows] in/out
+ *   tokens_dev    int32 [total_rows] in/out (committed rows written)
+ *   argmax_dev    int32 [total_rows] in/out, nullable: in, the previous
+ *                 step's argmax (-1 = none); out, this step's argmax for every
+ *                 row of M_t.  NULL: churn is reported as 0.
+ *   conf_dev      float [total_rows], nullable: conf of every row of M_t
+ *   committed_dev int32 [batch][k], nullable: request-local positions
+ *                 committed this step in rank order, -1 padded
+ *   stats_dev     float [batch][2], nullable: (mean conf over M_t, churn)
+ *   workspace     device scratch of davet_unmask_topk_workspace() bytes
+ * Device-side checks: request boundaries outside [0, total_rows] set
+ * DAVET_DEV_ARG and are clamped.
+ */
+davet_status davet_unmask_topk(const void* logits, int V, const int32_t* cu_resp_dev, int batch,
+                               int64_t total_rows, int k, uint8_t* masked_dev, int32_t* tokens_dev,
+                               int32_t* argmax_dev, float* conf_dev, int32_t* committed_dev, float* stats_dev,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DAVET_H_ */

@@ -1,0 +1,527 @@
+// attention.cu -- bidirectional varlen multi-head attention of one denoising
+// step (Sec. 3.1, Eq. 1), on the sm_103a tensor cores.
+//
+// Design (one persistent CTA per SM, 192 threads, warp-specialized):
+//   warp 4       TMA producer: the Q tile once per work item, then K and V
+//                tiles (128 keys x D) into a 2-stage ring, 128-byte swizzled.
+//   warp 5       MMA issuer and TMEM owner: S = Q K^T into one of two TMEM
+//                S buffers (128 x 128 fp32), then O += P V into the TMEM O
+//                accumulator (128 x D fp32).  QK of tile j+1 is issued before
+//                PV of tile j so the tensor cores run while softmax works.
+//   warps 0-3    softmax + epilogue: thread r owns query row r of the tile;
+//                reads its S row from TMEM, keeps the running max in the
+//                log2 domain, writes P (bf16) to shared memory in the
+//                swizzled K-major layout the MMA reads, rescales O in TMEM
+//                only when the max grows by more than 2^8 (the result is
+//                unchanged: O and the row sum carry the same stale max), and
+//                finally normalizes O and stores it as bf16.
+// Work items are (request, head, 128-row query tile); items are ordered
+// longest request first and, within a request, head-major so that CTAs
+// running together share a head's K/V in L2.  Keys past the end of a request
+// are masked to -inf and their V rows zeroed in shared memory, so tiles may
+// straddle request boundaries and the end of the buffer.
+#include <algorithm>
+#include <cstdio>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace davet {
+namespace attn {
+
+constexpr int BM = 128;          // query rows per tile (MMA M)
+constexpr int BN = 128;          // keys per tile (MMA N of QK^T, K of PV)
+constexpr int NS = 2;            // K/V pipeline stages
+constexpr int kThreads = 192;    // 4 softmax warps + TMA warp + MMA warp
+constexpr int kMaxBatch = 1024;  // requests per call
+constexpr int kLptMaxBatch = 128;
+constexpr int kChunkBytes = 128 * 128;  // 128 rows x 128 B (64 bf16) swizzled chunk
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+template <int D>
+struct Smem {
+  static constexpr int KC = D / 64;
+  alignas(1024) uint8_t q[KC][kChunkBytes];
+  alignas(1024) uint8_t k[NS][KC][kChunkBytes];
+  alignas(1024) uint8_t v[NS][KC][kChunkBytes];
+  alignas(1024) uint8_t p[2][kChunkBytes];  // keys 0-63 | 64-127
+  uint64_t q_full, q_empty, p_full, o_done, fin;
+  uint64_t k_full[NS], v_full[NS], kv_empty[NS], s_full[2];
+  uint32_t tmem;
+  int abort;
+  int n_req;   // requests with at least one row
+  int n_items;
+  int32_t req_start[kMaxBatch];
+  int32_t req_len[kMaxBatch];
+  int32_t order[kMaxBatch];   // request index of the i-th scheduled request
+  int32_t cum[kMaxBatch + 1]; // items before the i-th scheduled request
+};
+
+struct Params {
+  const int32_t* cu;
+  int batch;
+  int H;
+  int max_rows;
+  float scale_log2;
+  uint16_t* out;
+  unsigned* err;
+};
+
+struct Item {
+  int start, len, qt, h, nkv;
+};
+
+// Coordinate along the tensor map's second dimension: slot (0 = query,
+// 1 = key, 2 = value) of head h.
+__device__ __forceinline__ int h_coord(int slot, int h, int H) { return slot * H + h; }
+
+template <int D>
+__device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H) {
+  // largest i with cum[i] <= item
+  int lo = 0, hi = s.n_req - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s.cum[mid] <= item) lo = mid; else hi = mid - 1;
+  }
+  const int b = s.order[lo];
+  const int local = item - s.cum[lo];
+  const int len = s.req_len[b];
+  const int nq = (len + BM - 1) / BM;
+  Item it;
+  it.start = s.req_start[b];
+  it.len = len;
+  it.h = local / nq;
+  it.qt = local - it.h * nq;
+  it.nkv = (len + BN - 1) / BN;
+  return it;
+}
+
+// All lanes wait; the outcome is made warp-uniform.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned* err, volatile int* abort_flag) {
+  const bool ok = mbar_wait(bar, parity, err, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attention_kernel(const __grid_constant__ CUtensorMap tmap, Params prm) {
+  constexpr int KC = D / 64;
+  extern __shared__ uint8_t smem_raw[];
+  Smem<D>& s = *reinterpret_cast<Smem<D>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const int H = prm.H;
+
+  // ---------------------------------------------------------- schedule
+  if (tid == 0) {
+    s.abort = 0;
+    bool bad = false;
+    int prev_end = 0;
+    int n = 0;
+    for (int b = 0; b < prm.batch; ++b) {
+      int a = prm.cu[b], e = prm.cu[b + 1];
+      if (a < prev_end || a > prm.max_rows || e < a || e > prm.max_rows) bad = true;
+      a = min(max(a, prev_end), prm.max_rows);
+      e = min(max(e, a), prm.max_rows);
+      prev_end = e;
+      s.req_start[b] = a;
+      s.req_len[b] = e - a;
+      if (e > a) s.order[n++] = b;
+    }
+    if (bad && blockIdx.x == 0) raise_error(prm.err, DEV_ERR_ARG);
+    s.n_req = n;
+  }
+  __syncthreads();
+  // longest request first (stable); only for modest batches
+  if (s.n_req <= kLptMaxBatch) {
+    int my_b = -1, my_rank = 0;
+    if (tid < s.n_req) {
+      my_b = s.order[tid];
+      const int L = s.req_len[my_b];
+      for (int j = 0; j < s.n_req; ++j) {
+        const int bj = s.order[j];
+        const int Lj = s.req_len[bj];
+        my_rank += (Lj > L) || (Lj == L && bj < my_b);
+      }
+    }
+    __syncthreads();
+    if (tid < s.n_req) s.order[my_rank] = my_b;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    int acc = 0;
+    for (int i = 0; i < s.n_req; ++i) {
+      s.cum[i] = acc;
+      acc += ((s.req_len[s.order[i]] + BM - 1) / BM) * H;
+    }
+    s.cum[s.n_req] = acc;
+    s.n_items = acc;
+  }
+  __syncthreads();
+  if (static_cast<int>(blockIdx.x) >= s.n_items) return;  // uniform: nothing to do
+
+  // ---------------------------------------------------- barriers, TMEM
+  if (tid == 0) {
+    mbar_init(&s.q_full, 1);
+    mbar_init(&s.q_empty, 1);
+    mbar_init(&s.p_full, 128);
+    mbar_init(&s.o_done, 1);
+    mbar_init(&s.fin, 1);
+    for (int i = 0; i < NS; ++i) {
+      mbar_init(&s.k_full[i], 1);
+      mbar_init(&s.v_full[i], 1);
+      mbar_init(&s.kv_empty[i], 1);
+    }
+    mbar_init(&s.s_full[0], 1);
+    mbar_init(&s.s_full[1], 1);
+    fence_mbar_init();
+  }
+  if (warp == 5) {
+    tmem_alloc(&s.tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s.tmem;
+  volatile int* abort_flag = &s.abort;
+
+  if (warp == 4) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmap);
+      uint32_t it = 0, wi = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
+        const Item w = decode(s, item, H);
+        if (wi > 0) ok = mbar_wait(&s.q_empty, (wi - 1) & 1, prm.err, abort_flag);
+        if (!ok) break;
+        mbar_arrive_expect_tx(&s.q_full, KC * kChunkBytes);
+        for (int c = 0; c < KC; ++c) tma_load_3d(s.q[c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), w.start + w.qt * BM);
+        for (int j = 0; j < w.nkv; ++j, ++it) {
+          const int st = it % NS;
+          if (it >= NS) ok = mbar_wait(&s.kv_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          const int row = w.start + j * BN;
+          mbar_arrive_expect_tx(&s.k_full[st], KC * kChunkBytes);
+          for (int c = 0; c < KC; ++c) tma_load_3d(s.k[st][c], &tmap, &s.k_full[st], 64 * c, h_coord(1, w.h, H), row);
+          mbar_arrive_expect_tx(&s.v_full[st], KC * kChunkBytes);
+          for (int c = 0; c < KC; ++c) tma_load_3d(s.v[st][c], &tmap, &s.v_full[st], 64 * c, h_coord(2, w.h, H), row);
+        }
+      }
+      if (!ok) {
+        // let copies already in flight land before the CTA exits
+        for (uint32_t i = (it > NS ? it - NS : 0); i < it; ++i) {
+          mbar_wait(&s.k_full[i % NS], (i / NS) & 1, nullptr, nullptr);
+          mbar_wait(&s.v_full[i % NS], (i / NS) & 1, nullptr, nullptr);
+        }
+      }
+    }
+  } else if (warp == 5) {
+    // --------------------------------------------------------- MMA issuer
+    constexpr uint32_t kIdescQK = idesc_bf16_f32(BM, BN, false, false);
+    constexpr uint32_t kIdescPV = idesc_bf16_f32(BM, D, false, true);
+    uint32_t it = 0, wi = 0;
+    bool ok = true;
+
+    auto issue_pv = [&](uint32_t i, bool first, int valid_keys) -> bool {
+      const int st = i % NS;
+      if (!warp_wait(&s.p_full, i & 1, prm.err, abort_flag)) return false;
+      if (!warp_wait(&s.v_full[st], (i / NS) & 1, prm.err, abort_flag)) return false;
+      tc_fence_after();
+      if (valid_keys < BN) {
+        // keys past the request end: zero their V rows (P is 0 there, but the
+        // rows may hold anything, including non-finite values)
+        for (int c = 0; c < KC; ++c) {
+          uint4* base = reinterpret_cast<uint4*>(s.v[st][c]);
+          for (int idx = valid_keys * 8 + lane; idx < BN * 8; idx += 32) base[idx] = make_uint4(0, 0, 0, 0);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+      }
+      if (lane == 0) {
+        const uint32_t v0 = smem_u32(s.v[st][0]);
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t a = sw128_desc(smem_u32(s.p[kk >> 2]) + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = sw128_desc(v0 + kk * 2048, kChunkBytes, 1024);
+          umma_ss(tmem + kColO, a, b, kIdescPV, (first && kk == 0) ? 0u : 1u);
+        }
+        umma_commit(&s.o_done);
+        umma_commit(&s.kv_empty[st]);
+      }
+      __syncwarp();
+      return true;
+    };
+
+    for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
+      const Item w = decode(s, item, H);
+      ok = warp_wait(&s.q_full, wi & 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      for (int j = 0; j < w.nkv; ++j, ++it) {
+        const int st = it % NS;
+        const uint32_t sb = it & 1;
+        ok = warp_wait(&s.k_full[st], (it / NS) & 1, prm.err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        if (lane == 0) {
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk & 3) * 32;
+            const uint64_t a = sw128_desc(smem_u32(s.q[kk >> 2]) + off, 16, 1024);
+            const uint64_t b = sw128_desc(smem_u32(s.k[st][kk >> 2]) + off, 16, 1024);
+            umma_ss(tmem + (sb ? kColS1 : kColS0), a, b, kIdescQK, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(&s.s_full[sb]);
+          if (j == w.nkv - 1) umma_commit(&s.q_empty);
+        }
+        __syncwarp();
+        if (j > 0) {
+          ok = issue_pv(it - 1, j == 1, BN);
+          if (!ok) break;
+        }
+      }
+      if (!ok) break;
+      const int last_valid = w.len - (w.nkv - 1) * BN;
+      ok = issue_pv(it - 1, w.nkv == 1, last_valid);
+    }
+    // wait until every issued MMA has completed before TMEM is released
+    if (lane == 0) {
+      umma_commit(&s.fin);
+      mbar_wait(&s.fin, 0, nullptr, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------- softmax + epilogue
+    const int r = tid;  // query row within the tile == TMEM lane
+    const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    uint32_t it = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x) {
+      const Item w = decode(s, item, H);
+      float m = -INFINITY;  // running max of scale*log2(e)*score
+      float l = 0.f;        // running sum of 2^(t - m)
+      for (int j = 0; j < w.nkv; ++j, ++it) {
+        const uint32_t sb = it & 1;
+        ok = warp_wait(&s.s_full[sb], (it >> 1) & 1, prm.err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        float t[BN];
+        {
+          uint32_t raw[32];
+#pragma unroll
+          for (int c = 0; c < BN / 32; ++c) {
+            tmem_ld32(tmem + lane_base + (sb ? kColS1 : kColS0) + 32 * c, raw);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) t[32 * c + i] = __uint_as_float(raw[i]);
+          }
+        }
+        const int valid = min(BN, w.len - j * BN);
+        float mt = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < BN; ++i) {
+          t[i] = (i < valid) ? t[i] * prm.scale_log2 : -INFINITY;
+          mt = fmaxf(mt, t[i]);
+        }
+        float m_new = m, factor = 1.f;
+        bool need = false;
+        if (j == 0) {
+          m_new = mt;
+        } else if (mt > m + kRescaleThreshold) {
+          m_new = mt;
+          factor = ex2(m - m_new);
+          need = true;
+        }
+        uint32_t pk[BN / 2];
+        float rs = 0.f;
+#pragma unroll
+        for (int i = 0; i < BN; i += 2) {
+          const float p0 = ex2(t[i] - m_new);
+          const float p1 = ex2(t[i + 1] - m_new);
+          rs += p0 + p1;
+          pk[i / 2] = pack_bf16x2(p0, p1);
+        }
+        l = (j == 0) ? rs : l * factor + rs;
+        m = m_new;
+        if (j > 0) {
+          // PV of the previous tile done: P buffer free, O settled
+          ok = warp_wait(&s.o_done, (it - 1) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          tc_fence_after();
+          if (__any_sync(0xffffffffu, need)) {
+            uint32_t o[32];
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+              tmem_ld32(tmem + lane_base + kColO + 32 * c, o);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+              tmem_st32(tmem + lane_base + kColO + 32 * c, o);
+            }
+            tmem_wait_st();
+          }
+        }
+        // P row -> swizzled K-major tile: 16-byte piece q of row r lands at
+        // piece (q ^ (r & 7)) of the row's 128-byte line.
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint8_t* row = s.p[c] + r * 128;
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const int base = c * 32 + q * 4;
+            const uint4 val = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
+            *reinterpret_cast<uint4*>(row + ((q ^ (r & 7)) << 4)) = val;
+          }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(&s.p_full);
+      }
+      if (!ok) break;
+      // ------------------------------------------------------- epilogue
+      ok = warp_wait(&s.o_done, (it - 1) & 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      const float inv_l = 1.f / l;
+      const int qrow = w.qt * BM + r;
+      const bool row_ok = qrow < w.len;
+      uint16_t* dst = prm.out + (static_cast<int64_t>(w.start + qrow) * H + w.h) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tmem + lane_base + kColO + 32 * c, o);
+        tmem_wait_ld();
+        if (row_ok) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * c);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(o[8 * q + 0]) * inv_l, __uint_as_float(o[8 * q + 1]) * inv_l);
+            v.y = pack_bf16x2(__uint_as_float(o[8 * q + 2]) * inv_l, __uint_as_float(o[8 * q + 3]) * inv_l);
+            v.z = pack_bf16x2(__uint_as_float(o[8 * q + 4]) * inv_l, __uint_as_float(o[8 * q + 5]) * inv_l);
+            v.w = pack_bf16x2(__uint_as_float(o[8 * q + 6]) * inv_l, __uint_as_float(o[8 * q + 7]) * inv_l);
+            d4[q] = v;
+          }
+        }
+      }
+      tc_fence_before();
+    }
+  }
+
+  // ------------------------------------------------------------ teardown
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace attn
+
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+struct DeviceInfo {
+  int sms = 0;
+  bool attr_set[2] = {false, false};
+};
+DeviceInfo g_dev[64];
+std::mutex g_dev_mu;
+
+template <int D>
+davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_rows, int H, float scale, void* out,
+                    cudaStream_t stream) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= 64) return DAVET_ERR_UNSUPPORTED;
+  const size_t smem = sizeof(attn::Smem<D>) + 1024;
+  {
+    std::lock_guard<std::mutex> g(g_dev_mu);
+    DeviceInfo& di = g_dev[dev];
+    if (di.sms == 0) {
+      e = cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return cuda_fail(e);
+    }
+    const int slot = D == 128 ? 1 : 0;
+    if (!di.attr_set[slot]) {
+      e = cudaFuncSetAttribute(attn::attention_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem));
+      if (e != cudaSuccess) return cuda_fail(e);
+      di.attr_set[slot] = true;
+    }
+  }
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return DAVET_ERR_CUDA;
+
+  CUtensorMap tmap;
+  const cuuint64_t gdim[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(3 * H),
+                              static_cast<cuuint64_t>(max_rows)};
+  const cuuint64_t gstride[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(3) * H * D * 2};
+  const cuuint32_t box[3] = {64, 1, 128};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(qkv), gdim, gstride, box, estride,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS) return DAVET_ERR_INVALID_ARG;
+
+  attn::Params prm;
+  prm.cu = cu;
+  prm.batch = batch;
+  prm.H = H;
+  prm.max_rows = static_cast<int>(max_rows);
+  prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
+  prm.out = static_cast<uint16_t*>(out);
+  prm.err = err;
+
+  const int64_t items_bound = ((max_rows + attn::BM - 1) / attn::BM + batch) * static_cast<int64_t>(H);
+  const int grid = static_cast<int>(std::min<int64_t>(items_bound, g_dev[dev].sms));
+  if (grid <= 0) return DAVET_OK;
+  attn::attention_kernel<D><<<grid, attn::kThreads, smem, stream>>>(tmap, prm);
+  return check_launch();
+}
+
+}  // namespace
+}  // namespace davet
+
+extern "C" davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev, int batch,
+                                             int64_t max_total_rows, int H, int D, float scale, void* out,
+                                             void* stream) {
+  using namespace davet;
+  if (batch < 0 || max_total_rows < 0 || H < 1 || !(scale > 0.f)) return DAVET_ERR_INVALID_ARG;
+  if (batch == 0 || max_total_rows == 0) return DAVET_OK;
+  if (!qkv || !cu_seqlens_dev || !out) return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(qkv) | reinterpret_cast<uintptr_t>(out)) & 15u) return DAVET_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return DAVET_ERR_UNSUPPORTED;
+  if (batch > attn::kMaxBatch) return DAVET_ERR_UNSUPPORTED;
+  if (max_total_rows > (int64_t(1) << 30) || static_cast<int64_t>(3) * H > 65535) return DAVET_ERR_UNSUPPORTED;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return D == 128 ? launch<128>(qkv, cu_seqlens_dev, batch, max_total_rows, H, scale, out, st)
+                  : launch<64>(qkv, cu_seqlens_dev, batch, max_total_rows, H, scale, out, st);
+}

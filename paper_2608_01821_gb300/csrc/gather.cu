@@ -1,0 +1,199 @@
+// gather.cu -- packs the input of one denoising step (Eq. 5): for every
+// request, the rows of the view its level selects followed by its prompt and
+// answer rows, plus the cu_seqlens boundaries, all computed on the device so
+// the call needs no host synchronization.
+//
+// Every block first derives the per-request lengths and their prefix sum in
+// shared memory (a block-wide scan; requests are few), then copies rows with
+// one warp per row: each lane moves 16-byte slices, eight loads in flight
+// before the matching stores, so a warp keeps 4 KB of one row in flight.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace davet {
+namespace gat {
+
+constexpr int kThreads = 256;
+constexpr int kMaxBatch = 1024;
+constexpr int kMaxLevels = 5;
+
+struct Geom {
+  int side[kMaxLevels];
+  int n_levels;
+  int C8;
+};
+
+struct Args {
+  const uint4* const* pyr;
+  const int32_t* tiles;
+  const uint4* text;
+  const int64_t* text_off;
+  const int32_t* prompt;
+  const int32_t* resp;
+  const int32_t* level;
+  int batch;
+  uint4* packed;
+  int32_t* cu_out;
+  long long cap;
+  unsigned* err;
+};
+
+__device__ __forceinline__ uint4 ld_nc(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+
+__global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
+  extern __shared__ long long sm[];
+  long long* s_cu = sm;                     // [batch+1] packed start of each request
+  long long* s_len = sm + a.batch + 1;      // [batch] packed rows of each request
+  long long* s_nvis = s_len + a.batch;      // [batch] visual rows
+  long long* s_vis0 = s_nvis + a.batch;     // [batch] first pyramid row of the chosen level
+  __shared__ long long s_warp[kThreads / 32];
+  __shared__ int s_bad;
+
+  const int tid = threadIdx.x;
+  if (tid == 0) s_bad = 0;
+  __syncthreads();
+
+  // -------- per-request lengths, then an exclusive scan into s_cu
+  const int per = (a.batch + kThreads - 1) / kThreads;
+  const int b0 = min(a.batch, tid * per), b1 = min(a.batch, b0 + per);
+  long long local = 0;
+  for (int b = b0; b < b1; ++b) {
+    const int lvl = a.level[b];
+    const int nt = a.tiles[b];
+    const int p = a.prompt[b], r = a.resp[b];
+    bool bad = false;
+    long long nvis = 0, vis0 = 0;
+    if (lvl < 0 || lvl >= g.n_levels || nt < 0) {
+      bad = true;
+    } else {
+      long long off = 0;
+      for (int l = 0; l < lvl; ++l) off += static_cast<long long>(nt) * g.side[l] * g.side[l];
+      vis0 = off;
+      nvis = static_cast<long long>(nt) * g.side[lvl] * g.side[lvl];
+    }
+    if (p < 0 || r < 0) bad = true;
+    if (bad) s_bad = 1;
+    s_nvis[b] = nvis;
+    s_vis0[b] = vis0;
+    const long long len = nvis + max(p, 0) + max(r, 0);
+    s_len[b] = len;
+    local += len;
+  }
+  // block-wide exclusive scan of the per-thread sums
+  const int lane = tid & 31, warp = tid >> 5;
+  long long incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  __syncthreads();
+  long long run = incl - local;
+  for (int w = 0; w < warp; ++w) run += s_warp[w];
+  for (int b = b0; b < b1; ++b) {
+    s_cu[b] = run;
+    run += s_len[b];
+  }
+  if (b0 < b1 && b1 == a.batch) s_cu[a.batch] = run;
+  if (a.batch == 0 && tid == 0) s_cu[0] = 0;
+  __syncthreads();
+
+  const long long total = s_cu[a.batch];
+  const long long rows = min(total, a.cap);
+  if (blockIdx.x == 0) {
+    for (int b = tid; b <= a.batch; b += kThreads) a.cu_out[b] = static_cast<int32_t>(min(s_cu[b], a.cap));
+    if (tid == 0) {
+      if (s_bad) raise_error(a.err, DEV_ERR_ARG);
+      if (total > a.cap) raise_error(a.err, DEV_ERR_CAPACITY);
+    }
+  }
+
+  // -------- row copies, one warp per row
+  const long long gwarp = (static_cast<long long>(blockIdx.x) * kThreads + tid) >> 5;
+  const long long nwarps = (static_cast<long long>(gridDim.x) * kThreads) >> 5;
+  const int C8 = g.C8;
+  for (long long row = gwarp; row < rows; row += nwarps) {
+    // request owning this row: largest b with s_cu[b] <= row
+    int lo = 0, hi = a.batch - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_cu[mid] <= row) lo = mid; else hi = mid - 1;
+    }
+    const int b = lo;
+    const long long j = row - s_cu[b];
+    const uint4* src;
+    if (j < s_nvis[b]) {
+      src = a.pyr[b] + (s_vis0[b] + j) * C8;
+    } else {
+      src = a.text + (a.text_off[b] + (j - s_nvis[b])) * C8;
+    }
+    uint4* dst = a.packed + row * C8;
+    int c = lane;
+    for (; c + 7 * 32 < C8; c += 8 * 32) {
+      uint4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = ld_nc(src + c + u * 32);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) dst[c + u * 32] = v[u];
+    }
+    for (; c < C8; c += 32) dst[c] = ld_nc(src + c);
+  }
+}
+
+}  // namespace gat
+}  // namespace davet
+
+extern "C" davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* tiles_dev,
+                                          const void* text, const int64_t* text_off_dev,
+                                          const int32_t* prompt_len_dev, const int32_t* resp_len_dev,
+                                          const int32_t* level_dev, int batch, int grid, int n_levels, int C,
+                                          void* packed, int32_t* cu_seqlens_dev, int64_t max_total_rows,
+                                          void* stream) {
+  using namespace davet;
+  using namespace davet::gat;
+  if (batch < 0 || grid < 1 || n_levels < 1 || C < 8 || C % 8 != 0 || max_total_rows < 0)
+    return DAVET_ERR_INVALID_ARG;
+  if (n_levels > kMaxLevels || grid > 65536) return DAVET_ERR_UNSUPPORTED;
+  if (batch > kMaxBatch) return DAVET_ERR_UNSUPPORTED;
+  if (max_total_rows > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
+  if (!cu_seqlens_dev) return DAVET_ERR_INVALID_ARG;
+  if (batch > 0 && (!pyr_ptrs_dev || !tiles_dev || !text || !text_off_dev || !prompt_len_dev || !resp_len_dev ||
+                    !level_dev || !packed))
+    return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(text) | reinterpret_cast<uintptr_t>(packed)) & 15u) return DAVET_ERR_INVALID_ARG;
+
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  Geom g;
+  int side[kMaxLevels];
+  davet_pyramid_layout(grid, n_levels, 0, side, nullptr);
+  for (int l = 0; l < kMaxLevels; ++l) g.side[l] = l < n_levels ? side[l] : 1;
+  g.n_levels = n_levels;
+  g.C8 = C / 8;
+  Args a;
+  a.pyr = reinterpret_cast<const uint4* const*>(pyr_ptrs_dev);
+  a.tiles = tiles_dev;
+  a.text = static_cast<const uint4*>(text);
+  a.text_off = text_off_dev;
+  a.prompt = prompt_len_dev;
+  a.resp = resp_len_dev;
+  a.level = level_dev;
+  a.batch = batch;
+  a.packed = static_cast<uint4*>(packed);
+  a.cu_out = cu_seqlens_dev;
+  a.cap = max_total_rows;
+  a.err = err;
+  const size_t smem = static_cast<size_t>(4 * batch + 1) * sizeof(long long);
+  // one warp per row: enough blocks to cover the capacity, at most 8 waves of 8 blocks per SM
+  const long long warps_needed = std::max<long long>(max_total_rows, 1);
+  const long long blocks = std::min<long long>((warps_needed + kThreads / 32 - 1) / (kThreads / 32), 152LL * 8 * 2);
+  gather_kernel<<<static_cast<unsigned>(std::max<long long>(blocks, 1)), kThreads, smem,
+                  static_cast<cudaStream_t>(stream)>>>(a, g);
+  return check_launch();
+}

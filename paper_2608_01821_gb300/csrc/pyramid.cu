@@ -1,0 +1,205 @@
+// pyramid.cu -- evidence pyramid of one request (Sec. 4.3: an ordered
+// hierarchy of views built once from a single encoding by structured
+// pooling; the finest view is the encoding itself).
+//
+// One thread owns one coarsest-level cell of one tile and one 8-channel
+// (16-byte) slice of every level below it: it streams the level-0 tokens of
+// that cell's quadtree once with 128-bit loads, reduces 2x2 children level by
+// level in fp32 registers, and stores every level it passes through.  Each
+// input byte is read once and each output byte written once; consecutive
+// threads own consecutive channel slices, so every load and store of a warp
+// covers 512 contiguous bytes of one token row.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace davet {
+namespace pyr {
+
+constexpr int kMaxLevels = 5;
+
+struct Geom {
+  int side[kMaxLevels];
+  long long off[kMaxLevels + 1];  // first row of each level (level-major)
+  int n_tiles;
+  int C8;      // 16-byte slices per row
+  bool copy0;  // level 0 must be copied into the pyramid buffer
+};
+
+struct Ctx {
+  const uint4* __restrict__ feat;
+  uint4* __restrict__ pyr;
+  float4* __restrict__ pyr32;
+  int tile;
+  int cv;
+};
+
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ void store_row(const Ctx& c, const Geom& g, long long row, const float (&v)[8]) {
+  uint4 u;
+  u.x = pack_bf16x2(v[0], v[1]);
+  u.y = pack_bf16x2(v[2], v[3]);
+  u.z = pack_bf16x2(v[4], v[5]);
+  u.w = pack_bf16x2(v[6], v[7]);
+  c.pyr[row * g.C8 + c.cv] = u;
+  if (c.pyr32) {
+    float4* d = c.pyr32 + (row * g.C8 + c.cv) * 2;
+    d[0] = make_float4(v[0], v[1], v[2], v[3]);
+    d[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
+}
+
+// Mean of cell (y, x) of level L (fp32), or false if the cell lies outside
+// the level-L grid.  Level L >= 1 averages its in-range 2x2 children of
+// level L-1 (1, 2 or 4 of them, so the scale is an exact power of two).
+template <int L, int TOP>
+__device__ __forceinline__ bool cell(const Ctx& c, const Geom& g, int y, int x, float (&v)[8]) {
+  const int gs = g.side[L];
+  if (y >= gs || x >= gs) return false;
+  const long long row = g.off[L] + (static_cast<long long>(c.tile) * gs + y) * gs + x;
+  if constexpr (L == 0) {
+    const long long src = (static_cast<long long>(c.tile) * gs + y) * gs + x;
+    const uint4 u = ld_stream(c.feat + src * g.C8 + c.cv);
+    v[0] = bf16lo(u.x); v[1] = bf16hi(u.x);
+    v[2] = bf16lo(u.y); v[3] = bf16hi(u.y);
+    v[4] = bf16lo(u.z); v[5] = bf16hi(u.z);
+    v[6] = bf16lo(u.w); v[7] = bf16hi(u.w);
+    if (g.copy0) c.pyr[row * g.C8 + c.cv] = u;
+    if (c.pyr32) {
+      float4* d = c.pyr32 + (row * g.C8 + c.cv) * 2;
+      d[0] = make_float4(v[0], v[1], v[2], v[3]);
+      d[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+    return true;
+  } else {
+    float acc[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+    int n = 0;
+    if constexpr (L == TOP) {
+      // the top level walks its four subtrees one after another so that
+      // each subtree's loads are issued together without exhausting registers
+#pragma unroll 1
+      for (int q = 0; q < 4; ++q) {
+        float ch[8];
+        if (cell<L - 1, TOP>(c, g, 2 * y + (q >> 1), 2 * x + (q & 1), ch)) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[k] += ch[k];
+          ++n;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float ch[8];
+        if (cell<L - 1, TOP>(c, g, 2 * y + (q >> 1), 2 * x + (q & 1), ch)) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[k] += ch[k];
+          ++n;
+        }
+      }
+    }
+    const float inv = n == 4 ? 0.25f : (n == 2 ? 0.5f : 1.0f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = acc[k] * inv;
+    store_row(c, g, row, v);
+    return true;
+  }
+}
+
+template <int NL>
+__global__ void pyramid_kernel(const uint4* __restrict__ feat, uint4* __restrict__ pyr, float4* __restrict__ pyr32,
+                               Geom g) {
+  constexpr int TOP = NL - 1;
+  const int gt = g.side[TOP];
+  const long long cells = static_cast<long long>(gt) * gt;
+  const long long total = static_cast<long long>(g.n_tiles) * cells * g.C8;
+  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    Ctx c;
+    c.feat = feat;
+    c.pyr = pyr;
+    c.pyr32 = pyr32;
+    c.cv = static_cast<int>(i % g.C8);
+    const long long rest = i / g.C8;
+    const int cellid = static_cast<int>(rest % cells);
+    c.tile = static_cast<int>(rest / cells);
+    float v[8];
+    cell<TOP, TOP>(c, g, cellid / gt, cellid % gt, v);
+  }
+}
+
+}  // namespace pyr
+}  // namespace davet
+
+extern "C" davet_status davet_pyramid_layout(int grid, int n_levels, int n_tiles, int* level_side,
+                                             int64_t* level_row_offset) {
+  if (grid < 1 || n_levels < 1 || n_levels > davet::pyr::kMaxLevels || n_tiles < 0) return DAVET_ERR_INVALID_ARG;
+  if (grid > 65536) return DAVET_ERR_UNSUPPORTED;
+  int g = grid;
+  int64_t off = 0;
+  for (int l = 0; l < n_levels; ++l) {
+    if (level_side) level_side[l] = g;
+    if (level_row_offset) level_row_offset[l] = off;
+    off += static_cast<int64_t>(n_tiles) * g * g;
+    g = (g + 1) / 2;
+  }
+  if (level_row_offset) level_row_offset[n_levels] = off;
+  return DAVET_OK;
+}
+
+extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C,
+                                            float* pyr_f32, void* stream) {
+  using namespace davet;
+  using namespace davet::pyr;
+  if (n_tiles < 0 || grid < 1 || n_levels < 1 || C < 8) return DAVET_ERR_INVALID_ARG;
+  if (n_levels > kMaxLevels || grid > 65536) return DAVET_ERR_UNSUPPORTED;
+  if (C % 8 != 0) return DAVET_ERR_INVALID_ARG;
+  if (n_tiles == 0) return DAVET_OK;
+  if (!feat || !pyr) return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(feat) | reinterpret_cast<uintptr_t>(pyr) |
+       reinterpret_cast<uintptr_t>(pyr_f32)) & 15u)
+    return DAVET_ERR_INVALID_ARG;
+
+  Geom g;
+  int64_t off[kMaxLevels + 1];
+  int side[kMaxLevels];
+  davet_pyramid_layout(grid, n_levels, n_tiles, side, off);
+  for (int l = 0; l < kMaxLevels; ++l) g.side[l] = l < n_levels ? side[l] : 1;
+  for (int l = 0; l <= kMaxLevels; ++l) g.off[l] = l <= n_levels ? off[l] : off[n_levels];
+  g.n_tiles = n_tiles;
+  g.C8 = C / 8;
+  g.copy0 = feat != pyr;
+  if (g.copy0) {
+    // feat and the pyramid must not overlap when level 0 is copied
+    const uintptr_t f0 = reinterpret_cast<uintptr_t>(feat), p0 = reinterpret_cast<uintptr_t>(pyr);
+    const uintptr_t f1 = f0 + static_cast<uintptr_t>(off[1]) * C * 2;
+    const uintptr_t p1 = p0 + static_cast<uintptr_t>(off[n_levels]) * C * 2;
+    if (f0 < p1 && p0 < f1) return DAVET_ERR_INVALID_ARG;
+  }
+
+  const int gt = side[n_levels - 1];
+  const long long total = static_cast<long long>(n_tiles) * gt * gt * g.C8;
+  // small problems: smaller blocks spread over more SMs
+  const int threads = total >= 152LL * 2 * 256 ? 256 : (total >= 152LL * 2 * 128 ? 128 : 64);
+  const long long blocks = std::min<long long>((total + threads - 1) / threads, 152LL * 64);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const uint4* f = static_cast<const uint4*>(feat);
+  uint4* p = static_cast<uint4*>(pyr);
+  float4* p32 = reinterpret_cast<float4*>(pyr_f32);
+  switch (n_levels) {
+    case 1: pyramid_kernel<1><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+    case 2: pyramid_kernel<2><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+    case 3: pyramid_kernel<3><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+    case 4: pyramid_kernel<4><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+    default: pyramid_kernel<5><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+  }
+  return check_launch();
+}

@@ -1,0 +1,85 @@
+// status.cu -- status strings, the per-device error word and CUDA error
+// bookkeeping shared by every entry point.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace davet {
+
+namespace {
+__device__ unsigned g_error_word;
+
+thread_local int t_last_cuda_error = 0;
+
+constexpr int kMaxDevices = 64;
+unsigned* g_word_addr[kMaxDevices] = {};
+std::mutex g_word_mu;
+}  // namespace
+
+davet_status cuda_fail(cudaError_t e) {
+  t_last_cuda_error = static_cast<int>(e);
+  return DAVET_ERR_CUDA;
+}
+
+davet_status check_launch() {
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
+}
+
+unsigned* device_error_word() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    cuda_fail(e);
+    return nullptr;
+  }
+  if (dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> g(g_word_mu);
+  if (!g_word_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_error_word);
+    if (e != cudaSuccess) {
+      cuda_fail(e);
+      return nullptr;
+    }
+    g_word_addr[dev] = static_cast<unsigned*>(p);
+  }
+  return g_word_addr[dev];
+}
+
+}  // namespace davet
+
+extern "C" int davet_version(void) { return 100; }
+
+extern "C" const char* davet_status_string(int status) {
+  switch (status) {
+    case DAVET_OK: return "ok";
+    case DAVET_ERR_INVALID_ARG: return "invalid argument";
+    case DAVET_ERR_UNSUPPORTED: return "unsupported shape or size";
+    case DAVET_ERR_CUDA: return "CUDA error";
+    case DAVET_ERR_TIMEOUT: return "device wait timed out";
+    case DAVET_ERR_DEVICE: return "device-side check failed";
+    default: return "unknown status";
+  }
+}
+
+extern "C" int davet_last_cuda_error(void) { return davet::t_last_cuda_error; }
+
+extern "C" davet_status davet_device_status(unsigned* flags, int clear) {
+  using namespace davet;
+  if (device_error_word() == nullptr) return DAVET_ERR_CUDA;
+  unsigned w = 0;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaMemcpyFromSymbol(&w, g_error_word, sizeof w);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (clear) {
+    const unsigned zero = 0;
+    e = cudaMemcpyToSymbol(g_error_word, &zero, sizeof zero);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  if (flags) *flags = w;
+  if (w & DEV_ERR_TIMEOUT) return DAVET_ERR_TIMEOUT;
+  if (w) return DAVET_ERR_DEVICE;
+  return DAVET_OK;
+}

@@ -1,0 +1,168 @@
+"""Thin ctypes binding of libdavet.so (C ABI in include/davet.h).
+
+Argument marshalling only: each function takes torch tensors (or raw
+integer device pointers), passes their data pointers and sizes to the C
+entry point of the same name, and raises DavetError on a non-OK status.
+Every step of the computation runs in the library's CUDA kernels; there is no
+Python or CPU fallback, and loading fails loudly when the library is
+missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libdavet.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_TIMEOUT, ERR_DEVICE = range(6)
+DEV_TIMEOUT, DEV_CAPACITY, DEV_ARG = 0x1, 0x2, 0x4
+
+_lock = threading.Lock()
+_lib = None
+
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_i64 = ctypes.c_int64
+_int = ctypes.c_int
+_f32 = ctypes.c_float
+_sz = ctypes.c_size_t
+
+
+class DavetError(RuntimeError):
+    def __init__(self, fn: str, status: int, lib=None):
+        msg = lib.davet_status_string(status).decode() if lib is not None else str(status)
+        detail = ""
+        if status == ERR_CUDA and lib is not None:
+            detail = f" (cudaError {lib.davet_last_cuda_error()})"
+        super().__init__(f"{fn} failed: {msg}{detail}")
+        self.status = status
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _declare(lib):
+    sig = {
+        "davet_version": (_int, []),
+        "davet_status_string": (ctypes.c_char_p, [_int]),
+        "davet_last_cuda_error": (_int, []),
+        "davet_device_status": (_int, [ctypes.POINTER(ctypes.c_uint), _int]),
+        "davet_pyramid_layout": (_int, [_int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_i64)]),
+        "davet_build_pyramid": (_int, [_vp, _vp, _int, _int, _int, _int, _vp, _vp]),
+        "davet_gather_view": (_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _vp, _vp,
+                                     _i64, _vp]),
+        "davet_step_attention": (_int, [_vp, _vp, _int, _i64, _int, _int, _f32, _vp, _vp]),
+        "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
+        "davet_unmask_topk": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                     _vp]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+class Davet:
+    """The loaded library; methods mirror the C entry points."""
+
+    def __init__(self, lib):
+        self.lib = lib
+
+    def _check(self, fn, status):
+        if status != OK:
+            raise DavetError(fn, status, self.lib)
+
+    # ------------------------------------------------------------ utilities
+    def davet_version(self) -> int:
+        return int(self.lib.davet_version())
+
+    def davet_status_string(self, status: int) -> str:
+        return self.lib.davet_status_string(status).decode()
+
+    def davet_device_status(self, clear: bool = True) -> tuple[int, int]:
+        """(status, flags) of the device error word; synchronizes the device."""
+        flags = ctypes.c_uint(0)
+        st = self.lib.davet_device_status(ctypes.byref(flags), 1 if clear else 0)
+        return int(st), int(flags.value)
+
+    def davet_pyramid_layout(self, grid: int, n_levels: int, n_tiles: int):
+        side = (_int * n_levels)()
+        off = (_i64 * (n_levels + 1))()
+        self._check("davet_pyramid_layout", self.lib.davet_pyramid_layout(grid, n_levels, n_tiles, side, off))
+        return list(side), list(off)
+
+    # ---------------------------------------------------------------- path
+    def davet_build_pyramid(self, feat, pyr, n_tiles: int, grid: int, n_levels: int, C: int, pyr_f32=None,
+                            stream=None):
+        self._check("davet_build_pyramid",
+                    self.lib.davet_build_pyramid(_ptr(feat), _ptr(pyr), n_tiles, grid, n_levels, C, _ptr(pyr_f32),
+                                                 _stream(stream)))
+
+    def davet_gather_view(self, pyr_ptrs, tiles, text, text_off, prompt_len, resp_len, level, batch: int,
+                          grid: int, n_levels: int, C: int, packed, cu_seqlens, max_total_rows: int, stream=None):
+        self._check("davet_gather_view",
+                    self.lib.davet_gather_view(_ptr(pyr_ptrs), _ptr(tiles), _ptr(text), _ptr(text_off),
+                                               _ptr(prompt_len), _ptr(resp_len), _ptr(level), batch, grid,
+                                               n_levels, C, _ptr(packed), _ptr(cu_seqlens), max_total_rows,
+                                               _stream(stream)))
+
+    def davet_step_attention(self, qkv, cu_seqlens, batch: int, max_total_rows: int, H: int, D: int,
+                             scale: float, out, stream=None):
+        self._check("davet_step_attention",
+                    self.lib.davet_step_attention(_ptr(qkv), _ptr(cu_seqlens), batch, max_total_rows, H, D,
+                                                  float(scale), _ptr(out), _stream(stream)))
+
+    def davet_unmask_topk_workspace(self, total_rows: int, V: int, batch: int) -> int:
+        n = _sz(0)
+        self._check("davet_unmask_topk_workspace",
+                    self.lib.davet_unmask_topk_workspace(total_rows, V, batch, ctypes.byref(n)))
+        return int(n.value)
+
+    def davet_unmask_topk(self, logits, V: int, cu_resp, batch: int, total_rows: int, k: int, masked, tokens,
+                          argmax=None, conf=None, committed=None, stats=None, workspace=None,
+                          workspace_bytes: int = 0, stream=None):
+        if workspace is not None and not isinstance(workspace, int) and workspace_bytes == 0:
+            workspace_bytes = workspace.numel() * workspace.element_size()
+        self._check("davet_unmask_topk",
+                    self.lib.davet_unmask_topk(_ptr(logits), V, _ptr(cu_resp), batch, total_rows, k, _ptr(masked),
+                                               _ptr(tokens), _ptr(argmax), _ptr(conf), _ptr(committed),
+                                               _ptr(stats), _ptr(workspace), workspace_bytes, _stream(stream)))
+
+
+_handle = None
+
+
+def load_cdll(path: str = LIB_PATH):
+    """Load the shared library without touching a GPU (symbol checks)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise RuntimeError(f"libdavet.so not found at {path}: run paper_2608_01821_gb300.build() first "
+                                   "(the CUDA library is required; there is no fallback)")
+            _lib = _declare(ctypes.CDLL(path))
+    return _lib
+
+
+def load() -> Davet:
+    global _handle
+    if _handle is None:
+        _handle = Davet(load_cdll())
+    return _handle

@@ -1,0 +1,93 @@
+"""Host-side checks of the C ABI library that need no GPU: it builds for
+sm_103a, loads, exports every entry point declared in include/davet.h, and
+rejects invalid arguments with a status code before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import paper_2608_01821_gb300 as pkg
+    pkg.build()
+    from paper_2608_01821_gb300 import davet
+    return davet.load_cdll()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "davet.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(davet_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert "davet_build_pyramid" in names and "davet_unmask_topk" in names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_and_version(lib):
+    for code in range(6):
+        assert lib.davet_status_string(code)
+    assert lib.davet_status_string(99) == b"unknown status"
+    assert lib.davet_version() >= 100
+
+
+@pytest.mark.parametrize("grid,levels,tiles", [(27, 4, 1), (27, 4, 10), (12, 3, 1), (5, 5, 3), (1, 1, 2)])
+def test_pyramid_layout_matches_oracle(lib, grid, levels, tiles):
+    side = (ctypes.c_int * levels)()
+    off = (ctypes.c_int64 * (levels + 1))()
+    assert lib.davet_pyramid_layout(grid, levels, tiles, side, off) == 0
+    assert list(side) == oracle.level_sides(grid, levels)
+    assert list(off) == oracle.level_offsets(grid, levels, tiles)
+
+
+def test_invalid_arguments_are_rejected_without_a_device(lib):
+    INV, UNS = 1, 2
+    p = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
+    null = None
+    assert lib.davet_pyramid_layout(0, 4, 1, None, None) == INV
+    assert lib.davet_pyramid_layout(27, 6, 1, None, None) == INV
+    # pyramid: C not a multiple of 8, null pointers, misalignment, too many levels
+    assert lib.davet_build_pyramid(p, p, 1, 27, 4, 12, null, null) == INV
+    assert lib.davet_build_pyramid(null, p, 1, 27, 4, 16, null, null) == INV
+    assert lib.davet_build_pyramid(ctypes.c_void_p((1 << 20) + 2), p, 1, 27, 4, 16, null, null) == INV
+    assert lib.davet_build_pyramid(p, p, 1, 27, 6, 16, null, null) == UNS
+    assert lib.davet_build_pyramid(p, p, 0, 27, 4, 16, null, null) == 0  # no tiles: no-op
+    # attention: unsupported head dim, bad scale, null pointers
+    f = ctypes.c_float
+    assert lib.davet_step_attention(p, p, 1, 128, 4, 96, f(0.1), p, null) == UNS
+    assert lib.davet_step_attention(p, p, 1, 128, 4, 64, f(0.0), p, null) == INV
+    assert lib.davet_step_attention(null, p, 1, 128, 4, 64, f(0.1), p, null) == INV
+    assert lib.davet_step_attention(p, p, 2000, 128, 4, 64, f(0.1), p, null) == UNS
+    assert lib.davet_step_attention(p, p, 0, 128, 4, 64, f(0.1), p, null) == 0  # empty batch
+    # gather: bad levels count, batch too large
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 16, p, p, 100, null) == INV
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 16, p, p, 100, null) == UNS
+    # unmask: k out of range, V not a multiple of 8, workspace too small
+    n = ctypes.c_size_t(0)
+    assert lib.davet_unmask_topk_workspace(128, 1000, 1, ctypes.byref(n)) == 0 and n.value > 0
+    ws_needed = n.value
+    assert lib.davet_unmask_topk(p, 1000, p, 1, 128, 0, p, p, null, null, null, null, p, ws_needed, null) == INV
+    assert lib.davet_unmask_topk(p, 1001, p, 1, 128, 2, p, p, null, null, null, null, p, ws_needed, null) == INV
+    assert lib.davet_unmask_topk(p, 1000, p, 1, 128, 2, p, p, null, null, null, null, p, ws_needed - 1,
+                                 null) == INV
+    assert lib.davet_unmask_topk(p, 1000, p, 0, 128, 2, p, p, null, null, null, null, p, ws_needed, null) == 0
+
+
+def test_package_fails_loudly_without_library(tmp_path):
+    from paper_2608_01821_gb300 import davet
+    saved = davet._lib
+    davet._lib = None
+    try:
+        with pytest.raises(RuntimeError, match="no fallback"):
+            davet.load_cdll(str(tmp_path / "missing.so"))
+    finally:
+        davet._lib = saved

@@ -1,0 +1,126 @@
+"""Parity of davet_step_attention (Sec. 3.1, Eq. 1) with the fp64 oracle.
+
+Tolerance for bf16 inputs: max |gpu - oracle| <= 1e-2 and relative L2 error
+<= 5e-3 over the compared outputs.  Cases span one and many 128-row tiles,
+ragged tails, empty and one-row requests, both head dimensions, garbage
+(non-finite) rows past the last request, and the full packed shapes of the
+8B-class workloads, checked on sampled (row, head) pairs.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import ATTN_MAX_ABS, ATTN_REL_L2, attn_errors, bf16_to_f64
+from paper_2608_01821_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def run(davet, qkv_cpu, cu, H, D, max_rows=None, garbage_tail=False):
+    dev = torch.device("cuda")
+    N = qkv_cpu.shape[0]
+    max_rows = max_rows or N
+    qkv = torch.empty((max_rows, 3, H, D), dtype=torch.bfloat16, device=dev)
+    qkv[:N].copy_(qkv_cpu)
+    if garbage_tail and max_rows > N:
+        qkv[N:].view(torch.int16).fill_(0x7FC0)  # bf16 NaN
+    out = torch.full((max_rows, H, D), 3.0, dtype=torch.bfloat16, device=dev)
+    cu_d = torch.tensor(cu, dtype=torch.int32, device=dev)
+    davet.davet_step_attention(qkv, cu_d, len(cu) - 1, max_rows, H, D, 1.0 / math.sqrt(D), out)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    return out
+
+
+@pytest.mark.parametrize("lens,H,D", [
+    ([192], 4, 64),            # tiny workload shape
+    ([1], 2, 128),
+    ([127], 2, 128),
+    ([128], 2, 128),
+    ([129], 2, 128),
+    ([300, 0, 5, 257], 3, 128),
+    ([513, 64], 2, 64),
+    ([1000], 1, 128),
+])
+def test_dense_parity(davet, lens, H, D):
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    qkv = workloads.qkv_rows(N, H, D, seed=sum(lens) + H + D)
+    out = run(davet, qkv, cu, H, D)
+    ref = oracle.attention(qkv, cu, H, D, 1.0 / math.sqrt(D))
+    got = bf16_to_f64(out[:N])
+    assert np.isfinite(got).all()
+    max_abs, rel = attn_errors(got, ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
+
+
+def test_rows_past_the_last_request_do_not_leak(davet):
+    H, D = 2, 128
+    lens = [200, 77]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    qkv = workloads.qkv_rows(N, H, D, seed=5)
+    out = run(davet, qkv, cu, H, D, max_rows=N + 300, garbage_tail=True)
+    ref = oracle.attention(qkv, cu, H, D, 1.0 / math.sqrt(D))
+    got = bf16_to_f64(out[:N])
+    assert np.isfinite(got).all()
+    max_abs, rel = attn_errors(got, ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2
+    # rows past cu[batch] are not written
+    assert (out[N:].float() == 3.0).all()
+
+
+def test_identical_keys_give_mean_of_values(davet):
+    H, D, L = 2, 128, 333
+    qkv = workloads.qkv_rows(L, H, D, seed=6)
+    qkv[:, 1] = qkv[0:1, 1]
+    out = run(davet, qkv, [0, L], H, D)
+    mean_v = bf16_to_f64(qkv[:, 2]).mean(axis=0)
+    got = bf16_to_f64(out)
+    assert np.abs(got - mean_v[None]).max() <= ATTN_MAX_ABS
+
+
+def test_growing_scores_force_the_rescale_path(davet):
+    # key norms grow along the sequence, so later key tiles carry maxima far
+    # above the first tile's (by much more than 2^8 in the log2 domain) and
+    # the running max must be raised and O rescaled; values are halved to
+    # keep outputs within the range where the absolute bound is meaningful
+    H, D, L = 2, 64, 700
+    qkv = workloads.qkv_rows(L, H, D, seed=7)
+    grow = torch.linspace(0.5, 5.5, L).view(L, 1, 1)
+    qkv[:, 0] = (qkv[:, 0].float() * 2).to(torch.bfloat16)
+    qkv[:, 1] = (qkv[:, 1].float() * grow).to(torch.bfloat16)
+    qkv[:, 2] = (qkv[:, 2].float() * 0.5).to(torch.bfloat16)
+    cu = np.array([0, L], np.int32)
+    out = run(davet, qkv, cu, H, D)
+    ref = oracle.attention(qkv, cu, H, D, 1.0 / math.sqrt(D))
+    max_abs, rel = attn_errors(bf16_to_f64(out), ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
+
+
+@pytest.mark.parametrize("name", ["single", "anyres", "highres", "ragged"])
+def test_full_size_sampled(davet, name):
+    """The packed step shapes of each workload at level 0 (the longest
+    sequences) and at its coarsest scheduled level; 64 sampled (row, head)
+    outputs per request are compared with the oracle."""
+    w = workloads.make(name)
+    rng = np.random.default_rng(hash(name) % 1000)
+    for level in sorted({0, int(w.schedule.max())}):
+        lens = [w.seq_len(b, level) for b in range(w.batch)]
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        N = int(cu[-1])
+        qkv = workloads.qkv_rows(N, w.H, w.D, seed=w.seed * 10 + level)
+        out = run(davet, qkv, cu, w.H, w.D, max_rows=w.max_total_rows())
+        rows, heads = [], []
+        for b in range(w.batch):
+            rows += list(rng.integers(cu[b], cu[b + 1], size=64))
+            heads += list(rng.integers(0, w.H, size=64))
+        rows = np.array(rows, np.int64)
+        heads = np.array(heads, np.int32)
+        ref = oracle.attention_rows(qkv, cu, w.H, w.D, w.scale, rows, heads)
+        got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
+        max_abs, rel = attn_errors(got, ref)
+        assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (name, level, max_abs, rel)
