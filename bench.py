@@ -128,6 +128,8 @@ def run_ours(args, rank, world, local_rank):
     # step logits: a pool of distinct device buffers, step t uses t % P
     logit_bytes = w.total_resp * w.V * 2
     P = max(2, min(w.T, int((16 << 30) // max(logit_bytes, 1))))
+    if args.logit_pool:
+        P = max(1, min(P, args.logit_pool))
     pool = torch.empty((P, w.total_resp, w.V), dtype=torch.bfloat16, device=dev)
     for i in range(P):
         workloads.logits_device(w, i, dev, out=pool[i])
@@ -185,7 +187,7 @@ def run_ours(args, rank, world, local_rank):
     comp = kernel_times(pl, w, pool, P, stream)
 
     # ---------------------------------------------------------- e2e
-    e2e = run_e2e(args, pl, w, dev, stream, world)
+    e2e = None if args.no_e2e else run_e2e(args, pl, w, dev, stream, world)
 
     out = None
     if rank == 0:
@@ -226,7 +228,8 @@ def run_ours(args, rank, world, local_rank):
                 "logit_pool": P,
             },
             "components": {
-                k: {kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in v.items()}
+                k: ({kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in v.items()}
+                    if isinstance(v, dict) else v)
                 for k, v in comp.items()
             },
             "roofline": {
@@ -248,37 +251,73 @@ def run_ours(args, rank, world, local_rank):
     return out
 
 
-def kernel_times(pl, w, pool, P, stream):
-    """Average device time per call of each kernel over one eager pass."""
+def kernel_times(pl, w, pool, P, stream, reps=3):
+    """Average device time per call of each kernel.
+
+    The pass is captured once more into a CUDA graph with an event record
+    node before and after every library call, so each interval is the
+    kernel(s) of that call plus graph scheduling, without host launch
+    overhead; the graph is replayed `reps` times and the intervals summed.
+    Falls back to eager events when the event type cannot be captured."""
     import torch
-    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    rec = {"pyramid": [], "gather": [], "attention": [], "unmask": []}
-    with torch.cuda.stream(stream):
-        pl.reset_state()
-        a, b = ev(), ev()
+
+    def mk():
+        try:
+            return torch.cuda.Event(enable_timing=True, external=True)
+        except TypeError:
+            return None
+
+    probe = mk()
+    calls = []  # (kind, start, end)
+    ev = []
+
+    def timed(kind, fn):
+        a, b = mk(), mk()
         a.record(stream)
-        pl.build_pyramids()
+        fn()
         b.record(stream)
-        rec["pyramid"].append((a, b))
+        calls.append((kind, a, b))
+
+    def instrumented_pass():
+        pl.reset_state()
+        timed("pyramid", pl.build_pyramids)
         for t in range(w.T):
-            e = [ev() for _ in range(4)]
-            e[0].record(stream)
-            pl.gather(t)
-            e[1].record(stream)
-            pl.attention()
-            e[2].record(stream)
-            pl.unmask(t, pool[t % P])
-            e[3].record(stream)
-            rec["gather"].append((e[0], e[1]))
-            rec["attention"].append((e[1], e[2]))
-            rec["unmask"].append((e[2], e[3]))
-    torch.cuda.synchronize()
-    ms = {k: sum(x.elapsed_time(y) for x, y in v) for k, v in rec.items()}
+            timed("gather", lambda t=t: pl.gather(t))
+            timed("attention", pl.attention)
+            timed("unmask", lambda t=t: pl.unmask(t, pool[t % P]))
+
+    totals = {"pyramid": 0.0, "gather": 0.0, "attention": 0.0, "unmask": 0.0}
+    mode = "graph"
+    if probe is not None:
+        try:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                instrumented_pass()
+            for _ in range(reps):
+                g.replay()
+                torch.cuda.synchronize()
+                for kind, a, b in calls:
+                    totals[kind] += a.elapsed_time(b) / reps
+        except Exception:
+            probe = None
+            totals = {k: 0.0 for k in totals}
+            calls.clear()
+    if probe is None:
+        mode = "eager"
+        with torch.cuda.stream(stream):
+            def mk():  # noqa: F811
+                return torch.cuda.Event(enable_timing=True)
+            instrumented_pass()
+        torch.cuda.synchronize()
+        for kind, a, b in calls:
+            totals[kind] += a.elapsed_time(b)
+    ms = totals
     flops = sum(w.attention_flops(t) for t in range(w.T))
     gbytes = sum(w.gather_bytes(t) for t in range(w.T))
     ubytes = sum(w.unmask_bytes(t) for t in range(w.T))
     pbytes = w.pyramid_bytes()
     return {
+        "timing_mode": mode,
         "pyramid": {"launches": w.batch, "ms": ms["pyramid"], "bytes": pbytes,
                     "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9},
         "gather": {"launches": w.T, "ms": ms["gather"], "bytes": gbytes,
@@ -473,6 +512,32 @@ def run_reference(args, rank, world):
                     "d2h_bytes_per_step": 0}}
 
 
+def run_profile(args):
+    """Minimal launch sequence for profilers: the workload's inputs for one
+    step and `--steps` launches of one kernel (after `--warmup` launches)."""
+    import torch
+
+    from paper_2608_01821_gb300 import davet, workloads
+    from paper_2608_01821_gb300.pipeline import Pipeline
+    dev = torch.device("cuda", 0)
+    lib = davet.load()
+    w = workloads.make(args.config)
+    pl = Pipeline(w, dev, lib)
+    pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w))
+    t = args.profile_step
+    lg = workloads.logits_device(w, t, dev)
+    pl.build_pyramids()
+    pl.gather(t)
+    fn = {"pyramid": pl.build_pyramids, "gather": lambda: pl.gather(t), "attention": pl.attention,
+          "unmask": lambda: (pl.reset_state(), pl.unmask(t, lg))}[args.profile]
+    for _ in range(args.warmup + args.steps):
+        fn()
+    torch.cuda.synchronize()
+    st, flags = lib.davet_device_status()
+    print(json.dumps({"profile": args.profile, "workload": w.name, "step": t, "status": st, "flags": flags}))
+    return 0 if st == 0 else 1
+
+
 # ------------------------------------------------------------ dist glue
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -516,8 +581,15 @@ def main(argv=None):
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--logit-pool", type=int, default=0, help="cap on distinct device logit buffers")
+    ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "unmask"], default=None,
+                    help="only set up one step and launch this kernel --steps times (for ncu captures)")
+    ap.add_argument("--profile-step", type=int, default=0)
     args = ap.parse_args(argv)
     rank, world, local = dist_env()
+    if args.profile:
+        return run_profile(args)
     if args.impl == "reference":
         out = run_reference(args, rank, world)
         if out is not None:

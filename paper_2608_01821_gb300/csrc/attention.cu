@@ -1,25 +1,28 @@
 // attention.cu -- bidirectional varlen multi-head attention of one denoising
 // step (Sec. 3.1, Eq. 1), on the sm_103a tensor cores.
 //
-// Design (one persistent CTA per SM, 192 threads, warp-specialized):
-//   warp 4       TMA producer: the Q tile once per work item, then K and V
-//                tiles (128 keys x D) into a 2-stage ring, 128-byte swizzled.
-//   warp 5       MMA issuer and TMEM owner: S = Q K^T into one of two TMEM
-//                S buffers (128 x 128 fp32), then O += P V into the TMEM O
-//                accumulator (128 x D fp32).  QK of tile j+1 is issued before
-//                PV of tile j so the tensor cores run while softmax works.
-//   warps 0-3    softmax + epilogue: thread r owns query row r of the tile;
-//                reads its S row from TMEM, keeps the running max in the
-//                log2 domain, writes P (bf16) to shared memory in the
-//                swizzled K-major layout the MMA reads, rescales O in TMEM
-//                only when the max grows by more than 2^8 (the result is
-//                unchanged: O and the row sum carry the same stale max), and
-//                finally normalizes O and stores it as bf16.
-// Work items are (request, head, 128-row query tile); items are ordered
-// longest request first and, within a request, head-major so that CTAs
-// running together share a head's K/V in L2.  Keys past the end of a request
-// are masked to -inf and their V rows zeroed in shared memory, so tiles may
-// straddle request boundaries and the end of the buffer.
+// One persistent CTA per SM (320 threads, warp-specialized).  A work item is
+// (request, head, block of up to two 128-row query tiles A and B):
+//   warp 8       TMA producer: Q_A and Q_B once per item, then K and V tiles
+//                of 128 keys into a 2-stage ring (128-byte swizzle).
+//   warp 9       MMA issuer and TMEM owner.  Per key tile j it issues
+//                PV_A(j), S_A(j+1), PV_B(j), S_B(j+1), so the tensor pipe
+//                works on one tile while the softmax of the other runs.
+//   warps 0-3    softmax of tile A, warps 4-7 softmax of tile B: thread r
+//                owns query row r; it reads its S row (fp32) from TMEM,
+//                keeps the running max in the log2 domain, writes
+//                P = 2^(s*c - m) as bf16 back into the first half of its S
+//                columns (the PV MMA reads A from TMEM), rescales its O row
+//                only when the max grows by more than 2^8 (O and the row sum
+//                keep the same stale max, so the result is unchanged) and,
+//                after the last key tile, normalizes O and stores it as bf16.
+// TMEM: S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
+// Items are ordered longest request first and, within a request,
+// head-major, so CTAs running together share a head's K/V in L2.  Keys past
+// the end of a request are masked to -inf and their V rows zeroed in shared
+// memory, so key tiles may straddle request boundaries and the buffer end.
+// With few items (short sequences) the host selects one query tile per item
+// so that more SMs get work.
 #include <algorithm>
 #include <cstdio>
 #include <mutex>
@@ -30,25 +33,28 @@ namespace davet {
 namespace attn {
 
 constexpr int BM = 128;          // query rows per tile (MMA M)
-constexpr int BN = 128;          // keys per tile (MMA N of QK^T, K of PV)
+constexpr int BN = 128;          // keys per tile (N of S = Q K^T, K of O += P V)
 constexpr int NS = 2;            // K/V pipeline stages
-constexpr int kThreads = 192;    // 4 softmax warps + TMA warp + MMA warp
+constexpr int kThreads = 320;    // 2 softmax warpgroups + TMA warp + MMA warp
+constexpr int kWarpTma = 8, kWarpMma = 9;
 constexpr int kMaxBatch = 1024;  // requests per call
-constexpr int kLptMaxBatch = 128;
+constexpr int kLptMaxBatch = 256;
 constexpr int kChunkBytes = 128 * 128;  // 128 rows x 128 B (64 bf16) swizzled chunk
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+__host__ __device__ constexpr uint32_t col_s(int t) { return t * 128u; }
+__host__ __device__ constexpr uint32_t col_o(int t) { return 256u + t * 128u; }
 
 template <int D>
 struct Smem {
   static constexpr int KC = D / 64;
-  alignas(1024) uint8_t q[KC][kChunkBytes];
+  alignas(1024) uint8_t q[2][KC][kChunkBytes];
   alignas(1024) uint8_t k[NS][KC][kChunkBytes];
   alignas(1024) uint8_t v[NS][KC][kChunkBytes];
-  alignas(1024) uint8_t p[2][kChunkBytes];  // keys 0-63 | 64-127
-  uint64_t q_full, q_empty, p_full, o_done, fin;
-  uint64_t k_full[NS], v_full[NS], kv_empty[NS], s_full[2];
+  uint64_t q_full, q_empty, fin;
+  uint64_t k_full[NS], v_full[NS], kv_empty[NS];
+  uint64_t s_full[2], p_full[2], o_full[2];
   uint32_t tmem;
   int abort;
   int n_req;   // requests with at least one row
@@ -64,13 +70,14 @@ struct Params {
   int batch;
   int H;
   int max_rows;
+  int qtiles;  // query tiles per work item (1 or 2)
   float scale_log2;
   uint16_t* out;
   unsigned* err;
 };
 
 struct Item {
-  int start, len, qt, h, nkv;
+  int start, len, q0, h, nkv, ntile;  // q0: first query row of the item within the request
 };
 
 // Coordinate along the tensor map's second dimension: slot (0 = query,
@@ -78,7 +85,7 @@ struct Item {
 __device__ __forceinline__ int h_coord(int slot, int h, int H) { return slot * H + h; }
 
 template <int D>
-__device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H) {
+__device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H, int qtiles) {
   // largest i with cum[i] <= item
   int lo = 0, hi = s.n_req - 1;
   while (lo < hi) {
@@ -88,13 +95,15 @@ __device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H) {
   const int b = s.order[lo];
   const int local = item - s.cum[lo];
   const int len = s.req_len[b];
-  const int nq = (len + BM - 1) / BM;
+  const int rows_per_item = BM * qtiles;
+  const int nq = (len + rows_per_item - 1) / rows_per_item;
   Item it;
   it.start = s.req_start[b];
   it.len = len;
   it.h = local / nq;
-  it.qt = local - it.h * nq;
+  it.q0 = (local - it.h * nq) * rows_per_item;
   it.nkv = (len + BN - 1) / BN;
+  it.ntile = (qtiles == 2 && it.q0 + BM < len) ? 2 : 1;
   return it;
 }
 
@@ -115,6 +124,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = tid >> 5;
   const int lane = tid & 31;
   const int H = prm.H;
+  const int qtiles = prm.qtiles;
 
   // ---------------------------------------------------------- schedule
   if (tid == 0) {
@@ -154,9 +164,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (tid == 0) {
     int acc = 0;
+    const int rows_per_item = BM * qtiles;
     for (int i = 0; i < s.n_req; ++i) {
       s.cum[i] = acc;
-      acc += ((s.req_len[s.order[i]] + BM - 1) / BM) * H;
+      acc += ((s.req_len[s.order[i]] + rows_per_item - 1) / rows_per_item) * H;
     }
     s.cum[s.n_req] = acc;
     s.n_items = acc;
@@ -168,19 +179,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     mbar_init(&s.q_full, 1);
     mbar_init(&s.q_empty, 1);
-    mbar_init(&s.p_full, 128);
-    mbar_init(&s.o_done, 1);
     mbar_init(&s.fin, 1);
     for (int i = 0; i < NS; ++i) {
       mbar_init(&s.k_full[i], 1);
       mbar_init(&s.v_full[i], 1);
       mbar_init(&s.kv_empty[i], 1);
     }
-    mbar_init(&s.s_full[0], 1);
-    mbar_init(&s.s_full[1], 1);
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(&s.s_full[t], 1);
+      mbar_init(&s.p_full[t], 128);
+      mbar_init(&s.o_full[t], 1);
+    }
     fence_mbar_init();
   }
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     tmem_alloc(&s.tmem, kTmemCols);
     tmem_relinquish();
   }
@@ -190,18 +202,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = s.tmem;
   volatile int* abort_flag = &s.abort;
 
-  if (warp == 4) {
+  if (warp == kWarpTma) {
     // ------------------------------------------------------ TMA producer
     if (lane == 0) {
       tma_prefetch_desc(&tmap);
       uint32_t it = 0, wi = 0;
       bool ok = true;
       for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
-        const Item w = decode(s, item, H);
+        const Item w = decode(s, item, H, qtiles);
         if (wi > 0) ok = mbar_wait(&s.q_empty, (wi - 1) & 1, prm.err, abort_flag);
         if (!ok) break;
-        mbar_arrive_expect_tx(&s.q_full, KC * kChunkBytes);
-        for (int c = 0; c < KC; ++c) tma_load_3d(s.q[c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), w.start + w.qt * BM);
+        mbar_arrive_expect_tx(&s.q_full, w.ntile * KC * kChunkBytes);
+        for (int t = 0; t < w.ntile; ++t)
+          for (int c = 0; c < KC; ++c)
+            tma_load_3d(s.q[t][c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), w.start + w.q0 + t * BM);
         for (int j = 0; j < w.nkv; ++j, ++it) {
           const int st = it % NS;
           if (it >= NS) ok = mbar_wait(&s.kv_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
@@ -221,74 +235,93 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kWarpMma) {
     // --------------------------------------------------------- MMA issuer
     constexpr uint32_t kIdescQK = idesc_bf16_f32(BM, BN, false, false);
     constexpr uint32_t kIdescPV = idesc_bf16_f32(BM, D, false, true);
     uint32_t it = 0, wi = 0;
+    uint32_t np[2] = {0, 0};  // P tiles consumed per query tile
     bool ok = true;
 
-    auto issue_pv = [&](uint32_t i, bool first, int valid_keys) -> bool {
-      const int st = i % NS;
-      if (!warp_wait(&s.p_full, i & 1, prm.err, abort_flag)) return false;
-      if (!warp_wait(&s.v_full[st], (i / NS) & 1, prm.err, abort_flag)) return false;
-      tc_fence_after();
-      if (valid_keys < BN) {
-        // keys past the request end: zero their V rows (P is 0 there, but the
-        // rows may hold anything, including non-finite values)
-        for (int c = 0; c < KC; ++c) {
-          uint4* base = reinterpret_cast<uint4*>(s.v[st][c]);
-          for (int idx = valid_keys * 8 + lane; idx < BN * 8; idx += 32) base[idx] = make_uint4(0, 0, 0, 0);
+    // S_t = Q_t K^T for the K tile in stage st
+    auto issue_s = [&](int t, int st) {
+      if (lane == 0) {
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk & 3) * 32;
+          const uint64_t a = sw128_desc(smem_u32(s.q[t][kk >> 2]) + off, 16, 1024);
+          const uint64_t b = sw128_desc(smem_u32(s.k[st][kk >> 2]) + off, 16, 1024);
+          umma_ss(tmem + col_s(t), a, b, kIdescQK, kk > 0 ? 1u : 0u);
         }
-        fence_proxy_async_smem();
-        __syncwarp();
+        umma_commit(&s.s_full[t]);
       }
+      __syncwarp();
+    };
+    // O_t (+)= P_t V for the V tile in stage st, P read from TMEM
+    auto issue_pv = [&](int t, int st, bool first) {
       if (lane == 0) {
         const uint32_t v0 = smem_u32(s.v[st][0]);
 #pragma unroll
         for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t a = sw128_desc(smem_u32(s.p[kk >> 2]) + (kk & 3) * 32, 16, 1024);
           const uint64_t b = sw128_desc(v0 + kk * 2048, kChunkBytes, 1024);
-          umma_ss(tmem + kColO, a, b, kIdescPV, (first && kk == 0) ? 0u : 1u);
+          umma_ts(tmem + col_o(t), tmem + col_s(t) + kk * 8, b, kIdescPV, (first && kk == 0) ? 0u : 1u);
         }
-        umma_commit(&s.o_done);
-        umma_commit(&s.kv_empty[st]);
       }
       __syncwarp();
-      return true;
+    };
+    auto commit = [&](uint64_t* bar) {
+      if (lane == 0) umma_commit(bar);
+      __syncwarp();
     };
 
     for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
-      const Item w = decode(s, item, H);
+      const Item w = decode(s, item, H, qtiles);
       ok = warp_wait(&s.q_full, wi & 1, prm.err, abort_flag);
       if (!ok) break;
       tc_fence_after();
-      for (int j = 0; j < w.nkv; ++j, ++it) {
+      // prologue: S for key tile 0
+      ok = warp_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      for (int t = 0; t < w.ntile; ++t) issue_s(t, it % NS);
+      if (w.nkv == 1) commit(&s.q_empty);
+      for (int j = 0; ok && j < w.nkv; ++j, ++it) {
         const int st = it % NS;
-        const uint32_t sb = it & 1;
-        ok = warp_wait(&s.k_full[st], (it / NS) & 1, prm.err, abort_flag);
+        const int st1 = (it + 1) % NS;
+        const bool more = j + 1 < w.nkv;
+        ok = warp_wait(&s.v_full[st], (it / NS) & 1, prm.err, abort_flag);
         if (!ok) break;
-        tc_fence_after();
-        if (lane == 0) {
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk & 3) * 32;
-            const uint64_t a = sw128_desc(smem_u32(s.q[kk >> 2]) + off, 16, 1024);
-            const uint64_t b = sw128_desc(smem_u32(s.k[st][kk >> 2]) + off, 16, 1024);
-            umma_ss(tmem + (sb ? kColS1 : kColS0), a, b, kIdescQK, kk > 0 ? 1u : 0u);
+        const int valid_keys = min(BN, w.len - j * BN);
+        if (valid_keys < BN) {
+          // keys past the request end: zero their V rows (P is 0 there, but
+          // the rows may hold anything, including non-finite values)
+          for (int c = 0; c < KC; ++c) {
+            uint4* base = reinterpret_cast<uint4*>(s.v[st][c]);
+            for (int idx = valid_keys * 8 + lane; idx < BN * 8; idx += 32) base[idx] = make_uint4(0, 0, 0, 0);
           }
-          umma_commit(&s.s_full[sb]);
-          if (j == w.nkv - 1) umma_commit(&s.q_empty);
+          fence_proxy_async_smem();
+          __syncwarp();
         }
-        __syncwarp();
-        if (j > 0) {
-          ok = issue_pv(it - 1, j == 1, BN);
+        if (more) {
+          ok = warp_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
           if (!ok) break;
         }
+        for (int t = 0; t < w.ntile; ++t) {
+          ok = warp_wait(&s.p_full[t], np[t] & 1, prm.err, abort_flag);
+          if (!ok) break;
+          ++np[t];
+          tc_fence_after();
+          issue_pv(t, st, j == 0);
+          if (more) {
+            issue_s(t, st1);
+            if (j + 1 == w.nkv - 1 && t == w.ntile - 1) commit(&s.q_empty);
+          } else {
+            commit(&s.o_full[t]);
+          }
+        }
+        if (!ok) break;
+        commit(&s.kv_empty[st]);
       }
-      if (!ok) break;
-      const int last_valid = w.len - (w.nkv - 1) * BN;
-      ok = issue_pv(it - 1, w.nkv == 1, last_valid);
     }
     // wait until every issued MMA has completed before TMEM is released
     if (lane == 0) {
@@ -298,115 +331,109 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------- softmax + epilogue
-    const int r = tid;  // query row within the tile == TMEM lane
-    const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-    uint32_t it = 0;
+    const int t = warp >> 2;             // query tile of this warpgroup
+    const int r = tid & 127;             // query row within the tile == TMEM lane
+    const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_addr = tmem + lane_base + col_s(t);
+    const uint32_t o_addr = tmem + lane_base + col_o(t);
+    const float c = prm.scale_log2;
+    uint32_t ns = 0, no = 0;
     bool ok = true;
     for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x) {
-      const Item w = decode(s, item, H);
-      float m = -INFINITY;  // running max of scale*log2(e)*score
-      float l = 0.f;        // running sum of 2^(t - m)
-      for (int j = 0; j < w.nkv; ++j, ++it) {
-        const uint32_t sb = it & 1;
-        ok = warp_wait(&s.s_full[sb], (it >> 1) & 1, prm.err, abort_flag);
+      const Item w = decode(s, item, H, qtiles);
+      if (t >= w.ntile) continue;
+      float m = -INFINITY;  // running max of c * score (log2 domain)
+      float l = 0.f;        // running sum of 2^(c*score - m)
+      for (int j = 0; j < w.nkv; ++j, ++ns) {
+        ok = warp_wait(&s.s_full[t], ns & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        float t[BN];
+        float x[BN];
         {
           uint32_t raw[32];
 #pragma unroll
-          for (int c = 0; c < BN / 32; ++c) {
-            tmem_ld32(tmem + lane_base + (sb ? kColS1 : kColS0) + 32 * c, raw);
+          for (int q = 0; q < BN / 32; ++q) {
+            tmem_ld32(s_addr + 32 * q, raw);
             tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) t[32 * c + i] = __uint_as_float(raw[i]);
+            for (int i = 0; i < 32; ++i) x[32 * q + i] = __uint_as_float(raw[i]);
           }
         }
         const int valid = min(BN, w.len - j * BN);
-        float mt = -INFINITY;
+        if (valid < BN) {
 #pragma unroll
-        for (int i = 0; i < BN; ++i) {
-          t[i] = (i < valid) ? t[i] * prm.scale_log2 : -INFINITY;
-          mt = fmaxf(mt, t[i]);
+          for (int i = 0; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
         }
-        float m_new = m, factor = 1.f;
+        float mx = x[0];
+#pragma unroll
+        for (int i = 1; i < BN; ++i) mx = fmaxf(mx, x[i]);
+        const float mt = mx * c;
+        float factor = 1.f;
         bool need = false;
         if (j == 0) {
-          m_new = mt;
+          m = mt;
         } else if (mt > m + kRescaleThreshold) {
-          m_new = mt;
-          factor = ex2(m - m_new);
+          factor = ex2(m - mt);
+          m = mt;
           need = true;
         }
-        uint32_t pk[BN / 2];
+        const float neg_m = -m;
         float rs = 0.f;
 #pragma unroll
-        for (int i = 0; i < BN; i += 2) {
-          const float p0 = ex2(t[i] - m_new);
-          const float p1 = ex2(t[i + 1] - m_new);
-          rs += p0 + p1;
-          pk[i / 2] = pack_bf16x2(p0, p1);
+        for (int q = 0; q < BN / 32; ++q) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float p0 = ex2(fmaf(x[32 * q + 2 * i], c, neg_m));
+            const float p1 = ex2(fmaf(x[32 * q + 2 * i + 1], c, neg_m));
+            rs += p0 + p1;
+            pk[i] = pack_bf16x2(p0, p1);
+          }
+          tmem_st16(s_addr + 16 * q, pk);
+        }
+        // O is settled here (S of this tile was issued after the previous
+        // PV of this tile) and no MMA touches it before P is published
+        if (j > 0 && __any_sync(0xffffffffu, need)) {
+          uint32_t o[32];
+#pragma unroll 1
+          for (int q = 0; q < D / 32; ++q) {
+            tmem_ld32(o_addr + 32 * q, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+            tmem_st32(o_addr + 32 * q, o);
+          }
         }
         l = (j == 0) ? rs : l * factor + rs;
-        m = m_new;
-        if (j > 0) {
-          // PV of the previous tile done: P buffer free, O settled
-          ok = warp_wait(&s.o_done, (it - 1) & 1, prm.err, abort_flag);
-          if (!ok) break;
-          tc_fence_after();
-          if (__any_sync(0xffffffffu, need)) {
-            uint32_t o[32];
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-              tmem_ld32(tmem + lane_base + kColO + 32 * c, o);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
-              tmem_st32(tmem + lane_base + kColO + 32 * c, o);
-            }
-            tmem_wait_st();
-          }
-        }
-        // P row -> swizzled K-major tile: 16-byte piece q of row r lands at
-        // piece (q ^ (r & 7)) of the row's 128-byte line.
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          uint8_t* row = s.p[c] + r * 128;
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const int base = c * 32 + q * 4;
-            const uint4 val = make_uint4(pk[base], pk[base + 1], pk[base + 2], pk[base + 3]);
-            *reinterpret_cast<uint4*>(row + ((q ^ (r & 7)) << 4)) = val;
-          }
-        }
-        fence_proxy_async_smem();
+        tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(&s.p_full);
+        mbar_arrive(&s.p_full[t]);
       }
       if (!ok) break;
       // ------------------------------------------------------- epilogue
-      ok = warp_wait(&s.o_done, (it - 1) & 1, prm.err, abort_flag);
+      ok = warp_wait(&s.o_full[t], no & 1, prm.err, abort_flag);
+      ++no;
       if (!ok) break;
       tc_fence_after();
       const float inv_l = 1.f / l;
-      const int qrow = w.qt * BM + r;
+      const int qrow = w.q0 + t * BM + r;
       const bool row_ok = qrow < w.len;
       uint16_t* dst = prm.out + (static_cast<int64_t>(w.start + qrow) * H + w.h) * D;
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
+      for (int q = 0; q < D / 32; ++q) {
         uint32_t o[32];
-        tmem_ld32(tmem + lane_base + kColO + 32 * c, o);
+        tmem_ld32(o_addr + 32 * q, o);
         tmem_wait_ld();
         if (row_ok) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * c);
+          uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * q);
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
+          for (int u = 0; u < 4; ++u) {
             uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(o[8 * q + 0]) * inv_l, __uint_as_float(o[8 * q + 1]) * inv_l);
-            v.y = pack_bf16x2(__uint_as_float(o[8 * q + 2]) * inv_l, __uint_as_float(o[8 * q + 3]) * inv_l);
-            v.z = pack_bf16x2(__uint_as_float(o[8 * q + 4]) * inv_l, __uint_as_float(o[8 * q + 5]) * inv_l);
-            v.w = pack_bf16x2(__uint_as_float(o[8 * q + 6]) * inv_l, __uint_as_float(o[8 * q + 7]) * inv_l);
-            d4[q] = v;
+            v.x = pack_bf16x2(__uint_as_float(o[8 * u + 0]) * inv_l, __uint_as_float(o[8 * u + 1]) * inv_l);
+            v.y = pack_bf16x2(__uint_as_float(o[8 * u + 2]) * inv_l, __uint_as_float(o[8 * u + 3]) * inv_l);
+            v.z = pack_bf16x2(__uint_as_float(o[8 * u + 4]) * inv_l, __uint_as_float(o[8 * u + 5]) * inv_l);
+            v.w = pack_bf16x2(__uint_as_float(o[8 * u + 6]) * inv_l, __uint_as_float(o[8 * u + 7]) * inv_l);
+            d4[u] = v;
           }
         }
       }
@@ -417,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -496,6 +523,9 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   prm.batch = batch;
   prm.H = H;
   prm.max_rows = static_cast<int>(max_rows);
+  // two query tiles per item unless that leaves most SMs idle
+  const int64_t items2 = ((max_rows + 2 * attn::BM - 1) / (2 * attn::BM)) * static_cast<int64_t>(H);
+  prm.qtiles = items2 >= 2LL * g_dev[dev].sms ? 2 : 1;
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
   prm.out = static_cast<uint16_t*>(out);
   prm.err = err;
