@@ -192,8 +192,7 @@ def run_ours(args, rank, world, local_rank):
     out = None
     if rank == 0:
         peaks = measured_peaks()
-        steps_total = w.T * args.steps * world
-        value = steps_total / total_s
+        value = whole_job_rate(w.T * args.steps, world, total_s)
         launches_per_pass = w.batch + w.T * 4
         attn_flops_launch = comp["attention"]["flops"] / comp["attention"]["launches"]
         attn_ms = comp["attention"]["ms"] / comp["attention"]["launches"]
@@ -561,6 +560,11 @@ def barrier(world):
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
+
+
+def whole_job_rate(units_per_rank: float, world: int, max_seconds: float) -> float:
+    """Units processed by all ranks divided by the slowest rank's time."""
+    return units_per_rank * world / max_seconds
 
 
 def allreduce_max(x: float, world: int, device) -> float:
