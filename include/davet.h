@@ -22,9 +22,10 @@
  *    the layout given per function.  Tensor base pointers must be 16-byte
  *    aligned.
  *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
- *    call only enqueues work on that stream and returns without waiting; no
- *    call synchronizes the host, so calls can be captured in a CUDA graph
- *    once each entry point has run at least once on the device outside of a
+ *    call only enqueues work on that stream and returns without waiting.
+ *    davet_build_pyramid, davet_gather_view, davet_step_attention and
+ *    davet_unmask_topk never synchronize the host, so they can be captured in
+ *    a CUDA graph once each has run at least once on the device outside of a
  *    capture (the first call per device resolves a few device addresses).
  *  - Host-visible argument checks run before anything is enqueued and return
  *    DAVET_ERR_INVALID_ARG or DAVET_ERR_UNSUPPORTED.  A failed launch returns
@@ -213,6 +214,41 @@ davet_status davet_unmask_topk(const void* logits, int V, const int32_t* cu_resp
                                int64_t total_rows, int k, uint8_t* masked_dev, int32_t* tokens_dev,
                                int32_t* argmax_dev, float* conf_dev, int32_t* committed_dev, float* stats_dev,
                                void* workspace, size_t workspace_bytes, void* stream);
+
+/* Size of the scratch array that davet_unmask_topk_noalloc uses (per device). */
+#define DAVET_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/*
+ * davet_unmask_topk without a workspace argument.  The paper has no
+ * counterpart to this entry point; it exists for callers of this library
+ * that cannot allocate device memory of their own.  Examples are plugins that
+ * only receive the input and output buffers from a host engine which owns and
+ * budgets all device memory, and latency-critical serving loops that must not
+ * call cudaMalloc because it can synchronize the device and stall the
+ * pipeline.
+ *
+ * Computes exactly what davet_unmask_topk computes, with the same arguments
+ * except the workspace.  Instead of a caller workspace it uses one scratch
+ * array of DAVET_NOALLOC_SCRATCH_BYTES (1 MiB) that the library places in
+ * device global memory; every device that loads the library holds that array
+ * until the process exits.  The call allocates nothing.
+ *   - Limit: sizes whose workspace (davet_unmask_topk_workspace) exceeds
+ *     DAVET_NOALLOC_SCRATCH_BYTES are rejected with DAVET_ERR_UNSUPPORTED
+ *     before anything is enqueued (about 43,000 answer rows at V = 126464).
+ *   - Set-up: the first call on each device looks up the array's device
+ *     address (cudaGetSymbolAddress) with that device current and caches it;
+ *     make that first call before any stream capture.
+ *   - Sharing: every call on a device uses the same array, and the array keeps
+ *     whatever the last call left in it.  Nothing in it needs clearing: a call
+ *     writes every scratch entry it later reads.  Calls whose kernels overlap
+ *     on the GPU (for example, issued on two streams with no ordering between
+ *     them) race on the array and give wrong results; order them on one
+ *     stream or with events.
+ */
+davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t* cu_resp_dev, int batch,
+                                       int64_t total_rows, int k, uint8_t* masked_dev, int32_t* tokens_dev,
+                                       int32_t* argmax_dev, float* conf_dev, int32_t* committed_dev,
+                                       float* stats_dev, void* stream);
 
 #ifdef __cplusplus
 }

@@ -13,6 +13,7 @@
 //     of a block-wide arg-max and commits them.
 #include <algorithm>
 #include <climits>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -162,7 +163,7 @@ struct SelArgs {
   float* conf_out;
   int32_t* committed;
   float* stats;
-  float* row_conf;  // workspace: conf of masked rows, -1 once committed
+  float* row_conf;  // workspace: conf of masked rows
   int32_t* row_idx; // workspace: argmax of masked rows
   unsigned* err;
 };
@@ -334,5 +335,103 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
   a.err = err;
   select_commit<<<batch, kSelThreads, 0, st>>>(a);
+  return check_launch();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of davet_unmask_topk.
+//
+// Its scratch lives in a fixed device array owned by the library, so the
+// caller passes only inputs and outputs.  Every device that loads the library
+// keeps this array for the life of the process, and all calls on a device
+// share it.
+namespace davet {
+namespace unm {
+
+constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;  // DAVET_NOALLOC_SCRATCH_BYTES
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+static uint8_t* g_noalloc_addr[kNoAllocMaxDevices] = {};
+static std::mutex g_noalloc_mu;
+
+// Device address of g_noalloc_scratch on the current device.  Host code only
+// sees a host-side stand-in for the array under its name, so the address is
+// asked for once per device, with that device current, and cached.
+static uint8_t* noalloc_scratch(davet_status* st) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    *st = cuda_fail(e);
+    return nullptr;
+  }
+  if (dev < 0 || dev >= kNoAllocMaxDevices) {
+    *st = DAVET_ERR_UNSUPPORTED;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> g(g_noalloc_mu);
+  if (!g_noalloc_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) {
+      *st = cuda_fail(e);
+      return nullptr;
+    }
+    g_noalloc_addr[dev] = static_cast<uint8_t*>(p);
+  }
+  return g_noalloc_addr[dev];
+}
+
+}  // namespace unm
+}  // namespace davet
+
+extern "C" davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t* cu_resp_dev, int batch,
+                                                  int64_t total_rows, int k, uint8_t* masked_dev,
+                                                  int32_t* tokens_dev, int32_t* argmax_dev, float* conf_dev,
+                                                  int32_t* committed_dev, float* stats_dev, void* stream) {
+  using namespace davet;
+  using namespace davet::unm;
+  if (batch < 0 || total_rows < 0 || V < 8 || V % 8 != 0 || k < 1 || k > 1024) return DAVET_ERR_INVALID_ARG;
+  if (batch == 0) return DAVET_OK;
+  if (!cu_resp_dev || !masked_dev || !tokens_dev) return DAVET_ERR_INVALID_ARG;
+  if (total_rows > 0 && !logits) return DAVET_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(logits) & 15u) return DAVET_ERR_INVALID_ARG;
+  if (batch > 65535 || total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
+  const Layout L = layout_for(total_rows, V);
+  if (L.bytes > kNoAllocScratchBytes) return DAVET_ERR_UNSUPPORTED;  // too many answer rows for the array
+  davet_status st = DAVET_OK;
+  uint8_t* ws = noalloc_scratch(&st);
+  if (!ws) return st;
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // Nothing in the scratch needs clearing: the select kernel reads only the
+  // partials, confidences and argmaxes of masked rows, and the row pass of
+  // this same call writes all of them first.
+  Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
+  if (total_rows > 0) {
+    const long long items = total_rows * L.nsplit;
+    row_pass<<<static_cast<unsigned>(items), kRowThreads, 0, s>>>(static_cast<const uint4*>(logits), V / 8,
+                                                                  masked_dev, total_rows, L.nsplit, partial);
+    const davet_status e = check_launch();
+    if (e != DAVET_OK) return e;
+  }
+  SelArgs a;
+  a.partial = partial;
+  a.nsplit = L.nsplit;
+  a.cu = cu_resp_dev;
+  a.batch = batch;
+  a.total_rows = total_rows;
+  a.k = k;
+  a.masked = masked_dev;
+  a.tokens = tokens_dev;
+  a.argmax = argmax_dev;
+  a.conf_out = conf_dev;
+  a.committed = committed_dev;
+  a.stats = stats_dev;
+  a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
+  a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
+  a.err = err;
+  select_commit<<<batch, kSelThreads, 0, s>>>(a);
   return check_launch();
 }

@@ -71,6 +71,8 @@ def _declare(lib):
         "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_unmask_topk": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                      _vp]),
+        "davet_unmask_topk_noalloc": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp,
+                                             _vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -144,6 +146,16 @@ class Davet:
                     self.lib.davet_unmask_topk(_ptr(logits), V, _ptr(cu_resp), batch, total_rows, k, _ptr(masked),
                                                _ptr(tokens), _ptr(argmax), _ptr(conf), _ptr(committed),
                                                _ptr(stats), _ptr(workspace), workspace_bytes, _stream(stream)))
+
+
+    def davet_unmask_topk_noalloc(self, logits, V: int, cu_resp, batch: int, total_rows: int, k: int, masked,
+                                  tokens, argmax=None, conf=None, committed=None, stats=None, stream=None):
+        """davet_unmask_topk for callers that cannot allocate device memory:
+        the library's own fixed scratch array replaces the workspace."""
+        self._check("davet_unmask_topk_noalloc",
+                    self.lib.davet_unmask_topk_noalloc(_ptr(logits), V, _ptr(cu_resp), batch, total_rows, k,
+                                                       _ptr(masked), _ptr(tokens), _ptr(argmax), _ptr(conf),
+                                                       _ptr(committed), _ptr(stats), _stream(stream)))
 
 
 _handle = None
