@@ -53,12 +53,13 @@ struct Smem {
   alignas(1024) uint8_t k[NS][KC][kChunkBytes];
   alignas(1024) uint8_t v[NS][KC][kChunkBytes];
   uint64_t q_full, q_empty, fin;
-  uint64_t k_full[NS], v_full[NS], kv_empty[NS];
+  uint64_t k_full[NS], v_full[NS], k_empty[NS], v_empty[NS];
   uint64_t s_full[2], p_full[2], o_full[2];
   uint32_t tmem;
   int abort;
   int n_req;   // requests with at least one row
   int n_items;
+  int qtiles;
   int32_t req_start[kMaxBatch];
   int32_t req_len[kMaxBatch];
   int32_t order[kMaxBatch];   // request index of the i-th scheduled request
@@ -70,14 +71,46 @@ struct Params {
   int batch;
   int H;
   int max_rows;
-  int qtiles;  // query tiles per work item (1 or 2)
+  int qtiles;    // query tiles per work item: 1, 2, or 0 = chosen on the device
+  int qt2_cost;  // cost of a two-tile item relative to a one-tile item, x16
   float scale_log2;
   uint16_t* out;
   unsigned* err;
 };
 
+// Optional timeline trace of CTA 0 (clock64 stamps), compiled in only with
+// -DDAVET_ATTN_TRACE for pipeline studies; the product build has none.
+#ifdef DAVET_ATTN_TRACE
+// region r (0 producer, 1 MMA, 2 softmax A, 3 softmax B) holds 2048 events;
+// plain stores only, so recording stays off the critical path
+__device__ unsigned long long* g_attn_trace;
+__device__ __forceinline__ void trace_event(unsigned region, unsigned& n, unsigned code, unsigned idx) {
+  unsigned long long* t = g_attn_trace;
+  if (blockIdx.x != 0 || t == nullptr || n >= 2048) return;
+  t[(region * 2048 + n) * 2] = clock64();
+  t[(region * 2048 + n) * 2 + 1] = (static_cast<unsigned long long>(code) << 32) | idx;
+  ++n;
+}
+#define ATTN_TRACE(region, code, idx) trace_event((region), trace_n, (code), (idx))
+#define ATTN_TRACE_DECL unsigned trace_n = 0
+#else
+#define ATTN_TRACE(region, code, idx) \
+  do {                                \
+  } while (0)
+#define ATTN_TRACE_DECL \
+  do {                  \
+  } while (0)
+#endif
+
 struct Item {
   int start, len, q0, h, nkv, ntile;  // q0: first query row of the item within the request
+  int kv0;  // key tile the item starts from (key tiles are visited cyclically)
+
+  // key tile visited at loop step j
+  __device__ __forceinline__ int key_tile(int j) const {
+    const int k = j + kv0;
+    return k >= nkv ? k - nkv : k;
+  }
 };
 
 // Coordinate along the tensor map's second dimension: slot (0 = query,
@@ -103,6 +136,10 @@ __device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H, int qt
   it.h = local / nq;
   it.q0 = (local - it.h * nq) * rows_per_item;
   it.nkv = (len + BN - 1) / BN;
+  // query blocks of one head start at evenly spread key tiles, so CTAs that
+  // run together on the same head read different K/V lines at any moment
+  const int qb = local - it.h * nq;
+  it.kv0 = static_cast<int>((static_cast<long long>(qb) * it.nkv) / nq);
   it.ntile = (qtiles == 2 && it.q0 + BM < len) ? 2 : 1;
   return it;
 }
@@ -124,11 +161,36 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = tid >> 5;
   const int lane = tid & 31;
   const int H = prm.H;
-  const int qtiles = prm.qtiles;
+
+  // ------------------------------------ barriers, TMEM (no global memory)
+  if (tid == 0) {
+    s.abort = 0;
+    mbar_init(&s.q_full, 1);
+    mbar_init(&s.q_empty, 1);
+    mbar_init(&s.fin, 1);
+    for (int i = 0; i < NS; ++i) {
+      mbar_init(&s.k_full[i], 1);
+      mbar_init(&s.v_full[i], 1);
+      mbar_init(&s.k_empty[i], 1);
+      mbar_init(&s.v_empty[i], 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(&s.s_full[t], 1);
+      mbar_init(&s.p_full[t], 128);
+      mbar_init(&s.o_full[t], 1);
+    }
+    fence_mbar_init();
+  }
+  if (warp == kWarpMma) {
+    tmem_alloc(&s.tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kWarpTma && lane == 0) tma_prefetch_desc(&tmap);
+  pdl_launch_dependents();
+  pdl_wait();  // cu_seqlens and qkv come from the previous kernel
 
   // ---------------------------------------------------------- schedule
   if (tid == 0) {
-    s.abort = 0;
     bool bad = false;
     int prev_end = 0;
     int n = 0;
@@ -163,8 +225,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
   }
   if (tid == 0) {
+    // query tiles per item: two tiles keep the tensor pipe busy while the
+    // other tile's softmax runs, one tile gives more items when sequences
+    // are short; pick the smaller estimated makespan (rounds of items over
+    // the grid, an item with two tiles costing qt2_cost/16 of a one-tile item)
+    int qt = prm.qtiles;
+    if (qt == 0) {
+      long long i1 = 0, i2 = 0;
+      for (int i = 0; i < s.n_req; ++i) {
+        const int L = s.req_len[s.order[i]];
+        i1 += (L + BM - 1) / BM;
+        i2 += (L + 2 * BM - 1) / (2 * BM);
+      }
+      const long long g = gridDim.x;
+      const long long c1 = ((i1 * H + g - 1) / g) * 16;
+      const long long c2 = ((i2 * H + g - 1) / g) * prm.qt2_cost;
+      qt = c2 <= c1 ? 2 : 1;
+    }
+    s.qtiles = qt;
     int acc = 0;
-    const int rows_per_item = BM * qtiles;
+    const int rows_per_item = BM * qt;
     for (int i = 0; i < s.n_req; ++i) {
       s.cum[i] = acc;
       acc += ((s.req_len[s.order[i]] + rows_per_item - 1) / rows_per_item) * H;
@@ -172,40 +252,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     s.cum[s.n_req] = acc;
     s.n_items = acc;
   }
-  __syncthreads();
-  if (static_cast<int>(blockIdx.x) >= s.n_items) return;  // uniform: nothing to do
-
-  // ---------------------------------------------------- barriers, TMEM
-  if (tid == 0) {
-    mbar_init(&s.q_full, 1);
-    mbar_init(&s.q_empty, 1);
-    mbar_init(&s.fin, 1);
-    for (int i = 0; i < NS; ++i) {
-      mbar_init(&s.k_full[i], 1);
-      mbar_init(&s.v_full[i], 1);
-      mbar_init(&s.kv_empty[i], 1);
-    }
-    for (int t = 0; t < 2; ++t) {
-      mbar_init(&s.s_full[t], 1);
-      mbar_init(&s.p_full[t], 128);
-      mbar_init(&s.o_full[t], 1);
-    }
-    fence_mbar_init();
-  }
-  if (warp == kWarpMma) {
-    tmem_alloc(&s.tmem, kTmemCols);
-    tmem_relinquish();
-  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s.tmem;
+  const int qtiles = s.qtiles;
   volatile int* abort_flag = &s.abort;
 
   if (warp == kWarpTma) {
     // ------------------------------------------------------ TMA producer
     if (lane == 0) {
-      tma_prefetch_desc(&tmap);
+      ATTN_TRACE_DECL;
       uint32_t it = 0, wi = 0;
       bool ok = true;
       for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
@@ -218,13 +275,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_3d(s.q[t][c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), w.start + w.q0 + t * BM);
         for (int j = 0; j < w.nkv; ++j, ++it) {
           const int st = it % NS;
-          if (it >= NS) ok = mbar_wait(&s.kv_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
+          const int row = w.start + w.key_tile(j) * BN;
+          // K of stage st is free once the S MMAs of the tile that used it completed
+          if (it >= NS) ok = mbar_wait(&s.k_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
           if (!ok) break;
-          const int row = w.start + j * BN;
+          ATTN_TRACE(0, 2, it);
           mbar_arrive_expect_tx(&s.k_full[st], KC * kChunkBytes);
           for (int c = 0; c < KC; ++c) tma_load_3d(s.k[st][c], &tmap, &s.k_full[st], 64 * c, h_coord(1, w.h, H), row);
+          // V of stage st is free once the PV MMAs of that tile completed
+          if (it >= NS) ok = mbar_wait(&s.v_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
+          if (!ok) break;
           mbar_arrive_expect_tx(&s.v_full[st], KC * kChunkBytes);
           for (int c = 0; c < KC; ++c) tma_load_3d(s.v[st][c], &tmap, &s.v_full[st], 64 * c, h_coord(2, w.h, H), row);
+          ATTN_TRACE(0, 1, it);
         }
       }
       if (!ok) {
@@ -237,98 +300,112 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == kWarpMma) {
     // --------------------------------------------------------- MMA issuer
-    constexpr uint32_t kIdescQK = idesc_bf16_f32(BM, BN, false, false);
-    constexpr uint32_t kIdescPV = idesc_bf16_f32(BM, D, false, true);
-    uint32_t it = 0, wi = 0;
-    uint32_t np[2] = {0, 0};  // P tiles consumed per query tile
-    bool ok = true;
+    // One thread issues every MMA.  tcgen05.mma issue is sensitive to the code
+    // around it (a branch between two MMAs starves the tensor pipe), so each
+    // group of D/16 or BN/16 MMAs is straight-line code with precomputed
+    // descriptors and immediate accumulate flags.
+    if (lane == 0) {
+      ATTN_TRACE_DECL;
+      constexpr uint32_t kIdescQK = idesc_bf16_f32(BM, BN, false, false);
+      constexpr uint32_t kIdescPV = idesc_bf16_f32(BM, D, false, true);
+      // only the start-address field (16-byte units) differs between MMAs
+      const uint64_t q_desc0 = sw128_desc(smem_u32(s.q[0][0]), 16, 1024);
+      const uint64_t k_desc0 = sw128_desc(smem_u32(s.k[0][0]), 16, 1024);
+      const uint64_t v_desc0 = sw128_desc(smem_u32(s.v[0][0]), kChunkBytes, 1024);
+      constexpr uint32_t kTile16 = (KC * kChunkBytes) >> 4;  // one Q tile / K or V stage
+      uint32_t it = 0, wi = 0;
+      uint32_t np[2] = {0, 0};  // P tiles consumed per query tile
+      bool ok = true;
 
-    // S_t = Q_t K^T for the K tile in stage st
-    auto issue_s = [&](int t, int st) {
-      if (lane == 0) {
+      // S_t = Q_t K^T for the K tile in stage st
+      auto issue_s = [&](int t, int st) {
+        const uint64_t a0 = q_desc0 + t * kTile16;
+        const uint64_t b0 = k_desc0 + st * kTile16;
+        const uint32_t d = tmem + col_s(t);
+        umma_ss_imm<false>(d, a0, b0, kIdescQK);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk & 3) * 32;
-          const uint64_t a = sw128_desc(smem_u32(s.q[t][kk >> 2]) + off, 16, 1024);
-          const uint64_t b = sw128_desc(smem_u32(s.k[st][kk >> 2]) + off, 16, 1024);
-          umma_ss(tmem + col_s(t), a, b, kIdescQK, kk > 0 ? 1u : 0u);
+        for (int kk = 1; kk < D / 16; ++kk) {
+          const uint32_t off = ((kk >> 2) * kChunkBytes + (kk & 3) * 32) >> 4;
+          umma_ss_imm<true>(d, a0 + off, b0 + off, kIdescQK);
         }
         umma_commit(&s.s_full[t]);
-      }
-      __syncwarp();
-    };
-    // O_t (+)= P_t V for the V tile in stage st, P read from TMEM
-    auto issue_pv = [&](int t, int st, bool first) {
-      if (lane == 0) {
-        const uint32_t v0 = smem_u32(s.v[st][0]);
+      };
+      // O_t (+)= P_t V for the V tile in stage st, P read from TMEM
+      auto issue_pv = [&](int t, int st, bool first) {
+        const uint64_t b0 = v_desc0 + st * kTile16;
+        const uint32_t d = tmem + col_o(t);
+        const uint32_t a = tmem + col_s(t);
+        if (first)
+          umma_ts_imm<false>(d, a, b0, kIdescPV);
+        else
+          umma_ts_imm<true>(d, a, b0, kIdescPV);
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t b = sw128_desc(v0 + kk * 2048, kChunkBytes, 1024);
-          umma_ts(tmem + col_o(t), tmem + col_s(t) + kk * 8, b, kIdescPV, (first && kk == 0) ? 0u : 1u);
-        }
-      }
-      __syncwarp();
-    };
-    auto commit = [&](uint64_t* bar) {
-      if (lane == 0) umma_commit(bar);
-      __syncwarp();
-    };
+        for (int kk = 1; kk < BN / 16; ++kk) umma_ts_imm<true>(d, a + kk * 8, b0 + kk * (2048 >> 4), kIdescPV);
+      };
 
-    for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
-      const Item w = decode(s, item, H, qtiles);
-      ok = warp_wait(&s.q_full, wi & 1, prm.err, abort_flag);
-      if (!ok) break;
-      tc_fence_after();
-      // prologue: S for key tile 0
-      ok = warp_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
-      if (!ok) break;
-      tc_fence_after();
-      for (int t = 0; t < w.ntile; ++t) issue_s(t, it % NS);
-      if (w.nkv == 1) commit(&s.q_empty);
-      for (int j = 0; ok && j < w.nkv; ++j, ++it) {
-        const int st = it % NS;
-        const int st1 = (it + 1) % NS;
-        const bool more = j + 1 < w.nkv;
-        ok = warp_wait(&s.v_full[st], (it / NS) & 1, prm.err, abort_flag);
+      for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
+        const Item w = decode(s, item, H, qtiles);
+        ok = mbar_wait(&s.q_full, wi & 1, prm.err, abort_flag);
         if (!ok) break;
-        const int valid_keys = min(BN, w.len - j * BN);
-        if (valid_keys < BN) {
-          // keys past the request end: zero their V rows (P is 0 there, but
-          // the rows may hold anything, including non-finite values)
-          for (int c = 0; c < KC; ++c) {
-            uint4* base = reinterpret_cast<uint4*>(s.v[st][c]);
-            for (int idx = valid_keys * 8 + lane; idx < BN * 8; idx += 32) base[idx] = make_uint4(0, 0, 0, 0);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-        }
-        if (more) {
-          ok = warp_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
+        // prologue: S for key tile 0
+        ok = mbar_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        issue_s(0, it % NS);
+        if (w.ntile == 2) issue_s(1, it % NS);
+        umma_commit(&s.k_empty[it % NS]);
+        if (w.nkv == 1) umma_commit(&s.q_empty);
+        for (int j = 0; j < w.nkv; ++j, ++it) {
+          const int st = it % NS;
+          const int st1 = (it + 1) % NS;
+          const bool more = j + 1 < w.nkv;
+          ok = mbar_wait(&s.v_full[st], (it / NS) & 1, prm.err, abort_flag);
           if (!ok) break;
-        }
-        for (int t = 0; t < w.ntile; ++t) {
-          ok = warp_wait(&s.p_full[t], np[t] & 1, prm.err, abort_flag);
+          ATTN_TRACE(1, 10, it);
+          // tile A: PV, then S of the next key tile
+          ok = mbar_wait(&s.p_full[0], np[0] & 1, prm.err, abort_flag);
           if (!ok) break;
-          ++np[t];
+          ATTN_TRACE(1, 12, it);
+          ++np[0];
           tc_fence_after();
-          issue_pv(t, st, j == 0);
+          issue_pv(0, st, j == 0);
+          if (w.ntile == 1) umma_commit(&s.v_empty[st]);
           if (more) {
-            issue_s(t, st1);
-            if (j + 1 == w.nkv - 1 && t == w.ntile - 1) commit(&s.q_empty);
+            ok = mbar_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
+            if (!ok) break;
+            ATTN_TRACE(1, 11, it);
+            tc_fence_after();
+            issue_s(0, st1);
+            if (w.ntile == 1) {
+              umma_commit(&s.k_empty[st1]);
+              if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
+            }
           } else {
-            commit(&s.o_full[t]);
+            umma_commit(&s.o_full[0]);
+          }
+          if (w.ntile == 2) {
+            // tile B: PV, then S of the next key tile
+            ok = mbar_wait(&s.p_full[1], np[1] & 1, prm.err, abort_flag);
+            if (!ok) break;
+            ATTN_TRACE(1, 13, it);
+            ++np[1];
+            tc_fence_after();
+            issue_pv(1, st, j == 0);
+            umma_commit(&s.v_empty[st]);
+            if (more) {
+              issue_s(1, st1);
+              umma_commit(&s.k_empty[st1]);
+              if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
+            } else {
+              umma_commit(&s.o_full[1]);
+            }
           }
         }
-        if (!ok) break;
-        commit(&s.kv_empty[st]);
       }
-    }
-    // wait until every issued MMA has completed before TMEM is released
-    if (lane == 0) {
+      // wait until every issued MMA has completed before TMEM is released
       umma_commit(&s.fin);
       mbar_wait(&s.fin, 0, nullptr, nullptr);
     }
-    __syncwarp();
   } else {
     // ------------------------------------------------- softmax + epilogue
     const int t = warp >> 2;             // query tile of this warpgroup
@@ -336,6 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t s_addr = tmem + lane_base + col_s(t);
     const uint32_t o_addr = tmem + lane_base + col_o(t);
+    ATTN_TRACE_DECL;
     const float c = prm.scale_log2;
     uint32_t ns = 0, no = 0;
     bool ok = true;
@@ -347,26 +425,47 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < w.nkv; ++j, ++ns) {
         ok = warp_wait(&s.s_full[t], ns & 1, prm.err, abort_flag);
         if (!ok) break;
+        if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
         tc_fence_after();
-        float x[BN];
-        {
-          uint32_t raw[32];
+        // all four TMEM loads in flight before one wait
+        uint32_t raw[BN];
 #pragma unroll
-          for (int q = 0; q < BN / 32; ++q) {
-            tmem_ld32(s_addr + 32 * q, raw);
-            tmem_wait_ld();
+        for (int q = 0; q < BN / 32; ++q)
+          tmem_ld32(s_addr + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&raw[32 * q]));
+        tmem_wait_ld();
+        if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
+        float* x = reinterpret_cast<float*>(raw);
+        const int valid = min(BN, w.len - w.key_tile(j) * BN);
+        if (t == 0 && valid < BN) {
+          // keys past the request end: zero their V rows before PV reads them
+          // (P is 0 there, but the rows may hold anything, including
+          // non-finite values).  Tile A's key-tile count equals the global
+          // key-tile counter, so ns names the V stage and phase.
+          ok = warp_wait(&s.v_full[ns % NS], (ns / NS) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          if (r >= valid) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) x[32 * q + i] = __uint_as_float(raw[i]);
+            for (int cc = 0; cc < KC; ++cc) {
+              uint4* row = reinterpret_cast<uint4*>(s.v[ns % NS][cc] + r * 128);
+#pragma unroll
+              for (int u = 0; u < 8; ++u) row[u] = make_uint4(0, 0, 0, 0);
+            }
           }
+          fence_proxy_async_smem();
         }
-        const int valid = min(BN, w.len - j * BN);
         if (valid < BN) {
 #pragma unroll
           for (int i = 0; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
         }
-        float mx = x[0];
+        // row max: eight independent chains of three-input max, then a tree
+        float mp[8];
 #pragma unroll
-        for (int i = 1; i < BN; ++i) mx = fmaxf(mx, x[i]);
+        for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
+#pragma unroll
+        for (int i = 16; i < BN; i += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+        const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
         const float mt = mx * c;
         float factor = 1.f;
         bool need = false;
@@ -378,19 +477,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           need = true;
         }
         const float neg_m = -m;
-        float rs = 0.f;
+        // p = 2^(c*s - m): packed FMA for two scores, two SFU exponentials;
+        // the row sum runs in two packed accumulators (four lanes)
+        float rsum[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int q = 0; q < BN / 32; ++q) {
           uint32_t pk[16];
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
-            const float p0 = ex2(fmaf(x[32 * q + 2 * i], c, neg_m));
-            const float p1 = ex2(fmaf(x[32 * q + 2 * i + 1], c, neg_m));
-            rs += p0 + p1;
+            float a0, a1;
+            ffma2(a0, a1, x[32 * q + 2 * i], x[32 * q + 2 * i + 1], c, c, neg_m, neg_m);
+            const float p0 = ex2(a0);
+            const float p1 = ex2(a1);
+            const int h = (i & 1) * 2;
+            fadd2(rsum[h], rsum[h + 1], rsum[h], rsum[h + 1], p0, p1);
             pk[i] = pack_bf16x2(p0, p1);
           }
           tmem_st16(s_addr + 16 * q, pk);
         }
+        const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
         // O is settled here (S of this tile was issued after the previous
         // PV of this tile) and no MMA touches it before P is published
         if (j > 0 && __any_sync(0xffffffffu, need)) {
@@ -408,6 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&s.p_full[t]);
+        if (r == 0) ATTN_TRACE(2 + t, 24 + t, ns);
       }
       if (!ok) break;
       // ------------------------------------------------------- epilogue
@@ -523,9 +629,9 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   prm.batch = batch;
   prm.H = H;
   prm.max_rows = static_cast<int>(max_rows);
-  // two query tiles per item unless that leaves most SMs idle
-  const int64_t items2 = ((max_rows + 2 * attn::BM - 1) / (2 * attn::BM)) * static_cast<int64_t>(H);
-  prm.qtiles = items2 >= 2LL * g_dev[dev].sms ? 2 : 1;
+  prm.qtiles = 0;
+  prm.qt2_cost = 26;
+  if (const char* e = std::getenv("DAVET_ATTN_QTILES")) prm.qtiles = std::atoi(e) == 1 ? 1 : (std::atoi(e) == 2 ? 2 : 0);
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
   prm.out = static_cast<uint16_t*>(out);
   prm.err = err;
@@ -533,12 +639,19 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   const int64_t items_bound = ((max_rows + attn::BM - 1) / attn::BM + batch) * static_cast<int64_t>(H);
   const int grid = static_cast<int>(std::min<int64_t>(items_bound, g_dev[dev].sms));
   if (grid <= 0) return DAVET_OK;
-  attn::attention_kernel<D><<<grid, attn::kThreads, smem, stream>>>(tmap, prm);
-  return check_launch();
+  e = davet::launch(attn::attention_kernel<D>, dim3(grid), dim3(attn::kThreads), smem, stream, tmap, prm);
+  return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }
 
 }  // namespace
 }  // namespace davet
+
+#ifdef DAVET_ATTN_TRACE
+extern "C" int davet_debug_attn_trace(void* buf) {
+  unsigned long long* p = static_cast<unsigned long long*>(buf);
+  return static_cast<int>(cudaMemcpyToSymbol(davet::attn::g_attn_trace, &p, sizeof p));
+}
+#endif
 
 extern "C" davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev, int batch,
                                              int64_t max_total_rows, int H, int D, float scale, void* out,

@@ -17,6 +17,7 @@ namespace gat {
 constexpr int kThreads = 256;
 constexpr int kMaxBatch = 1024;
 constexpr int kMaxLevels = 5;
+constexpr int kChunk = 256;  // 16-byte slices per warp task (4 KB)
 
 struct Geom {
   int side[kMaxLevels];
@@ -56,6 +57,8 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
 
   const int tid = threadIdx.x;
   if (tid == 0) s_bad = 0;
+  pdl_launch_dependents();
+  pdl_wait();
   __syncthreads();
 
   // -------- per-request lengths, then an exclusive scan into s_cu
@@ -114,11 +117,15 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
     }
   }
 
-  // -------- row copies, one warp per row
+  // -------- row copies: one warp per 4 KB chunk of a row
   const long long gwarp = (static_cast<long long>(blockIdx.x) * kThreads + tid) >> 5;
   const long long nwarps = (static_cast<long long>(gridDim.x) * kThreads) >> 5;
   const int C8 = g.C8;
-  for (long long row = gwarp; row < rows; row += nwarps) {
+  const int nchunk = (C8 + kChunk - 1) / kChunk;
+  const long long items = rows * nchunk;
+  for (long long it = gwarp; it < items; it += nwarps) {
+    const long long row = it / nchunk;
+    const int ch = static_cast<int>(it - row * nchunk);
     // request owning this row: largest b with s_cu[b] <= row
     int lo = 0, hi = a.batch - 1;
     while (lo < hi) {
@@ -134,15 +141,14 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
       src = a.text + (a.text_off[b] + (j - s_nvis[b])) * C8;
     }
     uint4* dst = a.packed + row * C8;
-    int c = lane;
-    for (; c + 7 * 32 < C8; c += 8 * 32) {
-      uint4 v[8];
+    const int c0 = ch * kChunk + lane;
+    uint4 v[kChunk / 32];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = ld_nc(src + c + u * 32);
+    for (int u = 0; u < kChunk / 32; ++u)
+      if (c0 + u * 32 < C8) v[u] = ld_nc(src + c0 + u * 32);
 #pragma unroll
-      for (int u = 0; u < 8; ++u) dst[c + u * 32] = v[u];
-    }
-    for (; c < C8; c += 32) dst[c] = ld_nc(src + c);
+    for (int u = 0; u < kChunk / 32; ++u)
+      if (c0 + u * 32 < C8) dst[c0 + u * 32] = v[u];
   }
 }
 
@@ -190,10 +196,12 @@ extern "C" davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const
   a.cap = max_total_rows;
   a.err = err;
   const size_t smem = static_cast<size_t>(4 * batch + 1) * sizeof(long long);
-  // one warp per row: enough blocks to cover the capacity, at most 8 waves of 8 blocks per SM
-  const long long warps_needed = std::max<long long>(max_total_rows, 1);
-  const long long blocks = std::min<long long>((warps_needed + kThreads / 32 - 1) / (kThreads / 32), 152LL * 8 * 2);
-  gather_kernel<<<static_cast<unsigned>(std::max<long long>(blocks, 1)), kThreads, smem,
-                  static_cast<cudaStream_t>(stream)>>>(a, g);
+  // one warp per 4 KB chunk: enough blocks to cover the capacity, at most 16 blocks per SM
+  const long long nchunk = (g.C8 + kChunk - 1) / kChunk;
+  const long long tasks = std::max<long long>(max_total_rows * nchunk, 1);
+  const long long blocks = std::min<long long>((tasks + kThreads / 32 - 1) / (kThreads / 32), 152LL * 16);
+  const cudaError_t e = launch(gather_kernel, dim3(static_cast<unsigned>(std::max<long long>(blocks, 1))),
+                               dim3(kThreads), smem, static_cast<cudaStream_t>(stream), a, g);
+  if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

@@ -118,6 +118,8 @@ template <int NL>
 __global__ void pyramid_kernel(const uint4* __restrict__ feat, uint4* __restrict__ pyr, float4* __restrict__ pyr32,
                                Geom g) {
   constexpr int TOP = NL - 1;
+  pdl_launch_dependents();
+  pdl_wait();
   const int gt = g.side[TOP];
   const long long cells = static_cast<long long>(gt) * gt;
   const long long total = static_cast<long long>(g.n_tiles) * cells * g.C8;
@@ -194,12 +196,14 @@ extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_t
   const uint4* f = static_cast<const uint4*>(feat);
   uint4* p = static_cast<uint4*>(pyr);
   float4* p32 = reinterpret_cast<float4*>(pyr_f32);
+  cudaError_t e;
   switch (n_levels) {
-    case 1: pyramid_kernel<1><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
-    case 2: pyramid_kernel<2><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
-    case 3: pyramid_kernel<3><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
-    case 4: pyramid_kernel<4><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
-    default: pyramid_kernel<5><<<blocks, threads, 0, st>>>(f, p, p32, g); break;
+    case 1: e = launch(pyramid_kernel<1>, dim3(blocks), dim3(threads), 0, st, f, p, p32, g); break;
+    case 2: e = launch(pyramid_kernel<2>, dim3(blocks), dim3(threads), 0, st, f, p, p32, g); break;
+    case 3: e = launch(pyramid_kernel<3>, dim3(blocks), dim3(threads), 0, st, f, p, p32, g); break;
+    case 4: e = launch(pyramid_kernel<4>, dim3(blocks), dim3(threads), 0, st, f, p, p32, g); break;
+    default: e = launch(pyramid_kernel<5>, dim3(blocks), dim3(threads), 0, st, f, p, p32, g); break;
   }
+  if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

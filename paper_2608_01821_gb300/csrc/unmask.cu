@@ -110,6 +110,8 @@ __device__ __forceinline__ void fold(Partial& p, uint4 u, int w0) {
 __global__ void __launch_bounds__(kRowThreads) row_pass(const uint4* __restrict__ logits, int V8,
                                                         const uint8_t* __restrict__ masked, long long total_rows,
                                                         int nsplit, Partial* __restrict__ out) {
+  pdl_launch_dependents();
+  pdl_wait();
   const long long item = blockIdx.x;
   const long long row = item / nsplit;
   const int split = static_cast<int>(item - row * nsplit);
@@ -197,6 +199,8 @@ __device__ __forceinline__ long long block_best(float c, long long pos, float* s
 }
 
 __global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.x;
   const long long cu0 = a.cu[b], cu1 = a.cu[b + 1];
   const long long s0 = min(max(cu0, 0LL), a.total_rows);
@@ -313,10 +317,10 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
   if (total_rows > 0) {
     const long long items = total_rows * L.nsplit;
-    row_pass<<<static_cast<unsigned>(items), kRowThreads, 0, st>>>(static_cast<const uint4*>(logits), V / 8,
-                                                                   masked_dev, total_rows, L.nsplit, partial);
-    davet_status e = check_launch();
-    if (e != DAVET_OK) return e;
+    const cudaError_t e = launch(row_pass, dim3(static_cast<unsigned>(items)), dim3(kRowThreads), 0, st,
+                                 static_cast<const uint4*>(logits), V / 8, static_cast<const uint8_t*>(masked_dev),
+                                 static_cast<long long>(total_rows), L.nsplit, partial);
+    if (e != cudaSuccess) return cuda_fail(e);
   }
   SelArgs a;
   a.partial = partial;
@@ -334,8 +338,8 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
   a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
   a.err = err;
-  select_commit<<<batch, kSelThreads, 0, st>>>(a);
-  return check_launch();
+  const cudaError_t e = launch(select_commit, dim3(batch), dim3(kSelThreads), 0, st, a);
+  return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }
 
 // ---------------------------------------------------------------------------
