@@ -41,8 +41,11 @@ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 inline Layout layout_for(int64_t total_rows, int V) {
   Layout L;
   const int64_t v8 = V / 8;
-  int64_t want = total_rows > 0 ? (1216 + total_rows - 1) / total_rows : 1;  // about 8 blocks per SM
-  const int64_t cap = std::max<int64_t>(1, v8 / 2048);                       // at least 2048 slices per split
+  // about six waves of 8 blocks per SM when every row is masked, so the grid
+  // keeps a short tail as rows are committed; each split keeps at least 1024
+  // 16-byte slices (16 KB) so the block-level merge stays cheap
+  int64_t want = total_rows > 0 ? (152 * 8 * 6 + total_rows - 1) / total_rows : 1;
+  const int64_t cap = std::max<int64_t>(1, v8 / 1024);
   L.nsplit = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(want, cap), 64)));
   L.off_partial = 0;
   L.off_conf = align256(static_cast<size_t>(total_rows) * L.nsplit * sizeof(Partial));
