@@ -193,7 +193,7 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0:
         peaks = measured_peaks()
         value = whole_job_rate(w.T * args.steps, world, total_s)
-        launches_per_pass = w.batch + w.T * 4
+        launches_per_pass = w.batch + w.T * 4  # pyramid per request; gather, attention, 2 unmask kernels per step
         attn_flops_launch = comp["attention"]["flops"] / comp["attention"]["launches"]
         attn_ms = comp["attention"]["ms"] / comp["attention"]["launches"]
         achieved = attn_flops_launch / (attn_ms * 1e-3) / 1e12

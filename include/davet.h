@@ -13,6 +13,8 @@
  *   davet_unmask_topk     argmax, confidence and confidence-ranked commit
  *                         (Sec. 3.1, Eq. 1-2) plus the mean confidence and
  *                         churn that drive the trajectory risk (Eq. 7)
+ *   davet_policy_*        the allocation policy that picks each step's view
+ *                         (Sec. 4.2, Eq. 6-8; Sec. 4.3, Eq. 9)
  *
  * Conventions shared by every entry point:
  *  - Pointers named *_dev, and every tensor argument, are DEVICE pointers on
@@ -177,7 +179,8 @@ davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev
 
 /* ------------------------------------------------------------ unmasking */
 
-/* Bytes of device workspace that davet_unmask_topk needs for these sizes. */
+/* Bytes of device workspace that davet_unmask_topk needs for these sizes
+ * (batch = number of requests). */
 davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, size_t* bytes);
 
 /*
@@ -206,7 +209,8 @@ davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, s
  *   committed_dev int32 [batch][k], nullable: request-local positions
  *                 committed this step in rank order, -1 padded
  *   stats_dev     float [batch][2], nullable: (mean conf over M_t, churn)
- *   workspace     device scratch of davet_unmask_topk_workspace() bytes
+ *   workspace     device scratch of davet_unmask_topk_workspace() bytes;
+ *                 calls that may run concurrently need separate workspaces
  * Device-side checks: request boundaries outside [0, total_rows] set
  * DAVET_DEV_ARG and are clamped.
  */
@@ -214,6 +218,46 @@ davet_status davet_unmask_topk(const void* logits, int V, const int32_t* cu_resp
                                int64_t total_rows, int k, uint8_t* masked_dev, int32_t* tokens_dev,
                                int32_t* argmax_dev, float* conf_dev, int32_t* committed_dev, float* stats_dev,
                                void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------ allocation policy */
+
+/*
+ * Evidence envelope of the denoising-aware allocation policy (Sec. 4.2,
+ * Eq. 6), computed once per request before denoising.
+ *   T            denoising steps, 1..4096
+ *   orientation  0 = early grounding, p_t = 1 - (t - 0.5)/T;
+ *                1 = late verification, p_t = (t - 0.5)/T  (t = 1..T)
+ *   B, rho       average budget and reserve fraction, in [0, 1]
+ *   demand_dev   double [batch] operation demand d(o) in [0, 1] (Table A);
+ *                NULL means d = 1 for every request (uniform demand)
+ *   lower_dev, upper_dev  double [batch][T] out:
+ *                lower = N(p; (1 - rho) B), upper = N(p; (1 - rho + rho d) B),
+ *                where N(p; m) = clip(s p, 0, 1) with s >= 0 chosen so that
+ *                the mean over the T steps equals m (the normalizer that
+ *                rescales the profile and clips it to [0, 1]).
+ * Computed in fp64.
+ */
+davet_status davet_policy_envelope(int T, int orientation, double B, double rho, const double* demand_dev,
+                                   int batch, double* lower_dev, double* upper_dev, void* stream);
+
+/*
+ * One step of the allocation policy: trajectory risk (Eq. 7), envelope
+ * interpolation (Eq. 8) and thirds quantization (Eq. 9), for step t
+ * (0-based; the paper's step t+1) of every request.
+ *   r = 1 at t = 0; otherwise r = 1 - alpha * cbar * (1 - chi) with
+ *   (cbar, chi) = stats_prev_dev[b] from the previous davet_unmask_topk call
+ *   (mean confidence over the positions still masked then, and churn);
+ *   b_t = lower[t] + r (upper[t] - lower[t]);
+ *   view = coarse if b_t < 1/3, mixed if b_t < 2/3, else high.
+ *   view_level      host int32 [3]: pyramid level used for the coarse, mixed
+ *                   and high views (level 0 is the full encoding)
+ *   level_out_dev   int32 [batch] out: the level for davet_gather_view
+ *   budget_out_dev  double [batch] out, nullable: b_t
+ * Computed in fp64.
+ */
+davet_status davet_policy_step(int t, int T, const double* lower_dev, const double* upper_dev,
+                               const float* stats_prev_dev, int batch, double alpha, const int32_t* view_level,
+                               int32_t* level_out_dev, double* budget_out_dev, void* stream);
 
 /* Size of the scratch array that davet_unmask_topk_noalloc uses (per device). */
 #define DAVET_NOALLOC_SCRATCH_BYTES (1u << 20)

@@ -38,7 +38,7 @@ struct Layout {
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-inline Layout layout_for(int64_t total_rows, int V) {
+inline Layout layout_for(int64_t total_rows, int V, int batch = 0) {
   Layout L;
   const int64_t v8 = V / 8;
   // about six waves of 8 blocks per SM when every row is masked, so the grid
@@ -51,6 +51,7 @@ inline Layout layout_for(int64_t total_rows, int V) {
   L.off_conf = align256(static_cast<size_t>(total_rows) * L.nsplit * sizeof(Partial));
   L.off_idx = L.off_conf + align256(static_cast<size_t>(total_rows) * sizeof(float));
   L.bytes = L.off_idx + align256(static_cast<size_t>(total_rows) * sizeof(int));
+  (void)batch;
   return L;
 }
 
@@ -201,10 +202,9 @@ __device__ __forceinline__ long long block_best(float c, long long pos, float* s
   return best;
 }
 
-__global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int b = blockIdx.x;
+// Merge the splits of request b's masked rows, count churn, take the top-k
+// and commit; run by one block of kSelThreads threads.
+__device__ __forceinline__ void select_request(const SelArgs& a, int b) {
   const long long cu0 = a.cu[b], cu1 = a.cu[b + 1];
   const long long s0 = min(max(cu0, 0LL), a.total_rows);
   const long long s1 = min(max(cu1, s0), a.total_rows);
@@ -219,8 +219,17 @@ __global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
   int n_masked = 0, n_both = 0, n_changed = 0;
   for (long long i = s0 + threadIdx.x; i < s1; i += kSelThreads) {
     if (!a.masked[i]) continue;
+    // load the row's partials eight at a time, then merge them
     Partial p = a.partial[i * a.nsplit];
-    for (int sp = 1; sp < a.nsplit; ++sp) p = merge(p, a.partial[i * a.nsplit + sp]);
+    for (int sp0 = 1; sp0 < a.nsplit; sp0 += 8) {
+      Partial q[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (sp0 + u < a.nsplit) q[u] = a.partial[i * a.nsplit + sp0 + u];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (sp0 + u < a.nsplit) p = merge(p, q[u]);
+    }
     const int idx = p.idx == INT_MAX ? 0 : p.idx;
     const float conf = 1.f / p.s;
     a.row_conf[i] = conf;
@@ -288,13 +297,19 @@ __global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
     for (int j = take + threadIdx.x; j < a.k; j += kSelThreads) a.committed[static_cast<long long>(b) * a.k + j] = -1;
 }
 
+
+__global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  select_request(a, blockIdx.x);
+}
+
 }  // namespace unm
 }  // namespace davet
 
 extern "C" davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, size_t* bytes) {
-  (void)batch;
-  if (total_rows < 0 || V < 8 || V % 8 != 0 || !bytes) return DAVET_ERR_INVALID_ARG;
-  *bytes = davet::unm::layout_for(total_rows, V).bytes;
+  if (total_rows < 0 || V < 8 || V % 8 != 0 || batch < 0 || !bytes) return DAVET_ERR_INVALID_ARG;
+  *bytes = davet::unm::layout_for(total_rows, V, batch).bytes;
   return DAVET_OK;
 }
 
@@ -311,20 +326,13 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   if (reinterpret_cast<uintptr_t>(logits) & 15u) return DAVET_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(workspace) & 255u) return DAVET_ERR_INVALID_ARG;
   if (batch > 65535 || total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
-  const Layout L = layout_for(total_rows, V);
+  const Layout L = layout_for(total_rows, V, batch);
   if (workspace_bytes < L.bytes) return DAVET_ERR_INVALID_ARG;
   unsigned* err = device_error_word();
   if (!err) return DAVET_ERR_CUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
-  if (total_rows > 0) {
-    const long long items = total_rows * L.nsplit;
-    const cudaError_t e = launch(row_pass, dim3(static_cast<unsigned>(items)), dim3(kRowThreads), 0, st,
-                                 static_cast<const uint4*>(logits), V / 8, static_cast<const uint8_t*>(masked_dev),
-                                 static_cast<long long>(total_rows), L.nsplit, partial);
-    if (e != cudaSuccess) return cuda_fail(e);
-  }
   SelArgs a;
   a.partial = partial;
   a.nsplit = L.nsplit;
@@ -341,6 +349,13 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
   a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
   a.err = err;
+  if (total_rows > 0) {
+    const long long items = total_rows * L.nsplit;
+    const cudaError_t e = launch(row_pass, dim3(static_cast<unsigned>(items)), dim3(kRowThreads), 0, st,
+                                 static_cast<const uint4*>(logits), V / 8, static_cast<const uint8_t*>(masked_dev),
+                                 static_cast<long long>(total_rows), L.nsplit, partial);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   const cudaError_t e = launch(select_commit, dim3(batch), dim3(kSelThreads), 0, st, a);
   return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }

@@ -71,6 +71,9 @@ def _declare(lib):
         "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_unmask_topk": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                      _vp]),
+        "davet_policy_envelope": (_int, [_int, _int, ctypes.c_double, ctypes.c_double, _vp, _int, _vp, _vp, _vp]),
+        "davet_policy_step": (_int, [_int, _int, _vp, _vp, _vp, _int, ctypes.c_double, ctypes.POINTER(_i32), _vp,
+                                     _vp, _vp]),
         "davet_unmask_topk_noalloc": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp,
                                              _vp]),
     }
@@ -147,6 +150,19 @@ class Davet:
                                                _ptr(tokens), _ptr(argmax), _ptr(conf), _ptr(committed),
                                                _ptr(stats), _ptr(workspace), workspace_bytes, _stream(stream)))
 
+
+    def davet_policy_envelope(self, T: int, orientation: int, B: float, rho: float, demand, batch: int, lower,
+                              upper, stream=None):
+        self._check("davet_policy_envelope",
+                    self.lib.davet_policy_envelope(T, orientation, float(B), float(rho), _ptr(demand), batch,
+                                                   _ptr(lower), _ptr(upper), _stream(stream)))
+
+    def davet_policy_step(self, t: int, T: int, lower, upper, stats_prev, batch: int, alpha: float, view_level,
+                          level_out, budget_out=None, stream=None):
+        vl = (_i32 * 3)(*[int(x) for x in view_level])
+        self._check("davet_policy_step",
+                    self.lib.davet_policy_step(t, T, _ptr(lower), _ptr(upper), _ptr(stats_prev), batch, float(alpha),
+                                               vl, _ptr(level_out), _ptr(budget_out), _stream(stream)))
 
     def davet_unmask_topk_noalloc(self, logits, V: int, cu_resp, batch: int, total_rows: int, k: int, masked,
                                   tokens, argmax=None, conf=None, committed=None, stats=None, stream=None):

@@ -51,7 +51,7 @@ class Pipeline:
         self.committed = torch.full((w.T, B, w.k), -1, dtype=torch.int32, device=self.dev)
         self.stats = torch.zeros((w.T, B, 2), dtype=torch.float32, device=self.dev)
         ws = self.lib.davet_unmask_topk_workspace(R, w.V, B)
-        self.workspace = torch.empty(max(ws, 256), dtype=torch.uint8, device=self.dev)
+        self.workspace = torch.zeros(max(ws, 256), dtype=torch.uint8, device=self.dev)
 
     # -------------------------------------------------------------- inputs
     def level0(self, b: int):

@@ -80,6 +80,16 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_unmask_topk(p, 1000, p, 1, 128, 2, p, p, null, null, null, null, p, ws_needed - 1,
                                  null) == INV
     assert lib.davet_unmask_topk(p, 1000, p, 0, 128, 2, p, p, null, null, null, null, p, ws_needed, null) == 0
+    # policy: bad T, orientation, budget; step past T; missing view table
+    d = ctypes.c_double
+    assert lib.davet_policy_envelope(0, 0, d(0.5), d(0.2), null, 1, p, p, null) == INV
+    assert lib.davet_policy_envelope(16, 2, d(0.5), d(0.2), null, 1, p, p, null) == INV
+    assert lib.davet_policy_envelope(16, 0, d(1.5), d(0.2), null, 1, p, p, null) == INV
+    assert lib.davet_policy_envelope(16, 0, d(0.5), d(0.2), null, 0, p, p, null) == 0
+    vl = (ctypes.c_int32 * 3)(2, 1, 0)
+    assert lib.davet_policy_step(16, 16, p, p, null, 1, d(0.5), vl, p, null, null) == INV
+    assert lib.davet_policy_step(0, 16, p, p, null, 1, d(1.5), vl, p, null, null) == INV
+    assert lib.davet_policy_step(0, 16, p, p, null, 1, d(0.5), None, p, null, null) == INV
 
 
 def test_package_fails_loudly_without_library(tmp_path):

@@ -1,0 +1,142 @@
+"""Parity of the device allocation policy (Sec. 4.2, Eq. 6-8; Sec. 4.3, Eq. 9)
+with the oracle's policy, which the CPU tests pin to closed forms and to the
+"High" step counts of Table D.
+
+Envelopes must agree within 1e-12 (both sides are fp64; the device inverts
+the normalizer exactly, the oracle bisects).  Budgets must agree within
+1e-12, and the chosen view must be identical unless the budget lies within
+1e-12 of a thirds threshold.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01821_gb300 import workloads
+from paper_2608_01821_gb300.pipeline import Pipeline
+
+pytestmark = pytest.mark.gpu
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def read_table(name):
+    rows = []
+    for line in open(os.path.join(GOLD, name)):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            rows.append(line.split())
+    return rows
+
+
+def settings():
+    return {r[0]: dict(T=int(r[1]), orient=0 if r[2] == "early" else 1, B=float(r[3]), rho=float(r[4]),
+                       alpha=float(r[5]))
+            for r in read_table("sec5_policy_defaults.txt")}
+
+
+DEMANDS = [float(r[1]) for r in read_table("table_a_demand_prior.txt")]
+
+
+def envelope(davet, T, orient, B, rho, demands, batch=None):
+    batch = len(demands) if demands is not None else batch
+    d = torch.tensor(demands, dtype=torch.float64, device="cuda") if demands is not None else None
+    lo = torch.full((max(batch, 1), T), float("nan"), dtype=torch.float64, device="cuda")
+    up = torch.full_like(lo, float("nan"))
+    davet.davet_policy_envelope(T, orient, B, rho, d, batch, lo, up)
+    torch.cuda.synchronize()
+    return lo.cpu().numpy(), up.cpu().numpy()
+
+
+@pytest.mark.parametrize("name", ["llada_v", "lavida"])
+def test_paper_settings_envelopes(davet, name):
+    s = settings()[name]
+    lo, up = envelope(davet, s["T"], s["orient"], s["B"], s["rho"], DEMANDS)
+    p = oracle.policy_profile(s["T"], "early" if s["orient"] == 0 else "late")
+    for i, d in enumerate(DEMANDS):
+        rlo, rup = oracle.policy_envelope(p, s["B"], s["rho"], d)
+        np.testing.assert_allclose(lo[i], rlo, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(up[i], rup, rtol=0, atol=1e-12)
+
+
+def test_uniform_demand_and_random_settings(davet):
+    rng = np.random.default_rng(0)
+    for T in (1, 7, 64, 128, 256, 1000):
+        for orient in (0, 1):
+            B = float(rng.uniform(0.05, 0.95))
+            rho = float(rng.uniform(0.0, 0.6))
+            p = oracle.policy_profile(T, "early" if orient == 0 else "late")
+            lo, up = envelope(davet, T, orient, B, rho, None, batch=2)  # no demand array: d = 1
+            rlo, rup = oracle.policy_envelope(p, B, rho, 1.0)
+            for i in range(2):
+                np.testing.assert_allclose(lo[i], rlo, rtol=0, atol=1e-12)
+                np.testing.assert_allclose(up[i], rup, rtol=0, atol=1e-12)
+            d = list(rng.uniform(0, 1, size=3))
+            lo, up = envelope(davet, T, orient, B, rho, d)
+            for i in range(3):
+                rlo, rup = oracle.policy_envelope(p, B, rho, d[i])
+                np.testing.assert_allclose(lo[i], rlo, rtol=0, atol=1e-12)
+                np.testing.assert_allclose(up[i], rup, rtol=0, atol=1e-12)
+                assert abs(up[i].mean() - (1 - rho + rho * d[i]) * B) < 1e-12 or up[i].min() == 1.0
+
+
+def test_step_matches_oracle_risk_budget_and_view(davet):
+    rng = np.random.default_rng(1)
+    T, batch = 32, 6
+    lo, up = envelope(davet, T, 1, 0.45, 0.2, list(rng.uniform(0.5, 1.0, size=batch)))
+    lo_d = torch.from_numpy(lo).cuda()
+    up_d = torch.from_numpy(up).cuda()
+    view_level = [3, 1, 0]
+    alpha = 0.5
+    level = torch.full((batch,), -9, dtype=torch.int32, device="cuda")
+    budget = torch.zeros(batch, dtype=torch.float64, device="cuda")
+    stats = torch.from_numpy(rng.uniform(0, 1, size=(batch, 2)).astype(np.float32)).cuda()
+    for t in range(T):
+        stats.copy_(torch.from_numpy(rng.uniform(0, 1, size=(batch, 2)).astype(np.float32)))
+        davet.davet_policy_step(t, T, lo_d, up_d, stats, batch, alpha, view_level, level, budget)
+        torch.cuda.synchronize()
+        st = stats.cpu().numpy().astype(np.float64)
+        got_b = budget.cpu().numpy()
+        got_l = level.cpu().numpy()
+        for b in range(batch):
+            r = oracle.policy_risk(t + 1, alpha, st[b, 0], st[b, 1])
+            want = oracle.policy_budget(lo[b, t], up[b, t], r)
+            assert abs(got_b[b] - want) < 1e-12
+            if min(abs(want - 1 / 3), abs(want - 2 / 3)) > 1e-12:
+                assert got_l[b] == view_level[oracle.policy_view(want)]
+
+
+def test_closed_loop_tiny_workload(davet):
+    """The policy picks every step's level on the device from the previous
+    step's unmasking statistics; the oracle policy fed the same statistics
+    picks the same levels, and the mean budget stays below B (Eq. 4)."""
+    w = workloads.make("tiny")
+    pl = Pipeline(w, "cuda", davet)
+    pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w))
+    pl.build_pyramids()
+    B, rho, alpha, d = 0.45, 0.2, 0.5, 0.824
+    lo = torch.empty((1, w.T), dtype=torch.float64, device="cuda")
+    up = torch.empty_like(lo)
+    davet.davet_policy_envelope(w.T, 1, B, rho, torch.tensor([d], dtype=torch.float64, device="cuda"), 1, lo, up)
+    view_level = [2, 1, 0]  # coarse, mixed, high -> pyramid levels of the 12/6/3 grid
+    level = torch.zeros((w.T, 1), dtype=torch.int32, device="cuda")
+    budget = torch.zeros((w.T, 1), dtype=torch.float64, device="cuda")
+    for t in range(w.T):
+        prev = pl.stats[t - 1] if t > 0 else None
+        davet.davet_policy_step(t, w.T, lo, up, prev, 1, alpha, view_level, level[t], budget[t])
+        pl.schedule[t].copy_(level[t])
+        pl.step(t, workloads.logits(w, t).cuda())
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    p = oracle.policy_profile(w.T, "late")
+    rlo, rup = oracle.policy_envelope(p, B, rho, d)
+    stats = pl.stats.cpu().numpy().astype(np.float64)
+    bud = budget.cpu().numpy()[:, 0]
+    for t in range(w.T):
+        r = oracle.policy_risk(t + 1, alpha, stats[t - 1, 0, 0] if t else 0.0, stats[t - 1, 0, 1] if t else 0.0)
+        want = oracle.policy_budget(rlo[t], rup[t], r)
+        assert abs(bud[t] - want) < 1e-12
+        assert level.cpu().numpy()[t, 0] == view_level[oracle.policy_view(want)]
+    assert bud.mean() <= B + 1e-12

@@ -39,7 +39,7 @@ class State:
 
     def step(self, davet, logits_cpu):
         d = self.d
-        ws = torch.empty(max(davet.davet_unmask_topk_workspace(self.R, self.V, self.B), 256), dtype=torch.uint8,
+        ws = torch.zeros(max(davet.davet_unmask_topk_workspace(self.R, self.V, self.B), 256), dtype=torch.uint8,
                          device="cuda")
         davet.davet_unmask_topk(logits_cpu.cuda(), self.V, d["cu"], self.B, self.R, self.k, d["masked"],
                                 d["tokens"], d["argmax"], d["conf"], d["committed"], d["stats"], ws)

@@ -59,7 +59,7 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(davet, resp, V, k):
     B = len(resp)
     ref = _state(resp, k)
     new = _state(resp, k)
-    ws = torch.empty(max(davet.davet_unmask_topk_workspace(R, V, B), 256), dtype=torch.uint8, device=dev)
+    ws = torch.zeros(max(davet.davet_unmask_topk_workspace(R, V, B), 256), dtype=torch.uint8, device=dev)
     g = torch.Generator(device="cpu").manual_seed(R + V + k)
     for call in range(2):
         lg = (torch.randn((R, V), generator=g) * 1.4142135).to(torch.bfloat16).to(dev)
