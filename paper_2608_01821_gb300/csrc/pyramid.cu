@@ -114,6 +114,107 @@ __device__ __forceinline__ bool cell(const Ctx& c, const Geom& g, int y, int x, 
   }
 }
 
+// Level-DEPTH cell (y, x) from its (2^DEPTH)^2 level-0 leaves: every leaf
+// load is issued before any store, so the loads are in flight together even
+// when the pyramid is built in place (the output may alias the input, which
+// would otherwise keep the compiler from moving later loads above earlier
+// stores).  Then the levels 1..DEPTH are reduced in registers and stored.
+template <int DEPTH>
+__device__ __forceinline__ bool subtree(const Ctx& c, const Geom& g, int y, int x, float (&out)[8]) {
+  constexpr int S = 1 << DEPTH;
+  const int gd = g.side[DEPTH];
+  if (y >= gd || x >= gd) return false;
+  const int g0 = g.side[0];
+  uint4 leaf[S * S];
+#pragma unroll
+  for (int i = 0; i < S; ++i)
+#pragma unroll
+    for (int j = 0; j < S; ++j) {
+      const int ly = y * S + i, lx = x * S + j;
+      if (ly < g0 && lx < g0) {
+        const long long src = (static_cast<long long>(c.tile) * g0 + ly) * g0 + lx;
+        leaf[i * S + j] = ld_stream(c.feat + src * g.C8 + c.cv);
+      } else {
+        leaf[i * S + j] = make_uint4(0, 0, 0, 0);
+      }
+    }
+  // level 0 side effects: the copy into the pyramid and the fp32 form
+  if (g.copy0 || c.pyr32) {
+#pragma unroll
+    for (int i = 0; i < S; ++i)
+#pragma unroll
+      for (int j = 0; j < S; ++j) {
+        const int ly = y * S + i, lx = x * S + j;
+        if (ly < g0 && lx < g0) {
+          const long long row = g.off[0] + (static_cast<long long>(c.tile) * g0 + ly) * g0 + lx;
+          const uint4 u = leaf[i * S + j];
+          if (g.copy0) c.pyr[row * g.C8 + c.cv] = u;
+          if (c.pyr32) {
+            float4* d = c.pyr32 + (row * g.C8 + c.cv) * 2;
+            d[0] = make_float4(bf16lo(u.x), bf16hi(u.x), bf16lo(u.y), bf16hi(u.y));
+            d[1] = make_float4(bf16lo(u.z), bf16hi(u.z), bf16lo(u.w), bf16hi(u.w));
+          }
+        }
+      }
+  }
+  // level 1 cells of the subtree
+  float l1[(S / 2) * (S / 2)][8];
+  const int g1 = g.side[1];
+#pragma unroll
+  for (int a = 0; a < S / 2; ++a)
+#pragma unroll
+    for (int b = 0; b < S / 2; ++b) {
+      float acc[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+      int n = 0;
+#pragma unroll
+      for (int qq = 0; qq < 4; ++qq) {
+        const int i = 2 * a + (qq >> 1), j = 2 * b + (qq & 1);
+        if (y * S + i < g0 && x * S + j < g0) {
+          const uint4 u = leaf[i * S + j];
+          acc[0] += bf16lo(u.x); acc[1] += bf16hi(u.x);
+          acc[2] += bf16lo(u.y); acc[3] += bf16hi(u.y);
+          acc[4] += bf16lo(u.z); acc[5] += bf16hi(u.z);
+          acc[6] += bf16lo(u.w); acc[7] += bf16hi(u.w);
+          ++n;
+        }
+      }
+      const float inv = n == 4 ? 0.25f : (n == 2 ? 0.5f : 1.0f);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) l1[a * (S / 2) + b][k] = acc[k] * inv;
+      const int y1 = y * (S / 2) + a, x1 = x * (S / 2) + b;
+      if (n > 0 && y1 < g1 && x1 < g1)
+        store_row(c, g, g.off[1] + (static_cast<long long>(c.tile) * g1 + y1) * g1 + x1, l1[a * (S / 2) + b]);
+    }
+  if constexpr (DEPTH == 1) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) out[k] = l1[0][k];
+    return true;
+  } else {
+    static_assert(DEPTH == 2, "subtree depth 1 or 2");
+    // the level-2 cell from its in-range level-1 children
+    float acc[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+    int n = 0;
+#pragma unroll
+    for (int qq = 0; qq < 4; ++qq) {
+      const int y1 = 2 * y + (qq >> 1), x1 = 2 * x + (qq & 1);
+      if (y1 < g1 && x1 < g1) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] += l1[qq][k];
+        ++n;
+      }
+    }
+    const float inv = n == 4 ? 0.25f : (n == 2 ? 0.5f : 1.0f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) out[k] = acc[k] * inv;
+    store_row(c, g, g.off[2] + (static_cast<long long>(c.tile) * gd + y) * gd + x, out);
+    return true;
+  }
+}
+
 template <int NL>
 __global__ void pyramid_kernel(const uint4* __restrict__ feat, uint4* __restrict__ pyr, float4* __restrict__ pyr32,
                                Geom g) {
@@ -122,19 +223,80 @@ __global__ void pyramid_kernel(const uint4* __restrict__ feat, uint4* __restrict
   pdl_wait();
   const int gt = g.side[TOP];
   const long long cells = static_cast<long long>(gt) * gt;
-  const long long total = static_cast<long long>(g.n_tiles) * cells * g.C8;
-  for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
-       i += static_cast<long long>(gridDim.x) * blockDim.x) {
-    Ctx c;
-    c.feat = feat;
-    c.pyr = pyr;
-    c.pyr32 = pyr32;
-    c.cv = static_cast<int>(i % g.C8);
-    const long long rest = i / g.C8;
-    const int cellid = static_cast<int>(rest % cells);
-    c.tile = static_cast<int>(rest / cells);
-    float v[8];
-    cell<TOP, TOP>(c, g, cellid / gt, cellid % gt, v);
+  if constexpr (NL == 1) {
+    // a single level: only the copy of level 0 (and its fp32 form) remains
+    const long long total = static_cast<long long>(g.n_tiles) * cells * g.C8;
+    for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
+         i += static_cast<long long>(gridDim.x) * blockDim.x) {
+      Ctx c;
+      c.feat = feat;
+      c.pyr = pyr;
+      c.pyr32 = pyr32;
+      c.cv = static_cast<int>(i % g.C8);
+      const long long rest = i / g.C8;
+      c.tile = static_cast<int>(rest / cells);
+      const int cellid = static_cast<int>(rest % cells);
+      float v[8];
+      cell<0, 0>(c, g, cellid / gt, cellid % gt, v);
+    }
+  } else {
+    // A block of 8 warps covers one top-level cell and 64 consecutive 16-byte
+    // channel slices: warp w reduces child subtree q = w % 4 for slices
+    // 32 * (w / 4) + lane, so every warp load reads 512 contiguous bytes of
+    // one token row; the four children are then combined through shared
+    // memory.
+    __shared__ float s_v[4][64][9];  // [child][slice][8 values + in-range flag]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int q = warp & 3;
+    const int cv_local = (warp >> 2) * 32 + lane;
+    const int chunks = (g.C8 + 63) / 64;
+    const long long units = static_cast<long long>(g.n_tiles) * cells * chunks;
+    for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+      const int chunk = static_cast<int>(u % chunks);
+      const long long rest = u / chunks;
+      const int cellid = static_cast<int>(rest % cells);
+      Ctx c;
+      c.feat = feat;
+      c.pyr = pyr;
+      c.pyr32 = pyr32;
+      c.tile = static_cast<int>(rest / cells);
+      c.cv = chunk * 64 + cv_local;
+      const int Y = cellid / gt, X = cellid % gt;
+      float v[8];
+      bool have = false;
+      // each warp's child subtree issues all its leaf loads together (five
+      // levels: the 64-leaf subtree walks its four quarters one at a time)
+      if (c.cv < g.C8) {
+        if constexpr (NL == 3 || NL == 4)
+          have = subtree<TOP - 1>(c, g, 2 * Y + (q >> 1), 2 * X + (q & 1), v);
+        else
+          have = cell<TOP - 1, NL >= 5 ? TOP - 1 : NL>(c, g, 2 * Y + (q >> 1), 2 * X + (q & 1), v);
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s_v[q][cv_local][k] = have ? v[k] : 0.f;
+      s_v[q][cv_local][8] = have ? 1.f : 0.f;
+      __syncthreads();
+      if (threadIdx.x < 64 && chunk * 64 + threadIdx.x < g.C8) {
+        const int sl = threadIdx.x;
+        float n = 0.f, acc[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+          n += s_v[qq][sl][8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[k] += s_v[qq][sl][k];
+        }
+        const float inv = n == 4.f ? 0.25f : (n == 2.f ? 0.5f : 1.0f);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) acc[k] *= inv;
+        Ctx ct = c;
+        ct.cv = chunk * 64 + sl;
+        const long long row = g.off[TOP] + (static_cast<long long>(c.tile) * gt + Y) * gt + X;
+        store_row(ct, g, row, acc);
+      }
+      __syncthreads();
+    }
   }
 }
 
@@ -188,10 +350,17 @@ extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_t
   }
 
   const int gt = side[n_levels - 1];
-  const long long total = static_cast<long long>(n_tiles) * gt * gt * g.C8;
-  // small problems: smaller blocks spread over more SMs
-  const int threads = total >= 152LL * 2 * 256 ? 256 : (total >= 152LL * 2 * 128 ? 128 : 64);
-  const long long blocks = std::min<long long>((total + threads - 1) / threads, 152LL * 64);
+  int threads;
+  long long blocks;
+  if (n_levels > 1) {
+    // one block (8 warps) per (tile, top-level cell, 64-slice chunk)
+    threads = 256;
+    blocks = std::min<long long>(static_cast<long long>(n_tiles) * gt * gt * ((g.C8 + 63) / 64), 152LL * 64);
+  } else {
+    const long long total = static_cast<long long>(n_tiles) * gt * gt * g.C8;
+    threads = 256;
+    blocks = std::min<long long>((total + threads - 1) / threads, 152LL * 64);
+  }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const uint4* f = static_cast<const uint4*>(feat);
   uint4* p = static_cast<uint4*>(pyr);
