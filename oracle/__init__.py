@@ -15,6 +15,9 @@ Parity status of each function (what pins it is listed in the tests under
             cascade closed form, even-grid block means, ceil-mode library
             pooling, linearity)
   gather    pinned (structural row-id identities)
+  mixed     pinned (structural row-id identities, stride 1 = every token,
+            ordered coarse < mixed < high lengths); the subset rule itself is
+            a reading (a centred lattice), the paper prints none
   attention pinned (identical keys, single key, two-key sigmoid closed form,
             dominant key, permutation equivariance)
   unmask    pinned (closed-form confidences, tie rules, brute-force top-k)
@@ -61,6 +64,7 @@ def _load():
             build()
             lib = ctypes.CDLL(_LIB)
             lib.oracle_level_sides.restype = ctypes.c_int64
+            lib.oracle_mixed_view.restype = ctypes.c_int64
             lib.oracle_policy_risk.restype = ctypes.c_double
             lib.oracle_policy_budget.restype = ctypes.c_double
             lib.oracle_policy_view.restype = ctypes.c_int
@@ -131,12 +135,31 @@ def pyramid(feat_bf16, n_tiles: int, grid: int, n_levels: int, C: int) -> np.nda
 
 
 # ------------------------------------------------------------------- gather
+def mixed_rows_per_tile(grid: int, n_levels: int, coarse_level: int, stride: int) -> int:
+    """Rows of the mixed view per tile: the coarse level plus the lattice."""
+    g = level_sides(grid, n_levels)[coarse_level]
+    n = len(range(stride // 2, grid, stride))
+    return g * g + n * n
+
+
+def mixed_view(pyr_bf16, n_tiles: int, grid: int, n_levels: int, coarse_level: int, stride: int, C: int):
+    """The `mixed` view (Sec. 4.3) of one request's pyramid: uint16 [rows, C]."""
+    p = _as_u16(pyr_bf16).reshape(-1)
+    rows = n_tiles * mixed_rows_per_tile(grid, n_levels, coarse_level, stride)
+    out = np.empty((rows, C), dtype=np.uint16)
+    n = _load().oracle_mixed_view(_ptr(p, _c_u16p), n_tiles, grid, n_levels, coarse_level, stride, C,
+                                  _ptr(out, _c_u16p))
+    assert n == rows
+    return out
+
+
 def gather(pyrs, tiles, text_bf16, text_off, prompt_len, resp_len, level,
-           grid: int, n_levels: int, C: int):
+           grid: int, n_levels: int, C: int, mixed_rows_per_tile: int = 0):
     """Packed [view || prompt || response] rows per request (Eq. 5).
 
-    pyrs: list of per-request bf16 pyramids (level-major rows x C).
-    Returns (packed uint16 [N, C], cu int32 [batch+1])."""
+    pyrs: list of per-request bf16 pyramids (level-major rows x C), each
+    followed by its mixed view when mixed_rows_per_tile > 0 (level index
+    n_levels selects it).  Returns (packed uint16 [N, C], cu int32 [batch+1])."""
     batch = len(pyrs)
     p_arrs = [_as_u16(p).reshape(-1) for p in pyrs]
     ptrs = (_c_u16p * batch)(*[_ptr(p, _c_u16p) for p in p_arrs])
@@ -146,14 +169,19 @@ def gather(pyrs, tiles, text_bf16, text_off, prompt_len, resp_len, level,
     prompt_len = np.ascontiguousarray(prompt_len, dtype=np.int32)
     resp_len = np.ascontiguousarray(resp_len, dtype=np.int32)
     level = np.ascontiguousarray(level, dtype=np.int32)
-    sides = level_sides(grid, n_levels)
-    total = int(sum(int(tiles[b]) * sides[int(level[b])] ** 2 + int(prompt_len[b]) + int(resp_len[b])
-                    for b in range(batch)))
+    sides = level_sides(grid, n_levels) + [None]
+
+    def vis(b):
+        lv = int(level[b])
+        return int(tiles[b]) * (sides[lv] ** 2 if lv < n_levels else mixed_rows_per_tile)
+
+    total = int(sum(vis(b) + int(prompt_len[b]) + int(resp_len[b]) for b in range(batch)))
     out = np.empty((total, C), dtype=np.uint16)
     cu = np.empty(batch + 1, dtype=np.int32)
-    _load().oracle_gather(ptrs, _ptr(tiles, _c_i32p), _ptr(text, _c_u16p), _ptr(text_off, _c_i64p),
-                          _ptr(prompt_len, _c_i32p), _ptr(resp_len, _c_i32p), _ptr(level, _c_i32p),
-                          batch, grid, n_levels, C, _ptr(out, _c_u16p), _ptr(cu, _c_i32p))
+    _load().oracle_gather_mixed(ptrs, _ptr(tiles, _c_i32p), _ptr(text, _c_u16p), _ptr(text_off, _c_i64p),
+                                _ptr(prompt_len, _c_i32p), _ptr(resp_len, _c_i32p), _ptr(level, _c_i32p),
+                                batch, grid, n_levels, C, int(mixed_rows_per_tile), _ptr(out, _c_u16p),
+                                _ptr(cu, _c_i32p))
     return out, cu
 
 

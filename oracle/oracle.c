@@ -23,6 +23,8 @@
  *   oracle_unmask        distribution, its argmax, and the confidence-ranked
  *                        commitment of the top-k positions; Sec. 4.2 / Eq. 7
  *                        defines the mean confidence and churn statistics.
+ *   oracle_mixed_view    Sec. 4.3: the `mixed` view, coarse pooled tokens plus
+ *                        a fixed subset of unpooled tokens (a centred lattice).
  *   oracle_policy_*      Sec. 4.2 / Eq. 6-8 and Sec. 4.3 / Eq. 9: phase
  *                        profile, normalizer, evidence envelope, trajectory
  *                        risk, envelope interpolation, thirds quantization.
@@ -154,14 +156,16 @@ void oracle_pyramid_bf16(const uint16_t *feat, int n_tiles, int grid, int n_leve
  * (all tiles of that level in tile order, row-major within a tile) followed
  * by its P_b prompt rows and R_b response rows taken from
  * text[text_off[b] ...].  Rows are C bf16 values and are copied bit for bit.
- * pyr[b] is request b's pyramid in the layout of oracle_pyramid_f64.
+ * pyr[b] is request b's pyramid in the layout of oracle_pyramid_f64; when
+ * mixed_rows_per_tile > 0, its mixed view (oracle_mixed_view) follows the
+ * pooled levels and level index n_levels selects it.
  * cu[b] is the first packed row of request b; cu[batch] the total.
  */
-void oracle_gather(const uint16_t *const *pyr, const int32_t *tiles,
-                   const uint16_t *text, const int64_t *text_off,
-                   const int32_t *prompt_len, const int32_t *resp_len,
-                   const int32_t *level, int batch, int grid, int n_levels, int C,
-                   uint16_t *out, int32_t *cu)
+void oracle_gather_mixed(const uint16_t *const *pyr, const int32_t *tiles,
+                         const uint16_t *text, const int64_t *text_off,
+                         const int32_t *prompt_len, const int32_t *resp_len,
+                         const int32_t *level, int batch, int grid, int n_levels, int C,
+                         int mixed_rows_per_tile, uint16_t *out, int32_t *cu)
 {
     int side[32];
     oracle_level_sides(grid, n_levels, side);
@@ -169,9 +173,11 @@ void oracle_gather(const uint16_t *const *pyr, const int32_t *tiles,
     cu[0] = 0;
     for (int b = 0; b < batch; ++b) {
         const int l = level[b];
+        /* level index n_levels names the mixed view, stored after the pooled levels */
         int64_t level_start = 0;
-        for (int j = 0; j < l; ++j) level_start += (int64_t)tiles[b] * side[j] * side[j];
-        const int64_t n_vis = (int64_t)tiles[b] * side[l] * side[l];
+        for (int j = 0; j < l && j < n_levels; ++j) level_start += (int64_t)tiles[b] * side[j] * side[j];
+        const int64_t n_vis = l < n_levels ? (int64_t)tiles[b] * side[l] * side[l]
+                                           : (int64_t)tiles[b] * mixed_rows_per_tile;
         for (int64_t r = 0; r < n_vis; ++r, ++row)
             memcpy(out + row * C, pyr[b] + (level_start + r) * C, (size_t)C * 2);
         const int64_t n_text = (int64_t)prompt_len[b] + resp_len[b];
@@ -179,6 +185,16 @@ void oracle_gather(const uint16_t *const *pyr, const int32_t *tiles,
             memcpy(out + row * C, text + (text_off[b] + r) * C, (size_t)C * 2);
         cu[b + 1] = (int32_t)row;
     }
+}
+
+void oracle_gather(const uint16_t *const *pyr, const int32_t *tiles,
+                   const uint16_t *text, const int64_t *text_off,
+                   const int32_t *prompt_len, const int32_t *resp_len,
+                   const int32_t *level, int batch, int grid, int n_levels, int C,
+                   uint16_t *out, int32_t *cu)
+{
+    oracle_gather_mixed(pyr, tiles, text, text_off, prompt_len, resp_len, level, batch, grid, n_levels, C,
+                        0, out, cu);
 }
 
 /* -------------------------------------------------------------- attention */
@@ -463,4 +479,37 @@ int oracle_policy_view(double b)
     if (b < 1.0 / 3.0) return 0;
     if (b < 2.0 / 3.0) return 1;
     return 2;
+}
+
+/* ------------------------------------------------------------- mixed view */
+
+/*
+ * The `mixed` evidence view of Sec. 4.3: the pooled (`coarse`) representation
+ * augmented with a fixed subset of unpooled tokens.  Reading: per tile, all
+ * rows of pyramid level `coarse_level` (row-major), followed by the level-0
+ * tokens on a centred stride-`stride` lattice, (y, x) with
+ * y = stride/2 + i*stride < grid and x = stride/2 + j*stride < grid, row-major;
+ * tiles follow one another.  `pyr` is a level-major pyramid of n_tiles tiles
+ * (layout of oracle_pyramid_f64) holding bf16 bits; rows are copied bit for
+ * bit.  Returns the rows written (rows per tile times n_tiles).
+ */
+int64_t oracle_mixed_view(const uint16_t *pyr, int n_tiles, int grid, int n_levels, int coarse_level,
+                          int stride, int C, uint16_t *out)
+{
+    int side[32];
+    oracle_level_sides(grid, n_levels, side);
+    int64_t off[33];
+    off[0] = 0;
+    for (int l = 0; l < n_levels; ++l)
+        off[l + 1] = off[l] + (int64_t)n_tiles * side[l] * side[l];
+    const int gc = side[coarse_level];
+    int64_t row = 0;
+    for (int t = 0; t < n_tiles; ++t) {
+        for (int i = 0; i < gc * gc; ++i, ++row)
+            memcpy(out + row * C, pyr + (off[coarse_level] + (int64_t)t * gc * gc + i) * C, (size_t)C * 2);
+        for (int y = stride / 2; y < grid; y += stride)
+            for (int x = stride / 2; x < grid; x += stride, ++row)
+                memcpy(out + row * C, pyr + ((int64_t)t * grid * grid + (int64_t)y * grid + x) * C, (size_t)C * 2);
+    }
+    return row;
 }
