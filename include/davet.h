@@ -8,7 +8,8 @@
  * path that the policy drives:
  *
  *   davet_build_pyramid   the evidence hierarchy (Sec. 4.3), once per request
- *   davet_gather_view     the step input [view || prompt || answer] (Eq. 5)
+ *   davet_gather_view     the step input [view || prompt || answer] (Eq. 5),
+ *                         the view a pooled level or the mixed view
  *   davet_step_attention  bidirectional attention over it (Sec. 3.1, Eq. 1)
  *   davet_unmask_topk     argmax, confidence and confidence-ranked commit
  *                         (Sec. 3.1, Eq. 1-2) plus the mean confidence and
@@ -124,14 +125,34 @@ davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int g
                                  float* pyr_f32, void* stream);
 
 /*
+ * Host-only layout helper for the mixed evidence view (Sec. 4.3: the pooled
+ * representation augmented with a fixed subset of unpooled tokens).  The
+ * paper does not fix the subset; this library takes, per tile, every row of
+ * pyramid level mixed_level followed by the level-0 tokens of a centred
+ * stride-s lattice, (y, x) with y, x in {s/2, s/2 + s, s/2 + 2s, ...} below
+ * grid, in row-major order.
+ *   grid, n_levels   as for davet_pyramid_layout
+ *   mixed_level      the pooled level, 0 <= mixed_level < n_levels
+ *   mixed_stride     s, 1 <= s <= grid
+ *   rows_per_tile    out (nullable): G_{mixed_level}^2 + n^2 with
+ *                    n = ceil((grid - s/2) / s)
+ * Example: grid 27, 4 levels, level 2 and s = 3 give 49 + 81 = 130 rows.
+ */
+davet_status davet_mixed_view_rows(int grid, int n_levels, int mixed_level, int mixed_stride,
+                                   int* rows_per_tile);
+
+/*
  * Packs the input of one denoising step for a batch of requests (Eq. 5:
  * the step is conditioned on v_t = A(v; b_t), the view selected for the
  * step, together with the query and the current answer state).  For request
  * b the packed rows are
- *     [ all rows of level level_dev[b] of its pyramid (tiles in order)
+ *     [ all rows of view level_dev[b] of its pyramid (tiles in order)
  *       || its prompt_len_dev[b] prompt rows || its resp_len_dev[b] answer rows ]
- * and requests follow one another in batch order.  Rows are copied bit for
- * bit.  cu_seqlens_dev[b] receives the first packed row of request b and
+ * and requests follow one another in batch order.  View l < n_levels is
+ * pyramid level l; view n_levels is the mixed view of
+ * davet_mixed_view_rows (tile by tile, its rows are read straight from the
+ * pyramid, nothing is stored for it).  Rows are copied bit for bit.
+ * cu_seqlens_dev[b] receives the first packed row of request b and
  * cu_seqlens_dev[batch] the total row count.
  *   pyr_ptrs_dev     device array [batch] of device pointers to each
  *                    request's bf16 pyramid (davet_build_pyramid layout)
@@ -140,18 +161,21 @@ davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int g
  *                    contiguous from row text_off_dev[b] (int64 [batch])
  *   prompt_len_dev, resp_len_dev, level_dev   int32 [batch]
  *   grid, n_levels, C  as for davet_build_pyramid (shared by the batch)
+ *   mixed_level, mixed_stride  the mixed view (as for davet_mixed_view_rows);
+ *                    mixed_stride = 0 means the batch has no mixed view
  *   packed           bf16 [max_total_rows][C] output
  *   cu_seqlens_dev   int32 [batch+1] output
- * Device-side checks: a level outside [0, n_levels) or a negative count sets
- * DAVET_DEV_ARG and the request contributes no visual rows; a total above
+ * Device-side checks: a level outside [0, n_levels) (or [0, n_levels] with
+ * a mixed view) or a negative count sets DAVET_DEV_ARG and the request
+ * contributes no visual rows; a total above
  * max_total_rows sets DAVET_DEV_CAPACITY, rows beyond the capacity are not
  * written and cu_seqlens is clamped to max_total_rows.
  */
 davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* tiles_dev, const void* text,
                                const int64_t* text_off_dev, const int32_t* prompt_len_dev,
                                const int32_t* resp_len_dev, const int32_t* level_dev, int batch, int grid,
-                               int n_levels, int C, void* packed, int32_t* cu_seqlens_dev,
-                               int64_t max_total_rows, void* stream);
+                               int n_levels, int mixed_level, int mixed_stride, int C, void* packed,
+                               int32_t* cu_seqlens_dev, int64_t max_total_rows, void* stream);
 
 /* ------------------------------------------------------- step attention */
 
@@ -249,8 +273,9 @@ davet_status davet_policy_envelope(int T, int orientation, double B, double rho,
  *   (mean confidence over the positions still masked then, and churn);
  *   b_t = lower[t] + r (upper[t] - lower[t]);
  *   view = coarse if b_t < 1/3, mixed if b_t < 2/3, else high.
- *   view_level      host int32 [3]: pyramid level used for the coarse, mixed
- *                   and high views (level 0 is the full encoding)
+ *   view_level      host int32 [3]: view index of davet_gather_view used for
+ *                   the coarse, mixed and high views (level 0 is the full
+ *                   encoding; n_levels is the mixed view)
  *   level_out_dev   int32 [batch] out: the level for davet_gather_view
  *   budget_out_dev  double [batch] out, nullable: b_t
  * Computed in fp64.

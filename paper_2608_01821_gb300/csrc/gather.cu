@@ -7,6 +7,12 @@
 // shared memory (a block-wide scan; requests are few), then copies rows with
 // one warp per row: each lane moves 16-byte slices, eight loads in flight
 // before the matching stores, so a warp keeps 4 KB of one row in flight.
+//
+// The mixed view (Sec. 4.3: pooled tokens plus a fixed subset of unpooled
+// ones) is never materialized: level index n_levels selects it, and its
+// source rows are computed per packed row -- per tile, the rows of the
+// coarse level, then the level-0 tokens of a centred stride-s lattice
+// (y, x in {s/2, s/2 + s, ...}), row-major.
 #include <algorithm>
 
 #include "common.cuh"
@@ -23,6 +29,11 @@ struct Geom {
   int side[kMaxLevels];
   int n_levels;
   int C8;
+  // mixed view; stride == 0 when the caller has none
+  int mixed_level;   // coarse level of the mixed view
+  int mixed_stride;  // lattice stride s over the level-0 grid
+  int mixed_n;       // lattice points per side
+  int mixed_rows;    // rows per tile: side[mixed_level]^2 + mixed_n^2
 };
 
 struct Args {
@@ -52,6 +63,7 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
   long long* s_len = sm + a.batch + 1;      // [batch] packed rows of each request
   long long* s_nvis = s_len + a.batch;      // [batch] visual rows
   long long* s_vis0 = s_nvis + a.batch;     // [batch] first pyramid row of the chosen level
+                                            // (mixed view: of its coarse level, stored as -1 - row)
   __shared__ long long s_warp[kThreads / 32];
   __shared__ int s_bad;
 
@@ -71,8 +83,14 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
     const int p = a.prompt[b], r = a.resp[b];
     bool bad = false;
     long long nvis = 0, vis0 = 0;
-    if (lvl < 0 || lvl >= g.n_levels || nt < 0) {
+    const bool mixed = lvl == g.n_levels && g.mixed_stride > 0;
+    if (lvl < 0 || (lvl >= g.n_levels && !mixed) || nt < 0) {
       bad = true;
+    } else if (mixed) {
+      long long off = 0;
+      for (int l = 0; l < g.mixed_level; ++l) off += static_cast<long long>(nt) * g.side[l] * g.side[l];
+      vis0 = -1 - off;
+      nvis = static_cast<long long>(nt) * g.mixed_rows;
     } else {
       long long off = 0;
       for (int l = 0; l < lvl; ++l) off += static_cast<long long>(nt) * g.side[l] * g.side[l];
@@ -136,7 +154,25 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
     const long long j = row - s_cu[b];
     const uint4* src;
     if (j < s_nvis[b]) {
-      src = a.pyr[b] + (s_vis0[b] + j) * C8;
+      const long long v0 = s_vis0[b];
+      long long prow;
+      if (v0 >= 0) {
+        prow = v0 + j;
+      } else {
+        // mixed view: tile t, row r of the tile
+        const long long t = j / g.mixed_rows;
+        const int r = static_cast<int>(j - t * g.mixed_rows);
+        const long long gc2 = static_cast<long long>(g.side[g.mixed_level]) * g.side[g.mixed_level];
+        if (r < gc2) {
+          prow = (-1 - v0) + t * gc2 + r;
+        } else {
+          const int i = static_cast<int>(r - gc2);
+          const int iy = i / g.mixed_n, ix = i - iy * g.mixed_n;
+          const int s = g.mixed_stride, G = g.side[0];
+          prow = t * G * G + static_cast<long long>(s / 2 + iy * s) * G + (s / 2 + ix * s);
+        }
+      }
+      src = a.pyr[b] + prow * C8;
     } else {
       src = a.text + (a.text_off[b] + (j - s_nvis[b])) * C8;
     }
@@ -158,14 +194,17 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(Args a, Geom g) {
 extern "C" davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* tiles_dev,
                                           const void* text, const int64_t* text_off_dev,
                                           const int32_t* prompt_len_dev, const int32_t* resp_len_dev,
-                                          const int32_t* level_dev, int batch, int grid, int n_levels, int C,
-                                          void* packed, int32_t* cu_seqlens_dev, int64_t max_total_rows,
-                                          void* stream) {
+                                          const int32_t* level_dev, int batch, int grid, int n_levels,
+                                          int mixed_level, int mixed_stride, int C, void* packed,
+                                          int32_t* cu_seqlens_dev, int64_t max_total_rows, void* stream) {
   using namespace davet;
   using namespace davet::gat;
   if (batch < 0 || grid < 1 || n_levels < 1 || C < 8 || C % 8 != 0 || max_total_rows < 0)
     return DAVET_ERR_INVALID_ARG;
   if (n_levels > kMaxLevels || grid > 65536) return DAVET_ERR_UNSUPPORTED;
+  int mixed_rows = 0;
+  if (mixed_stride != 0 && davet_mixed_view_rows(grid, n_levels, mixed_level, mixed_stride, &mixed_rows) != DAVET_OK)
+    return DAVET_ERR_INVALID_ARG;
   if (batch > kMaxBatch) return DAVET_ERR_UNSUPPORTED;
   if (max_total_rows > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
   if (!cu_seqlens_dev) return DAVET_ERR_INVALID_ARG;
@@ -182,6 +221,10 @@ extern "C" davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const
   for (int l = 0; l < kMaxLevels; ++l) g.side[l] = l < n_levels ? side[l] : 1;
   g.n_levels = n_levels;
   g.C8 = C / 8;
+  g.mixed_level = mixed_stride ? mixed_level : 0;
+  g.mixed_stride = mixed_stride;
+  g.mixed_n = mixed_stride ? (grid - mixed_stride / 2 + mixed_stride - 1) / mixed_stride : 0;
+  g.mixed_rows = mixed_rows;
   Args a;
   a.pyr = reinterpret_cast<const uint4* const*>(pyr_ptrs_dev);
   a.tiles = tiles_dev;
@@ -204,4 +247,18 @@ extern "C" davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const
                                dim3(kThreads), smem, static_cast<cudaStream_t>(stream), a, g);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
+}
+
+extern "C" davet_status davet_mixed_view_rows(int grid, int n_levels, int mixed_level, int mixed_stride,
+                                              int* rows_per_tile) {
+  if (grid < 1 || grid > 65536 || n_levels < 1 || n_levels > davet::gat::kMaxLevels) return DAVET_ERR_INVALID_ARG;
+  if (mixed_level < 0 || mixed_level >= n_levels || mixed_stride < 1 || mixed_stride > grid)
+    return DAVET_ERR_INVALID_ARG;
+  int side[davet::gat::kMaxLevels];
+  davet_pyramid_layout(grid, n_levels, 0, side, nullptr);
+  const long long n = (grid - mixed_stride / 2 + mixed_stride - 1) / mixed_stride;
+  const long long rows = static_cast<long long>(side[mixed_level]) * side[mixed_level] + n * n;
+  if (rows > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
+  if (rows_per_tile) *rows_per_tile = static_cast<int>(rows);
+  return DAVET_OK;
 }

@@ -65,8 +65,9 @@ def _declare(lib):
         "davet_device_status": (_int, [ctypes.POINTER(ctypes.c_uint), _int]),
         "davet_pyramid_layout": (_int, [_int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_i64)]),
         "davet_build_pyramid": (_int, [_vp, _vp, _int, _int, _int, _int, _vp, _vp]),
-        "davet_gather_view": (_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _vp, _vp,
-                                     _i64, _vp]),
+        "davet_mixed_view_rows": (_int, [_int, _int, _int, _int, ctypes.POINTER(_int)]),
+        "davet_gather_view": (_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _vp,
+                                     _vp, _i64, _vp]),
         "davet_step_attention": (_int, [_vp, _vp, _int, _i64, _int, _int, _f32, _vp, _vp]),
         "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_unmask_topk": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
@@ -113,6 +114,12 @@ class Davet:
         self._check("davet_pyramid_layout", self.lib.davet_pyramid_layout(grid, n_levels, n_tiles, side, off))
         return list(side), list(off)
 
+    def davet_mixed_view_rows(self, grid: int, n_levels: int, mixed_level: int, mixed_stride: int) -> int:
+        n = _int(0)
+        self._check("davet_mixed_view_rows",
+                    self.lib.davet_mixed_view_rows(grid, n_levels, mixed_level, mixed_stride, ctypes.byref(n)))
+        return int(n.value)
+
     # ---------------------------------------------------------------- path
     def davet_build_pyramid(self, feat, pyr, n_tiles: int, grid: int, n_levels: int, C: int, pyr_f32=None,
                             stream=None):
@@ -121,12 +128,13 @@ class Davet:
                                                  _stream(stream)))
 
     def davet_gather_view(self, pyr_ptrs, tiles, text, text_off, prompt_len, resp_len, level, batch: int,
-                          grid: int, n_levels: int, C: int, packed, cu_seqlens, max_total_rows: int, stream=None):
+                          grid: int, n_levels: int, mixed_level: int, mixed_stride: int, C: int, packed, cu_seqlens,
+                          max_total_rows: int, stream=None):
         self._check("davet_gather_view",
                     self.lib.davet_gather_view(_ptr(pyr_ptrs), _ptr(tiles), _ptr(text), _ptr(text_off),
                                                _ptr(prompt_len), _ptr(resp_len), _ptr(level), batch, grid,
-                                               n_levels, C, _ptr(packed), _ptr(cu_seqlens), max_total_rows,
-                                               _stream(stream)))
+                                               n_levels, mixed_level, mixed_stride, C, _ptr(packed),
+                                               _ptr(cu_seqlens), max_total_rows, _stream(stream)))
 
     def davet_step_attention(self, qkv, cu_seqlens, batch: int, max_total_rows: int, H: int, D: int,
                              scale: float, out, stream=None):

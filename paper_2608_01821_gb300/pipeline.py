@@ -81,8 +81,8 @@ class Pipeline:
     def gather(self, t: int, stream=None):
         w = self.w
         self.lib.davet_gather_view(self.pyr_ptrs, self.tiles, self.text, self.text_off, self.prompt, self.resp,
-                                   self.schedule[t], w.batch, w.grid, w.n_levels, w.C, self.packed, self.cu,
-                                   self.max_rows, stream)
+                                   self.schedule[t], w.batch, w.grid, w.n_levels, *w.mixed_args, w.C,
+                                   self.packed, self.cu, self.max_rows, stream)
 
     def attention(self, stream=None):
         w = self.w

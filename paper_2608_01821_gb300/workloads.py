@@ -22,6 +22,13 @@ dimension 128 and 384px tiles of 27x27 visual tokens):
            U{64..512}, 128 steps, level drawn per (step, request) from
            {0,1,2,3} with p = [0.25, 0.25, 0.30, 0.20], top-2, seed 4
 
+Two more exercise the mixed view (coarse level 2 plus a centred stride-3
+lattice of level-0 tokens, selected as view index n_levels):
+
+  tiny_mixed    tiny with views [0,0,3,3,2,2,3,0] (3 = mixed, 25 rows)
+  single_mixed  single with coarse / mixed / high thirds over 64 steps
+                (49 / 130 / 729 visual rows)
+
 Per-token channel count C = 3*H*D: each visual and text row carries the
 packed [query | key | value] projections of its token, so a gathered row is
 exactly one row of the attention input (pooling commutes with the linear
@@ -99,6 +106,9 @@ class Workload:
     V: int
     k: int
     seed: int
+    # mixed view (coarse pyramid level, lattice stride), selected as view
+    # index n_levels; None when the workload has no mixed view
+    mixed: tuple[int, int] | None = None
 
     @property
     def C(self) -> int:
@@ -118,15 +128,32 @@ class Workload:
     def pyramid_rows(self, b: int) -> int:
         return self.tiles[b] * sum(g * g for g in self.level_sides())
 
+    @property
+    def mixed_args(self) -> tuple[int, int]:
+        """(mixed_level, mixed_stride) as the gather takes them; (0, 0) = none."""
+        return self.mixed if self.mixed else (0, 0)
+
+    def view_rows_per_tile(self, level: int) -> int:
+        """Rows per tile of view `level`: a pyramid level, or the mixed view
+        (index n_levels): the coarse level plus the centred lattice."""
+        if level < self.n_levels:
+            return self.level_sides()[level] ** 2
+        assert level == self.n_levels and self.mixed, level
+        coarse, s = self.mixed
+        n = len(range(s // 2, self.grid, s))
+        return self.level_sides()[coarse] ** 2 + n * n
+
+    def n_views(self) -> int:
+        return self.n_levels + (1 if self.mixed else 0)
+
     def seq_len(self, b: int, level: int) -> int:
-        g = self.level_sides()[level]
-        return self.tiles[b] * g * g + self.prompt[b] + self.resp[b]
+        return self.tiles[b] * self.view_rows_per_tile(level) + self.prompt[b] + self.resp[b]
 
     def step_lengths(self, t: int) -> list[int]:
         return [self.seq_len(b, int(self.schedule[t, b])) for b in range(self.batch)]
 
     def max_total_rows(self) -> int:
-        return sum(self.seq_len(b, 0) for b in range(self.batch))
+        return sum(max(self.seq_len(b, v) for v in range(self.n_views())) for b in range(self.batch))
 
     @property
     def total_resp(self) -> int:
@@ -204,10 +231,24 @@ def make(name: str) -> Workload:
                 sched[t, b] = next(i for i, c in enumerate(cum) if u < c)
         return Workload("ragged", 16, 32, 128, 27, 4, tiles, prompt, resp, 128, sched,
                         VOCAB_8B, 2, 4)
+    if name == "tiny_mixed":
+        # coarse (level 2, 9 rows), mixed (index 3: level 2 + the 4x4 lattice of
+        # stride 3, 25 rows) and high (level 0, 144 rows)
+        return Workload("tiny_mixed", 1, 4, 64, 12, 3, [1], [16], [32], 8,
+                        np.array([[0], [0], [3], [3], [2], [2], [3], [0]], dtype=np.int32),
+                        1024, 4, 0, mixed=(2, 3))
+    if name == "single_mixed":
+        # the three-view hierarchy on one 27x27 tile: coarse (level 2, 49 rows)
+        # for t < 22, mixed (index 4: level 2 + the 9x9 lattice of stride 3,
+        # 130 rows) for t < 43, then high (level 0, 729 rows)
+        return Workload("single_mixed", 1, 32, 128, 27, 4, [1], [64], [128], 64,
+                        _sched_const(64, 1, lambda t: 2 if t < 22 else (4 if t < 43 else 0)), VOCAB_8B, 2, 1,
+                        mixed=(2, 3))
     raise ValueError(f"unknown workload {name!r}")
 
 
 NAMES = ("tiny", "single", "anyres", "highres", "ragged")
+MIXED_NAMES = ("tiny_mixed", "single_mixed")
 
 
 # ------------------------------------------------------------ value sources

@@ -49,6 +49,21 @@ def test_pyramid_layout_matches_oracle(lib, grid, levels, tiles):
     assert list(off) == oracle.level_offsets(grid, levels, tiles)
 
 
+@pytest.mark.parametrize("grid,levels,mixed_level,stride", [(27, 4, 2, 3), (27, 4, 3, 4), (12, 3, 2, 3), (5, 3, 1, 1),
+                                                             (27, 4, 0, 27), (1, 1, 0, 1)])
+def test_mixed_view_rows_matches_oracle(lib, grid, levels, mixed_level, stride):
+    n = ctypes.c_int(-1)
+    assert lib.davet_mixed_view_rows(grid, levels, mixed_level, stride, ctypes.byref(n)) == 0
+    assert n.value == oracle.mixed_rows_per_tile(grid, levels, mixed_level, stride)
+
+
+def test_mixed_view_rows_rejects_out_of_range(lib):
+    n = ctypes.c_int(-1)
+    for args in [(27, 4, 4, 3), (27, 4, -1, 3), (27, 4, 2, 0), (27, 4, 2, 28), (27, 6, 2, 3), (0, 4, 0, 1)]:
+        assert lib.davet_mixed_view_rows(*args, ctypes.byref(n)) == 1
+    assert n.value == -1
+
+
 def test_invalid_arguments_are_rejected_without_a_device(lib):
     INV, UNS = 1, 2
     p = ctypes.c_void_p(1 << 20)  # never dereferenced: validation fails first
@@ -69,8 +84,12 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_step_attention(p, p, 2000, 128, 4, 64, f(0.1), p, null) == UNS
     assert lib.davet_step_attention(p, p, 0, 128, 4, 64, f(0.1), p, null) == 0  # empty batch
     # gather: bad levels count, batch too large
-    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 16, p, p, 100, null) == INV
-    assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 16, p, p, 100, null) == UNS
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 0, 0, 16, p, p, 100, null) == INV
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 0, 0, 16, p, p, 100, null) == UNS
+    # gather: mixed view with a level or stride out of range
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 4, 4, 3, 16, p, p, 100, null) == INV
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 4, 2, 28, 16, p, p, 100, null) == INV
+    assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 4, 2, -1, 16, p, p, 100, null) == INV
     # unmask: k out of range, V not a multiple of 8, workspace too small
     n = ctypes.c_size_t(0)
     assert lib.davet_unmask_topk_workspace(128, 1000, 1, ctypes.byref(n)) == 0 and n.value > 0

@@ -40,7 +40,7 @@ def setup(davet, tiles, prompt, resp, grid, levels, C, seed):
     return d
 
 
-def run(davet, d, level, grid, levels, C, cap):
+def run(davet, d, level, grid, levels, C, cap, mixed=(0, 0)):
     dev = torch.device("cuda")
     B = len(level)
     # 64 guard rows past the capacity must stay untouched
@@ -48,7 +48,7 @@ def run(davet, d, level, grid, levels, C, cap):
     cu = torch.full((B + 1,), -5, dtype=torch.int32, device=dev)
     lv = torch.tensor(level, dtype=torch.int32, device=dev)
     davet.davet_gather_view(d["pyr_ptrs"], d["tiles"], d["text"], d["text_off"], d["prompt"], d["resp"], lv, B,
-                            grid, levels, C, packed, cu, cap)
+                            grid, levels, *mixed, C, packed, cu, cap)
     torch.cuda.synchronize()
     assert torch.isnan(packed[cap:].float()).all()
     return packed[:cap], cu
@@ -103,3 +103,61 @@ def test_level_out_of_range_is_flagged(davet):
     st, flags = davet.davet_device_status(clear=True)
     assert flags & 0x4
     assert list(cu.cpu().numpy()) == [0, 20, 20 + 196 + 20]
+
+
+def with_mixed(pyr, tiles, grid, levels, C, mixed):
+    """Oracle-side buffer: the pyramid followed by its materialized mixed view."""
+    p = bits(pyr)
+    if tiles == 0:
+        return p
+    return np.concatenate([p[: oracle.level_offsets(grid, levels, tiles)[-1]],
+                           oracle.mixed_view(pyr.cpu(), tiles, grid, levels, *mixed, C)])
+
+
+@pytest.mark.parametrize("level,mixed", [([4, 0, 4], (2, 3)), ([1, 4, 3], (2, 3)), ([4, 4, 2], (3, 4)),
+                                         ([4, 4, 4], (0, 27)), ([4, 2, 4], (1, 1))])
+def test_mixed_view_bit_exact(davet, level, mixed):
+    """The mixed view (Sec. 4.3) is gathered from the pyramid without being
+    stored; the oracle materializes it and gathers it as one more level."""
+    grid, levels, C = 27, 4, 256
+    tiles, prompt, resp = [2, 1, 3], [5, 0, 17], [9, 3, 0]
+    d = setup(davet, tiles, prompt, resp, grid, levels, C, 5)
+    mrows = davet.davet_mixed_view_rows(grid, levels, *mixed)
+    assert mrows == oracle.mixed_rows_per_tile(grid, levels, *mixed)
+    cap = sum(t * max(729, mrows) + p + r for t, p, r in zip(tiles, prompt, resp))
+    packed, cu = run(davet, d, level, grid, levels, C, cap, mixed)
+    assert davet.davet_device_status() == (0, 0)
+    pyrs = [with_mixed(p, t, grid, levels, C, mixed) for p, t in zip(d["pyrs"], tiles)]
+    ref, ref_cu = oracle.gather(pyrs, tiles, d["text"].cpu(), d["text_off_np"], prompt, resp, level, grid, levels,
+                                C, mixed_rows_per_tile=mrows)
+    assert list(cu.cpu().numpy()) == list(ref_cu)
+    assert np.array_equal(bits(packed[: int(ref_cu[-1])]), ref)
+
+
+def test_mixed_view_full_width_tiny_grid(davet):
+    """Odd channel tail (C/8 not a multiple of 32 lanes) on the 12x12 grid
+    with coarse level 2 and stride 3: 9 + 16 rows per tile."""
+    grid, levels, C = 12, 3, 768 + 8
+    tiles, prompt, resp = [1, 2], [16, 3], [32, 1]
+    d = setup(davet, tiles, prompt, resp, grid, levels, C, 6)
+    mixed = (2, 3)
+    assert davet.davet_mixed_view_rows(grid, levels, *mixed) == 25
+    cap = sum(t * 144 + p + r for t, p, r in zip(tiles, prompt, resp))
+    packed, cu = run(davet, d, [3, 3], grid, levels, C, cap, mixed)
+    assert davet.davet_device_status() == (0, 0)
+    pyrs = [with_mixed(p, t, grid, levels, C, mixed) for p, t in zip(d["pyrs"], tiles)]
+    ref, ref_cu = oracle.gather(pyrs, tiles, d["text"].cpu(), d["text_off_np"], prompt, resp, [3, 3], grid, levels,
+                                C, mixed_rows_per_tile=25)
+    assert list(cu.cpu().numpy()) == [0, 25 + 48, 25 + 48 + 50 + 4] == list(ref_cu)
+    assert np.array_equal(bits(packed[: int(ref_cu[-1])]), ref)
+
+
+def test_mixed_index_without_a_mixed_view_is_flagged(davet):
+    grid, levels, C = 27, 4, 64
+    tiles, prompt, resp = [1, 1], [10, 10], [10, 10]
+    d = setup(davet, tiles, prompt, resp, grid, levels, C, 7)
+    davet.davet_device_status(clear=True)
+    packed, cu = run(davet, d, [4, 2], grid, levels, C, 2000)
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags & 0x4
+    assert list(cu.cpu().numpy()) == [0, 20, 20 + 49 + 20]

@@ -32,8 +32,21 @@ def oracle_pyramids(w, feats):
     return out
 
 
-def test_tiny_workload_every_step(davet):
-    w = workloads.make("tiny")
+def oracle_gather_inputs(w, gpu_pyr):
+    """Per-request buffers for the oracle gather: the pyramid, followed by
+    the oracle's materialized mixed view when the workload has one."""
+    if not w.mixed:
+        return gpu_pyr, 0
+    out = []
+    for b, p in enumerate(gpu_pyr):
+        mv = oracle.mixed_view(p, w.tiles[b], w.grid, w.n_levels, *w.mixed, w.C)
+        out.append(np.concatenate([bits(p), mv]))
+    return out, w.view_rows_per_tile(w.n_levels)
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_mixed"])
+def test_tiny_workload_every_step(davet, name):
+    w = workloads.make(name)
     pl, feats, text = make_pipeline(davet, w)
     pyr_ref = oracle_pyramids(w, feats)
     # the GPU pyramid rounds the same values: compare it bitwise through the
@@ -43,6 +56,7 @@ def test_tiny_workload_every_step(davet):
     for b in range(w.batch):
         diff = (gpu_pyr[b].float() - pyr_ref[b].float()).abs()
         assert float(diff.max()) <= 2 ** -7  # at most one bf16 step on |x| < 2
+    oracle_pyr, mrows = oracle_gather_inputs(w, gpu_pyr)
     masked = np.ones(w.total_resp, np.uint8)
     tokens = np.full(w.total_resp, -1, np.int32)
     argmax = np.full(w.total_resp, -1, np.int32)
@@ -52,8 +66,8 @@ def test_tiny_workload_every_step(davet):
         pl.step(t, lg.cuda())
         torch.cuda.synchronize()
         assert davet.davet_device_status() == (0, 0)
-        packed_ref, cu_ref = oracle.gather(gpu_pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp,
-                                           w.schedule[t], w.grid, w.n_levels, w.C)
+        packed_ref, cu_ref = oracle.gather(oracle_pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp,
+                                           w.schedule[t], w.grid, w.n_levels, w.C, mixed_rows_per_tile=mrows)
         N = int(cu_ref[-1])
         assert list(pl.cu.cpu().numpy()) == list(cu_ref)
         assert np.array_equal(bits(pl.packed[:N]), packed_ref)
@@ -73,7 +87,7 @@ def test_tiny_workload_every_step(davet):
     assert masked.sum() == 0
 
 
-@pytest.mark.parametrize("name", ["single", "anyres", "highres", "ragged"])
+@pytest.mark.parametrize("name", ["single", "anyres", "highres", "ragged", "single_mixed"])
 def test_workload_sampled_steps(davet, name):
     """Full-size inputs in the benchmark's launch configuration: the gather is
     compared bit for bit at one step per distinct level, attention on sampled
@@ -81,6 +95,7 @@ def test_workload_sampled_steps(davet, name):
     w = workloads.make(name)
     pl, feats, text = make_pipeline(davet, w)
     gpu_pyr = [v.cpu() for v in pl.pyr_views]
+    oracle_pyr, mrows = oracle_gather_inputs(w, gpu_pyr)
     # pyramid: one request, first tile, all levels against the oracle
     side = w.level_sides()
     ref_off = oracle.level_offsets(w.grid, w.n_levels, 1)
@@ -110,8 +125,8 @@ def test_workload_sampled_steps(davet, name):
             pl.unmask(t, lg_dev)
         torch.cuda.synchronize()
         assert davet.davet_device_status() == (0, 0)
-        packed_ref, cu_ref = oracle.gather(gpu_pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp,
-                                           w.schedule[t], w.grid, w.n_levels, w.C)
+        packed_ref, cu_ref = oracle.gather(oracle_pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp,
+                                           w.schedule[t], w.grid, w.n_levels, w.C, mixed_rows_per_tile=mrows)
         N = int(cu_ref[-1])
         assert list(pl.cu.cpu().numpy()) == list(cu_ref)
         assert np.array_equal(bits(pl.packed[:N]), packed_ref)

@@ -108,11 +108,14 @@ def test_step_matches_oracle_risk_budget_and_view(davet):
                 assert got_l[b] == view_level[oracle.policy_view(want)]
 
 
-def test_closed_loop_tiny_workload(davet):
-    """The policy picks every step's level on the device from the previous
+@pytest.mark.parametrize("name,view_level", [("tiny", [2, 1, 0]), ("tiny_mixed", [2, 3, 0])])
+def test_closed_loop_tiny_workload(davet, name, view_level):
+    """The policy picks every step's view on the device from the previous
     step's unmasking statistics; the oracle policy fed the same statistics
-    picks the same levels, and the mean budget stays below B (Eq. 4)."""
-    w = workloads.make("tiny")
+    picks the same views, and the mean budget stays below B (Eq. 4).  With
+    the mixed view the three views are those of Sec. 4.3: coarse (level 2),
+    mixed (view index 3) and high (level 0)."""
+    w = workloads.make(name)
     pl = Pipeline(w, "cuda", davet)
     pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w))
     pl.build_pyramids()
@@ -120,7 +123,6 @@ def test_closed_loop_tiny_workload(davet):
     lo = torch.empty((1, w.T), dtype=torch.float64, device="cuda")
     up = torch.empty_like(lo)
     davet.davet_policy_envelope(w.T, 1, B, rho, torch.tensor([d], dtype=torch.float64, device="cuda"), 1, lo, up)
-    view_level = [2, 1, 0]  # coarse, mixed, high -> pyramid levels of the 12/6/3 grid
     level = torch.zeros((w.T, 1), dtype=torch.int32, device="cuda")
     budget = torch.zeros((w.T, 1), dtype=torch.float64, device="cuda")
     for t in range(w.T):

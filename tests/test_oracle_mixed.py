@@ -72,3 +72,13 @@ def test_gather_selects_the_mixed_view_as_level_n_levels():
                                levels, C, mixed_rows_per_tile=mrows)
     assert list(cu) == [0, n_tiles * mrows + 3, n_tiles * mrows + 3 + n_tiles * 729 + 4]
     np.testing.assert_array_equal(packed[:n_tiles * mrows], mixed)
+
+
+def test_mixed_workloads_view_rows():
+    from paper_2608_01821_gb300 import workloads
+    for name in workloads.MIXED_NAMES:
+        w = workloads.make(name)
+        assert w.view_rows_per_tile(w.n_levels) == oracle.mixed_rows_per_tile(w.grid, w.n_levels, *w.mixed)
+        assert set(np.unique(w.schedule)) <= set(range(w.n_views()))
+    w = workloads.make("single_mixed")
+    assert [w.seq_len(0, v) for v in (2, 4, 0)] == [49 + 192, 130 + 192, 729 + 192]
