@@ -234,7 +234,9 @@ davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, s
  *                 committed this step in rank order, -1 padded
  *   stats_dev     float [batch][2], nullable: (mean conf over M_t, churn)
  *   workspace     device scratch of davet_unmask_topk_workspace() bytes;
- *                 calls that may run concurrently need separate workspaces
+ *                 its contents need no initialization (a call writes every
+ *                 entry it reads); calls that may run concurrently need
+ *                 separate workspaces
  * Device-side checks: request boundaries outside [0, total_rows] set
  * DAVET_DEV_ARG and are clamped.
  */
@@ -303,7 +305,7 @@ davet_status davet_policy_step(int t, int T, const double* lower_dev, const doub
  * until the process exits.  The call allocates nothing.
  *   - Limit: sizes whose workspace (davet_unmask_topk_workspace) exceeds
  *     DAVET_NOALLOC_SCRATCH_BYTES are rejected with DAVET_ERR_UNSUPPORTED
- *     before anything is enqueued (about 43,000 answer rows at V = 126464).
+ *     before anything is enqueued (about 43,000 answer rows).
  *   - Set-up: the first call on each device looks up the array's device
  *     address (cudaGetSymbolAddress) with that device current and caches it;
  *     make that first call before any stream capture.

@@ -2,15 +2,22 @@
 // Eq. 1-2) and the step statistics that feed the trajectory risk (Eq. 7).
 //
 // Two kernels:
-//  1. row pass: each (masked row, vocabulary split) is one block that streams
-//     its slice of bf16 logits once with 128-bit loads and keeps, per thread,
-//     an online (max, sum of 2^(x*log2e - max*log2e), first argmax) triple;
-//     triples merge with warp shuffles and shared memory into one partial per
-//     (row, split) in the workspace.
-//  2. select: one block per request merges the splits of its masked rows
-//     into (argmax, conf = 1/sum), counts churn against the previous argmax,
-//     then takes the top-k rows by (conf desc, position asc) with k rounds
-//     of a block-wide arg-max and commits them.
+//  1. row kernel: every (answer row, 8 KB vocabulary chunk) is one warp.
+//     A warp of a masked row streams its chunk of bf16 logits once with 128-bit
+//     loads (eight in flight per lane) and keeps, per lane, an online
+//     (max, sum of 2^(x*log2e - max*log2e), first argmax) triple, merged by
+//     shuffles and written to the workspace.  Independent warps keep many
+//     loads in flight per SM and hide each other's latencies.
+//  2. select: one CTA per request.  Each thread combines one row's chunk
+//     triples (stored chunk-major, so the loads coalesce; one round of
+//     loads) into (argmax, conf = 1/sum) held in shared memory, counting
+//     churn against the previous argmax; after one barrier, warp 0 forms
+//     the mean confidence and takes the top-k rows by (conf desc, position
+//     asc) with k rounds of a warp arg-max, and commits them.
+// Both kernels are latency-bound at small sizes: a dependent round trip to
+// L2 costs about half a microsecond here, so every load a kernel needs is
+// issued in one batch, without branches between the loads.
+
 #include <algorithm>
 #include <climits>
 #include <mutex>
@@ -20,61 +27,88 @@
 namespace davet {
 namespace unm {
 
-constexpr int kRowThreads = 256;
-constexpr int kSelThreads = 256;
+constexpr int kRowThreads = 256;  // 8 warps, one (row, chunk) unit each
+constexpr int kMaxChunks = 64;
+constexpr int kLoads = 8;         // 16-byte loads in flight per lane
+constexpr int kSelThreads = 256;  // one answer row per thread and pass
+constexpr int kSelSmemRows = 4096;
 constexpr float kLog2e = 1.4426950408889634f;
 
-struct Partial {
-  float m;    // max logit * log2(e)
-  float s;    // sum of 2^(x*log2e - m)
+struct __align__(16) Partial {
+  float m;    // max logit (raw, bf16-exact)
+  float s;    // sum of 2^(x*log2e - m*log2e)
   int idx;    // first index attaining the max
   int pad;
 };
 
 struct Layout {
-  int nsplit;
+  int nchunk;  // vocabulary chunks per row (one warp each)
   size_t off_partial, off_conf, off_idx, bytes;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-inline Layout layout_for(int64_t total_rows, int V, int batch = 0) {
+// Chunks of 512 slices (8 KB: two rounds of loads per lane), at most
+// kMaxChunks per row; when `max_bytes` is given (the allocation-free path),
+// fewer and longer chunks so that the layout fits.  The conf / argmax
+// arrays serve requests longer than kSelSmemRows rows.
+inline Layout layout_for(int64_t total_rows, int V, size_t max_bytes = ~size_t(0)) {
   Layout L;
   const int64_t v8 = V / 8;
-  // about six waves of 8 blocks per SM when every row is masked, so the grid
-  // keeps a short tail as rows are committed; each split keeps at least 1024
-  // 16-byte slices (16 KB) so the block-level merge stays cheap
-  int64_t want = total_rows > 0 ? (152 * 8 * 6 + total_rows - 1) / total_rows : 1;
-  const int64_t cap = std::max<int64_t>(1, v8 / 1024);
-  L.nsplit = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(want, cap), 64)));
+  const size_t rows = static_cast<size_t>(total_rows);
+  const size_t fixed = align256(rows * sizeof(float)) + align256(rows * sizeof(int32_t));
+  int64_t nchunk = std::max<int64_t>(1, std::min<int64_t>(kMaxChunks, (v8 + 511) / 512));
+  while (nchunk > 1 && align256(rows * nchunk * sizeof(Partial)) + fixed > max_bytes) --nchunk;
+  L.nchunk = static_cast<int>(nchunk);
   L.off_partial = 0;
-  L.off_conf = align256(static_cast<size_t>(total_rows) * L.nsplit * sizeof(Partial));
-  L.off_idx = L.off_conf + align256(static_cast<size_t>(total_rows) * sizeof(float));
-  L.bytes = L.off_idx + align256(static_cast<size_t>(total_rows) * sizeof(int));
-  (void)batch;
+  L.off_conf = align256(rows * L.nchunk * sizeof(Partial));
+  L.off_idx = L.off_conf + align256(rows * sizeof(float));
+  L.bytes = L.off_idx + align256(rows * sizeof(int32_t));
   return L;
 }
 
-__device__ __forceinline__ Partial merge(Partial a, Partial b) {
+// 2^x on the SFU; not volatile, so the compiler may interleave it
+__device__ __forceinline__ float sfu_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Warp-wide combination of the lanes' triples in two passes instead of
+// pairwise merges: the warp max M by shuffles, one rescale 2^((m - M)log2e)
+// per lane, then a shuffle sum and the smallest index among lanes at M.
+// Every lane returns the result.
+__device__ __forceinline__ Partial warp_combine(Partial p) {
+  float mx = p.m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float sm = p.s > 0.f ? p.s * sfu_ex2((p.m - mx) * kLog2e) : 0.f;
+  int ix = p.m == mx ? p.idx : INT_MAX;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sm += __shfl_xor_sync(0xffffffffu, sm, o);
+    ix = min(ix, __shfl_xor_sync(0xffffffffu, ix, o));
+  }
   Partial r;
-  r.m = fmaxf(a.m, b.m);
-  const float sa = a.s > 0.f ? a.s * ex2(a.m - r.m) : 0.f;
-  const float sb = b.s > 0.f ? b.s * ex2(b.m - r.m) : 0.f;
-  r.s = sa + sb;
-  r.idx = a.m > b.m ? a.idx : (b.m > a.m ? b.idx : min(a.idx, b.idx));
+  r.m = mx;
+  r.s = sm;
+  r.idx = ix;
   r.pad = 0;
   return r;
 }
 
-__device__ __forceinline__ Partial shfl_merge(Partial p) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    Partial q;
-    q.m = __shfl_xor_sync(0xffffffffu, p.m, o);
-    q.s = __shfl_xor_sync(0xffffffffu, p.s, o);
-    q.idx = __shfl_xor_sync(0xffffffffu, p.idx, o);
-    p = merge(p, q);
-  }
+__device__ __forceinline__ Partial empty_partial() {
+  Partial p;
+  p.m = -INFINITY;
+  p.s = 0.f;
+  p.idx = INT_MAX;
+  p.pad = 0;
   return p;
 }
 
@@ -86,79 +120,112 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
   return v;
 }
 
-// Fold one 16-byte slice (8 logits starting at vocabulary index w0) into p.
-__device__ __forceinline__ void fold(Partial& p, uint4 u, int w0) {
-  float x[8];
-  x[0] = bf16lo(u.x) * kLog2e; x[1] = bf16hi(u.x) * kLog2e;
-  x[2] = bf16lo(u.y) * kLog2e; x[3] = bf16hi(u.y) * kLog2e;
-  x[4] = bf16lo(u.z) * kLog2e; x[5] = bf16hi(u.z) * kLog2e;
-  x[6] = bf16lo(u.w) * kLog2e; x[7] = bf16hi(u.w) * kLog2e;
-  float vm = x[0];
-#pragma unroll
-  for (int k = 1; k < 8; ++k) vm = fmaxf(vm, x[k]);
-  if (vm > p.m) {
-    int first = 7;
-#pragma unroll
-    for (int k = 6; k >= 0; --k) first = (x[k] == vm) ? k : first;
-    p.idx = w0 + first;
-    p.s = p.s > 0.f ? p.s * ex2(p.m - vm) : 0.f;
-    p.m = vm;
-  }
-  // pairwise sum of the eight terms, then one add into the running sum
-  float e[8];
-#pragma unroll
-  for (int k = 0; k < 8; ++k) e[k] = ex2(x[k] - p.m);
-  p.s += ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+// A lane's running state: max m (raw), m * log2e, first argmax, and the sum
+// of 2^(x*log2e - m*log2e) in two accumulators (one per element parity).
+struct Run {
+  float m, ml, s0, s1;
+  int idx;
+};
+
+__device__ __forceinline__ Run empty_run() {
+  Run r;
+  r.m = -INFINITY;
+  r.ml = -INFINITY;
+  r.s0 = 0.f;
+  r.s1 = 0.f;
+  r.idx = INT_MAX;
+  return r;
 }
 
-__global__ void __launch_bounds__(kRowThreads) row_pass(const uint4* __restrict__ logits, int V8,
-                                                        const uint8_t* __restrict__ masked, long long total_rows,
-                                                        int nsplit, Partial* __restrict__ out) {
+// Fold one 16-byte slice (8 logits starting at vocabulary index w0) into r:
+// the slice's max comes from packed bf16 maxima; only a new running max
+// (rare after the first slices) takes the branch that finds its first
+// index and rescales the sums.  Each pair of terms costs one packed FMA,
+// two SFU exponentials and one packed add.
+__device__ __forceinline__ void fold(Run& r, uint4 u, int w0) {
+  const uint32_t mx = max_bf16x2(max_bf16x2(u.x, u.y), max_bf16x2(u.z, u.w));
+  const float vm = fmaxf(bf16lo(mx), bf16hi(mx));
+  if (vm > r.m) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    int first = 7;
+#pragma unroll
+    for (int k = 7; k >= 0; --k) {
+      const float xk = (k & 1) ? bf16hi(w[k >> 1]) : bf16lo(w[k >> 1]);
+      first = (xk == vm) ? k : first;
+    }
+    r.idx = w0 + first;
+    const float ml = vm * kLog2e;
+    const float f = r.s0 + r.s1 > 0.f ? sfu_ex2(r.ml - ml) : 0.f;
+    r.s0 *= f;
+    r.s1 *= f;
+    r.m = vm;
+    r.ml = ml;
+  }
+  const float nm = -r.ml;
+  float a[8];
+  ffma2(a[0], a[1], bf16lo(u.x), bf16hi(u.x), kLog2e, kLog2e, nm, nm);
+  ffma2(a[2], a[3], bf16lo(u.y), bf16hi(u.y), kLog2e, kLog2e, nm, nm);
+  ffma2(a[4], a[5], bf16lo(u.z), bf16hi(u.z), kLog2e, kLog2e, nm, nm);
+  ffma2(a[6], a[7], bf16lo(u.w), bf16hi(u.w), kLog2e, kLog2e, nm, nm);
+  float e[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) e[k] = sfu_ex2(a[k]);
+  float t0, t1, t2, t3;
+  fadd2(t0, t1, e[0], e[1], e[2], e[3]);
+  fadd2(t2, t3, e[4], e[5], e[6], e[7]);
+  fadd2(t0, t1, t0, t1, t2, t3);
+  fadd2(r.s0, r.s1, r.s0, r.s1, t0, t1);
+}
+
+__device__ __forceinline__ Partial to_partial(const Run& r) {
+  Partial p;
+  p.m = r.m;
+  p.s = r.s0 + r.s1;
+  p.idx = r.idx;
+  p.pad = 0;
+  return p;
+}
+
+struct RowArgs {
+  const uint4* logits;
+  int V8;
+  int nchunk;
+  int chunk;  // 16-byte slices per chunk
+  long long total_rows;
+  const uint8_t* masked;
+  Partial* partial;  // [nchunk][rows]
+};
+
+__global__ void __launch_bounds__(kRowThreads) row_kernel(RowArgs a) {
   pdl_launch_dependents();
   pdl_wait();
-  const long long item = blockIdx.x;
-  const long long row = item / nsplit;
-  const int split = static_cast<int>(item - row * nsplit);
-  if (row >= total_rows || !masked[row]) return;
-  const int per = (V8 + nsplit - 1) / nsplit;
-  const int lo = split * per, hi = min(V8, lo + per);
-  const uint4* base = logits + row * static_cast<long long>(V8);
-  Partial p;
-  p.m = -INFINITY;
-  p.s = 0.f;
-  p.idx = INT_MAX;
-  p.pad = 0;
-  int v = lo + threadIdx.x;
-  for (; v + 3 * kRowThreads < hi; v += 4 * kRowThreads) {
-    uint4 u[4];
+  const long long unit = (static_cast<long long>(blockIdx.x) * kRowThreads + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (unit >= a.total_rows * a.nchunk) return;
+  const long long row = unit / a.nchunk;
+  if (!a.masked[row]) return;
+  const int ch = static_cast<int>(unit - row * a.nchunk);
+  const int lo = ch * a.chunk, hi = min(a.V8, lo + a.chunk);
+  const uint4* base = a.logits + row * static_cast<long long>(a.V8);
+  Run run = empty_run();
+  // every load of an iteration is issued before the first fold
+  for (int v = lo + lane; v < hi; v += 32 * kLoads) {
+    uint4 u[kLoads];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) u[k] = ld_stream(base + v + k * kRowThreads);
+    for (int k = 0; k < kLoads; ++k)
+      if (v + 32 * k < hi) u[k] = ld_stream(base + v + 32 * k);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) fold(p, u[k], (v + k * kRowThreads) * 8);
+    for (int k = 0; k < kLoads; ++k)
+      if (v + 32 * k < hi) fold(run, u[k], (v + 32 * k) * 8);
   }
-  for (; v < hi; v += kRowThreads) fold(p, ld_stream(base + v), v * 8);
-
-  // block merge: warps, then warp 0 over the warp results
-  __shared__ Partial s_p[kRowThreads / 32];
-  p = shfl_merge(p);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane == 0) s_p[warp] = p;
-  __syncthreads();
-  if (warp == 0) {
-    Partial q;
-    if (lane < kRowThreads / 32) {
-      q = s_p[lane];
-    } else {
-      q.m = -INFINITY; q.s = 0.f; q.idx = INT_MAX; q.pad = 0;
-    }
-    q = shfl_merge(q);
-    if (lane == 0) out[item] = q;
-  }
+  const Partial p = warp_combine(to_partial(run));
+  // chunk-major, so the select's row-per-thread loads are coalesced
+  if (lane == 0) a.partial[static_cast<long long>(ch) * a.total_rows + row] = p;
 }
 
 struct SelArgs {
   const Partial* partial;
-  int nsplit;
+  int nchunk;
   const int32_t* cu;
   int batch;
   long long total_rows;
@@ -169,85 +236,123 @@ struct SelArgs {
   float* conf_out;
   int32_t* committed;
   float* stats;
-  float* row_conf;  // workspace: conf of masked rows
-  int32_t* row_idx; // workspace: argmax of masked rows
+  float* row_conf;   // workspace for requests longer than kSelSmemRows
+  int32_t* row_idx;
   unsigned* err;
 };
 
-// Block-wide arg-max of (conf, -pos): returns the winning row (or -1).
-__device__ __forceinline__ long long block_best(float c, long long pos, float* s_c, long long* s_pos) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+// Warp arg-max of (conf, -pos): the winning (conf, pos) on every lane.
+__device__ __forceinline__ void warp_best(float& c, long long& pos) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float c2 = __shfl_xor_sync(0xffffffffu, c, o);
     const long long p2 = __shfl_xor_sync(0xffffffffu, pos, o);
-    if (c2 > c || (c2 == c && p2 < pos)) { c = c2; pos = p2; }
-  }
-  if (lane == 0) { s_c[warp] = c; s_pos[warp] = pos; }
-  __syncthreads();
-  if (warp == 0) {
-    c = lane < kSelThreads / 32 ? s_c[lane] : -2.f;
-    pos = lane < kSelThreads / 32 ? s_pos[lane] : LLONG_MAX;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float c2 = __shfl_xor_sync(0xffffffffu, c, o);
-      const long long p2 = __shfl_xor_sync(0xffffffffu, pos, o);
-      if (c2 > c || (c2 == c && p2 < pos)) { c = c2; pos = p2; }
+    if (c2 > c || (c2 == c && p2 < pos)) {
+      c = c2;
+      pos = p2;
     }
-    if (lane == 0) { s_c[0] = c; s_pos[0] = pos; }
   }
-  __syncthreads();
-  const long long best = (s_c[0] >= 0.f) ? s_pos[0] : -1;
-  __syncthreads();
-  return best;
 }
 
-// Merge the splits of request b's masked rows, count churn, take the top-k
-// and commit; run by one block of kSelThreads threads.
-__device__ __forceinline__ void select_request(const SelArgs& a, int b) {
+// Combination of chunks [c0, min(c0 + 32, nc)) of one row's triples in two
+// passes: the max M, then the sum of s * 2^((m - M)log2e) and the smallest
+// index among chunks at M.
+__device__ __forceinline__ Partial combine_group(const Partial* __restrict__ part, long long rows, long long i, int c0,
+                                                 int nc) {
+  float m[32], sv[32];
+  int ix[32];
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    const bool ok = c0 + c < nc;
+    const Partial v = part[static_cast<long long>(ok ? c0 + c : 0) * rows + i];
+    m[c] = ok ? v.m : -INFINITY;
+    sv[c] = ok ? v.s : 0.f;
+    ix[c] = ok ? v.idx : INT_MAX;
+  }
+  float mx = m[0];
+#pragma unroll
+  for (int c = 1; c < 32; ++c) mx = fmaxf(mx, m[c]);
+  Partial r;
+  r.m = mx;
+  r.s = 0.f;
+  r.idx = INT_MAX;
+  r.pad = 0;
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    if (sv[c] > 0.f) r.s += sv[c] * sfu_ex2((m[c] - mx) * kLog2e);
+    if (m[c] == mx) r.idx = min(r.idx, ix[c]);
+  }
+  return r;
+}
+
+// (argmax, conf) of one row from all its chunk triples.
+__device__ __forceinline__ void combine_row(const Partial* __restrict__ part, long long rows, long long i, int nc,
+                                            float& conf, int& idx) {
+  Partial p = combine_group(part, rows, i, 0, nc);
+  for (int c0 = 32; c0 < nc; c0 += 32) {
+    const Partial q = combine_group(part, rows, i, c0, nc);
+    const float mx = fmaxf(p.m, q.m);
+    const float sp = p.s > 0.f ? p.s * sfu_ex2((p.m - mx) * kLog2e) : 0.f;
+    const float sq = q.s > 0.f ? q.s * sfu_ex2((q.m - mx) * kLog2e) : 0.f;
+    p.idx = p.m == mx ? (q.m == mx ? min(p.idx, q.idx) : p.idx) : q.idx;
+    p.m = mx;
+    p.s = sp + sq;
+  }
+  conf = 1.f / p.s;
+  idx = p.idx == INT_MAX ? 0 : p.idx;
+}
+
+// One CTA per request.  Each thread combines one row's chunk triples per
+// pass (one round of coalesced loads); after one barrier, warp 0 forms the
+// statistics and takes the top-k with k rounds of a warp arg-max over the
+// rows' confidences in shared memory.
+__global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
+  __shared__ float s_conf_buf[kSelSmemRows];
+  __shared__ int32_t s_idx_buf[kSelSmemRows];
+  __shared__ float s_sum[kSelThreads / 32];
+  __shared__ int s_cnt[3][kSelThreads / 32];
+  pdl_launch_dependents();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int kWarps = kSelThreads / 32;
   const long long cu0 = a.cu[b], cu1 = a.cu[b + 1];
   const long long s0 = min(max(cu0, 0LL), a.total_rows);
   const long long s1 = min(max(cu1, s0), a.total_rows);
-  if (threadIdx.x == 0 && (cu0 != s0 || cu1 != s1)) raise_error(a.err, DEV_ERR_ARG);
+  if (tid == 0 && (cu0 != s0 || cu1 != s1)) raise_error(a.err, DEV_ERR_ARG);
+  const long long n = s1 - s0;
+  // per-row results: shared memory when the request fits, else workspace;
+  // conf = -3 marks a row that is not masked (or already committed)
+  float* cbuf = n <= kSelSmemRows ? s_conf_buf : a.row_conf + s0;
+  int32_t* ibuf = n <= kSelSmemRows ? s_idx_buf : a.row_idx + s0;
 
-  __shared__ float s_c[kSelThreads / 32];
-  __shared__ long long s_pos[kSelThreads / 32];
-  __shared__ float s_sum[kSelThreads / 32];
-  __shared__ int s_cnt[3][kSelThreads / 32];
-
+  // the mask, the previous argmax and the chunk triples of a row are loaded
+  // together (triples of unmasked rows are stale and discarded)
   float conf_sum = 0.f;
   int n_masked = 0, n_both = 0, n_changed = 0;
-  for (long long i = s0 + threadIdx.x; i < s1; i += kSelThreads) {
-    if (!a.masked[i]) continue;
-    // load the row's partials eight at a time, then merge them
-    Partial p = a.partial[i * a.nsplit];
-    for (int sp0 = 1; sp0 < a.nsplit; sp0 += 8) {
-      Partial q[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (sp0 + u < a.nsplit) q[u] = a.partial[i * a.nsplit + sp0 + u];
-#pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (sp0 + u < a.nsplit) p = merge(p, q[u]);
+  for (long long r = tid; r < n; r += kSelThreads) {
+    const long long i = s0 + r;
+    const uint8_t m8 = a.masked[i];
+    const int prev = a.argmax ? a.argmax[i] : -1;
+    float conf;
+    int idx;
+    combine_row(a.partial, a.total_rows, i, a.nchunk, conf, idx);
+    if (!m8) {
+      cbuf[r] = -3.f;
+      continue;
     }
-    const int idx = p.idx == INT_MAX ? 0 : p.idx;
-    const float conf = 1.f / p.s;
-    a.row_conf[i] = conf;
-    a.row_idx[i] = idx;
+    cbuf[r] = conf;
+    ibuf[r] = idx;
     if (a.conf_out) a.conf_out[i] = conf;
-    if (a.argmax) {
-      const int prev = a.argmax[i];
-      if (prev >= 0) {
-        ++n_both;
-        n_changed += prev != idx;
-      }
-      a.argmax[i] = idx;
-    }
+    if (a.argmax) a.argmax[i] = idx;
     conf_sum += conf;
     ++n_masked;
+    if (prev >= 0) {
+      ++n_both;
+      n_changed += prev != idx;
+    }
   }
-  // block sums (fixed order: per warp, then warps in order)
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // block sums in a fixed order: a shuffle tree per warp, then warps in order
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     conf_sum += __shfl_xor_sync(0xffffffffu, conf_sum, o);
@@ -262,46 +367,88 @@ __device__ __forceinline__ void select_request(const SelArgs& a, int b) {
     s_cnt[2][warp] = n_changed;
   }
   __syncthreads();
+  if (warp != 0) return;
+
   float tot_conf = 0.f;
   int tot_masked = 0, tot_both = 0, tot_changed = 0;
-  for (int w = 0; w < kSelThreads / 32; ++w) {
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
     tot_conf += s_sum[w];
     tot_masked += s_cnt[0][w];
     tot_both += s_cnt[1][w];
     tot_changed += s_cnt[2][w];
   }
-  if (threadIdx.x == 0 && a.stats) {
+  if (lane == 0 && a.stats) {
     a.stats[2 * b + 0] = tot_masked ? tot_conf / static_cast<float>(tot_masked) : 0.f;
     a.stats[2 * b + 1] = tot_both ? static_cast<float>(tot_changed) / static_cast<float>(tot_both) : 0.f;
   }
-
-  // top-k: k rounds of a block-wide arg-max over the rows still masked
+  // top-k: k rounds of a warp arg-max over the rows still masked
   const int take = min(a.k, tot_masked);
-  for (int j = 0; j < take; ++j) {
+  int j = 0;
+  for (; j < take; ++j) {
     float best_c = -2.f;
     long long best_pos = LLONG_MAX;
-    for (long long i = s0 + threadIdx.x; i < s1; i += kSelThreads) {
-      if (!a.masked[i]) continue;
-      const float c = a.row_conf[i];
-      if (c > best_c || (c == best_c && i < best_pos)) { best_c = c; best_pos = i; }
+    for (long long i = lane; i < n; i += 32) {
+      const float c = cbuf[i];
+      if (c > best_c || (c == best_c && i < best_pos)) {
+        best_c = c;
+        best_pos = i;
+      }
     }
-    const long long w = block_best(best_c, best_pos, s_c, s_pos);
-    if (threadIdx.x == 0 && w >= 0) {
-      a.tokens[w] = a.row_idx[w];
-      a.masked[w] = 0;
-      if (a.committed) a.committed[static_cast<long long>(b) * a.k + j] = static_cast<int32_t>(w - s0);
+    const long long mine = best_pos;
+    warp_best(best_c, best_pos);
+    if (best_pos == LLONG_MAX) break;  // only when confidences are not numbers
+    if (mine == best_pos) {
+      a.tokens[s0 + best_pos] = ibuf[best_pos];
+      a.masked[s0 + best_pos] = 0;
+      cbuf[best_pos] = -3.f;
+      if (a.committed) a.committed[static_cast<long long>(b) * a.k + j] = static_cast<int32_t>(best_pos);
     }
-    __syncthreads();
+    __syncwarp();
   }
   if (a.committed)
-    for (int j = take + threadIdx.x; j < a.k; j += kSelThreads) a.committed[static_cast<long long>(b) * a.k + j] = -1;
+    for (int q = j + lane; q < a.k; q += 32) a.committed[static_cast<long long>(b) * a.k + q] = -1;
 }
 
-
-__global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
-  pdl_launch_dependents();
-  pdl_wait();
-  select_request(a, blockIdx.x);
+// Both kernels of one call on `stream`, over the workspace `ws` (layout L).
+inline davet_status enqueue(const void* logits, int V, const int32_t* cu, int batch, int64_t total_rows, int k,
+                            uint8_t* masked, int32_t* tokens, int32_t* argmax, float* conf, int32_t* committed,
+                            float* stats, uint8_t* ws, const Layout& L, cudaStream_t stream) {
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
+  if (total_rows > 0) {
+    RowArgs r;
+    r.logits = static_cast<const uint4*>(logits);
+    r.V8 = V / 8;
+    r.nchunk = L.nchunk;
+    r.chunk = (r.V8 + L.nchunk - 1) / L.nchunk;
+    r.total_rows = total_rows;
+    r.masked = masked;
+    r.partial = partial;
+    const long long warps = total_rows * L.nchunk;
+    const long long blocks = (warps + kRowThreads / 32 - 1) / (kRowThreads / 32);
+    const cudaError_t e = launch(row_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kRowThreads), 0, stream, r);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
+  SelArgs a;
+  a.partial = partial;
+  a.nchunk = L.nchunk;
+  a.cu = cu;
+  a.batch = batch;
+  a.total_rows = total_rows;
+  a.k = k;
+  a.masked = masked;
+  a.tokens = tokens;
+  a.argmax = argmax;
+  a.conf_out = conf;
+  a.committed = committed;
+  a.stats = stats;
+  a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
+  a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
+  a.err = err;
+  const cudaError_t e = launch(select_kernel, dim3(batch), dim3(kSelThreads), 0, stream, a);
+  return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }
 
 }  // namespace unm
@@ -309,7 +456,7 @@ __global__ void __launch_bounds__(kSelThreads) select_commit(SelArgs a) {
 
 extern "C" davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, size_t* bytes) {
   if (total_rows < 0 || V < 8 || V % 8 != 0 || batch < 0 || !bytes) return DAVET_ERR_INVALID_ARG;
-  *bytes = davet::unm::layout_for(total_rows, V, batch).bytes;
+  *bytes = davet::unm::layout_for(total_rows, V).bytes;
   return DAVET_OK;
 }
 
@@ -326,38 +473,10 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
   if (reinterpret_cast<uintptr_t>(logits) & 15u) return DAVET_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(workspace) & 255u) return DAVET_ERR_INVALID_ARG;
   if (batch > 65535 || total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
-  const Layout L = layout_for(total_rows, V, batch);
-  if (workspace_bytes < L.bytes) return DAVET_ERR_INVALID_ARG;
-  unsigned* err = device_error_word();
-  if (!err) return DAVET_ERR_CUDA;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
-  Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
-  SelArgs a;
-  a.partial = partial;
-  a.nsplit = L.nsplit;
-  a.cu = cu_resp_dev;
-  a.batch = batch;
-  a.total_rows = total_rows;
-  a.k = k;
-  a.masked = masked_dev;
-  a.tokens = tokens_dev;
-  a.argmax = argmax_dev;
-  a.conf_out = conf_dev;
-  a.committed = committed_dev;
-  a.stats = stats_dev;
-  a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
-  a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
-  a.err = err;
-  if (total_rows > 0) {
-    const long long items = total_rows * L.nsplit;
-    const cudaError_t e = launch(row_pass, dim3(static_cast<unsigned>(items)), dim3(kRowThreads), 0, st,
-                                 static_cast<const uint4*>(logits), V / 8, static_cast<const uint8_t*>(masked_dev),
-                                 static_cast<long long>(total_rows), L.nsplit, partial);
-    if (e != cudaSuccess) return cuda_fail(e);
-  }
-  const cudaError_t e = launch(select_commit, dim3(batch), dim3(kSelThreads), 0, st, a);
-  return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
+  const Layout L = layout_for(total_rows, V);
+  if (total_rows > 0 && workspace_bytes < L.bytes) return DAVET_ERR_INVALID_ARG;
+  return enqueue(logits, V, cu_resp_dev, batch, total_rows, k, masked_dev, tokens_dev, argmax_dev, conf_dev,
+                 committed_dev, stats_dev, static_cast<uint8_t*>(workspace), L, static_cast<cudaStream_t>(stream));
 }
 
 // ---------------------------------------------------------------------------
@@ -366,7 +485,8 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
 // Its scratch lives in a fixed device array owned by the library, so the
 // caller passes only inputs and outputs.  Every device that loads the library
 // keeps this array for the life of the process, and all calls on a device
-// share it.
+// share it.  Nothing in it needs clearing: the select reads only the
+// triples of masked rows, which the row kernel of the same call writes.
 namespace davet {
 namespace unm {
 
@@ -419,41 +539,11 @@ extern "C" davet_status davet_unmask_topk_noalloc(const void* logits, int V, con
   if (total_rows > 0 && !logits) return DAVET_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(logits) & 15u) return DAVET_ERR_INVALID_ARG;
   if (batch > 65535 || total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
-  const Layout L = layout_for(total_rows, V);
+  const Layout L = layout_for(total_rows, V, kNoAllocScratchBytes);
   if (L.bytes > kNoAllocScratchBytes) return DAVET_ERR_UNSUPPORTED;  // too many answer rows for the array
   davet_status st = DAVET_OK;
   uint8_t* ws = noalloc_scratch(&st);
   if (!ws) return st;
-  unsigned* err = device_error_word();
-  if (!err) return DAVET_ERR_CUDA;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // Nothing in the scratch needs clearing: the select kernel reads only the
-  // partials, confidences and argmaxes of masked rows, and the row pass of
-  // this same call writes all of them first.
-  Partial* partial = reinterpret_cast<Partial*>(ws + L.off_partial);
-  if (total_rows > 0) {
-    const long long items = total_rows * L.nsplit;
-    row_pass<<<static_cast<unsigned>(items), kRowThreads, 0, s>>>(static_cast<const uint4*>(logits), V / 8,
-                                                                  masked_dev, total_rows, L.nsplit, partial);
-    const davet_status e = check_launch();
-    if (e != DAVET_OK) return e;
-  }
-  SelArgs a;
-  a.partial = partial;
-  a.nsplit = L.nsplit;
-  a.cu = cu_resp_dev;
-  a.batch = batch;
-  a.total_rows = total_rows;
-  a.k = k;
-  a.masked = masked_dev;
-  a.tokens = tokens_dev;
-  a.argmax = argmax_dev;
-  a.conf_out = conf_dev;
-  a.committed = committed_dev;
-  a.stats = stats_dev;
-  a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
-  a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
-  a.err = err;
-  select_commit<<<batch, kSelThreads, 0, s>>>(a);
-  return check_launch();
+  return enqueue(logits, V, cu_resp_dev, batch, total_rows, k, masked_dev, tokens_dev, argmax_dev, conf_dev,
+                 committed_dev, stats_dev, ws, L, static_cast<cudaStream_t>(stream));
 }

@@ -76,7 +76,7 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(davet, resp, V, k):
 
 def test_noalloc_rejects_sizes_beyond_its_scratch(davet):
     lib = davet_mod.load_cdll()
-    too_many_rows = 50000  # needs more than the 1 MiB array at V = 126464
+    too_many_rows = 200000  # needs more than the 1 MiB array (8 bytes per row)
     n = ctypes.c_size_t(0)
     assert lib.davet_unmask_topk_workspace(too_many_rows, workloads.VOCAB_8B, 1, ctypes.byref(n)) == 0
     assert n.value > (1 << 20)
