@@ -84,15 +84,19 @@ struct Params {
 // region r (0 producer, 1 MMA, 2 softmax A, 3 softmax B) holds 2048 events;
 // plain stores only, so recording stays off the critical path
 __device__ unsigned long long* g_attn_trace;
-__device__ __forceinline__ void trace_event(unsigned region, unsigned& n, unsigned code, unsigned idx) {
-  unsigned long long* t = g_attn_trace;
+// the buffer pointer is read once per role (ATTN_TRACE_DECL), so an event
+// costs a clock read and two stores, not a global load
+__device__ __forceinline__ void trace_event(unsigned long long* t, unsigned region, unsigned& n, unsigned code,
+                                            unsigned idx) {
   if (blockIdx.x != 0 || t == nullptr || n >= 2048) return;
   t[(region * 2048 + n) * 2] = clock64();
   t[(region * 2048 + n) * 2 + 1] = (static_cast<unsigned long long>(code) << 32) | idx;
   ++n;
 }
-#define ATTN_TRACE(region, code, idx) trace_event((region), trace_n, (code), (idx))
-#define ATTN_TRACE_DECL unsigned trace_n = 0
+#define ATTN_TRACE(region, code, idx) trace_event(trace_buf, (region), trace_n, (code), (idx))
+#define ATTN_TRACE_DECL   \
+  unsigned trace_n = 0; \
+  unsigned long long* trace_buf = g_attn_trace
 #else
 #define ATTN_TRACE(region, code, idx) \
   do {                                \
@@ -428,11 +432,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
         tc_fence_after();
         // all four TMEM loads in flight before one wait
+        // the row in two halves: the second half's TMEM load is in flight
+        // while the first half's max is taken
         uint32_t raw[BN];
-#pragma unroll
-        for (int q = 0; q < BN / 32; ++q)
-          tmem_ld32(s_addr + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&raw[32 * q]));
-        tmem_wait_ld();
+        tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&raw[0]));
+        tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&raw[32]));
+        tmem_wait_ld_regs(&raw[0]);
+        tmem_ld32(s_addr + 64, *reinterpret_cast<uint32_t(*)[32]>(&raw[64]));
+        tmem_ld32(s_addr + 96, *reinterpret_cast<uint32_t(*)[32]>(&raw[96]));
         if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
         float* x = reinterpret_cast<float*>(raw);
         const int valid = min(BN, w.len - w.key_tile(j) * BN);
@@ -453,19 +460,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           fence_proxy_async_smem();
         }
-        if (valid < BN) {
+        if (valid < BN / 2) {
 #pragma unroll
-          for (int i = 0; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+          for (int i = 0; i < BN / 2; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
         }
         // row max: eight independent chains of three-input max, then a tree
         float mp[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
 #pragma unroll
-        for (int i = 16; i < BN; i += 16)
+        for (int i = 16; i < BN / 2; i += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+        tmem_wait_ld_regs(&raw[64]);
+        if (valid < BN) {
+#pragma unroll
+          for (int i = BN / 2; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+        }
+#pragma unroll
+        for (int i = BN / 2; i < BN; i += 16)
 #pragma unroll
           for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
         const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
+        if (r == 0) ATTN_TRACE(2 + t, 26 + t, ns);
         const float mt = mx * c;
         float factor = 1.f;
         bool need = false;
@@ -496,6 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st16(s_addr + 16 * q, pk);
         }
         const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
+        if (r == 0) ATTN_TRACE(2 + t, 28 + t, ns);
         // O is settled here (S of this tile was issued after the previous
         // PV of this tile) and no MMA touches it before P is published
         if (j > 0 && __any_sync(0xffffffffu, need)) {
