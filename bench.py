@@ -358,11 +358,16 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
 
 
 def run_e2e(args, pl, w, dev, stream, world):
-    """Same pass through the C ABI with pinned host inputs: features, text
-    and every step's logits copied in, committed tokens copied out.  Step
-    logits are copied on a second stream into a ring of three device buffers,
-    so the copy for step t+1 overlaps the kernels of step t (ordered with
-    events); the timed region spans both streams."""
+    """Same pass through the C ABI with pinned host inputs: features and text
+    copied in, every step's logits read from pinned host memory, committed
+    tokens copied out.
+
+    Mode "mapped" (default): the unmasking kernel reads each step's logits
+    straight from pinned host memory (device-addressable), so only the rows
+    still masked cross the host link.  Mode "copy": every step's full logits
+    are copied on a second stream into a ring of three device buffers, the
+    copy for step t+1 overlapping the kernels of step t (ordered with events);
+    the timed region spans both streams."""
     import torch
 
     from paper_2608_01821_gb300 import workloads
@@ -371,9 +376,12 @@ def run_e2e(args, pl, w, dev, stream, world):
     P = 4
     host_logits = [workloads.logits(w, t).pin_memory() for t in range(P)]
     NB = 3
-    dev_logits = [torch.empty((w.total_resp, w.V), dtype=torch.bfloat16, device=dev) for _ in range(NB)]
+    mapped = getattr(args, "e2e_mode", "mapped") == "mapped"
+    dev_logits = [] if mapped else [torch.empty((w.total_resp, w.V), dtype=torch.bfloat16, device=dev)
+                                    for _ in range(NB)]
     tokens_host = torch.empty(w.total_resp, dtype=torch.int32).pin_memory()
-    h2d = sum(f.numel() * 2 for f in feats) + text.numel() * 2 + w.T * w.total_resp * w.V * 2
+    logit_rows = sum(w.masked_rows(t) for t in range(w.T)) if mapped else w.T * w.total_resp
+    h2d = sum(f.numel() * 2 for f in feats) + text.numel() * 2 + logit_rows * w.V * 2
     d2h = w.total_resp * 4
     copy_stream = torch.cuda.Stream(device=dev)
     ready = [torch.cuda.Event() for _ in range(NB)]
@@ -388,7 +396,15 @@ def run_e2e(args, pl, w, dev, stream, world):
             dev_logits[slot].copy_(host_logits[t % P], non_blocking=True)
             ready[slot].record(copy_stream)
 
-    def one():
+    def one_mapped():
+        pl.reset_state()
+        pl.load_inputs(feats, text, non_blocking=True)
+        pl.build_pyramids()
+        for t in range(w.T):
+            pl.step(t, host_logits[t % P])
+        tokens_host.copy_(pl.tokens, non_blocking=True)
+
+    def one_copy():
         pass_start.record(stream)
         copy_stream.wait_event(pass_start)  # no copy starts before the pass (or under the previous one)
         for t in range(min(NB, w.T)):
@@ -405,6 +421,7 @@ def run_e2e(args, pl, w, dev, stream, world):
                 issue_copy(t + NB)
         tokens_host.copy_(pl.tokens, non_blocking=True)
 
+    one = one_mapped if mapped else one_copy
     with torch.cuda.stream(stream):
         one()
     torch.cuda.synchronize()
@@ -419,7 +436,7 @@ def run_e2e(args, pl, w, dev, stream, world):
     torch.cuda.synchronize()
     t = allreduce_max(s.elapsed_time(e) / 1e3, world, dev)
     return {"value": round(w.T * n * world / t, 3), "unit": "denoising steps/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "passes": n,
+            "d2h_bytes_per_step": int(d2h), "passes": n, "mode": "mapped" if mapped else "copy",
             "h2d_GBps": round(h2d * n / t / 1e9, 1)}
 
 
@@ -640,6 +657,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--logit-pool", type=int, default=0, help="cap on distinct device logit buffers")
+    ap.add_argument("--e2e-mode", choices=["mapped", "copy"], default="mapped",
+                    help="e2e logits: read from pinned host memory by the kernel, or copied to the device")
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)

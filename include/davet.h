@@ -19,7 +19,8 @@
  *
  * Conventions shared by every entry point:
  *  - Pointers named *_dev, and every tensor argument, are DEVICE pointers on
- *    the device current to the calling thread.  The caller owns every buffer;
+ *    the device current to the calling thread (davet_unmask_topk's logits may
+ *    also be device-addressable pinned host memory).  The caller owns every buffer;
  *    the library never allocates, frees or retains caller memory.
  *  - bf16 tensors are IEEE bfloat16 bit patterns (uint16), row-major, with
  *    the layout given per function.  Tensor base pointers must be 16-byte
@@ -219,7 +220,11 @@ davet_status davet_unmask_topk_workspace(int64_t total_rows, int V, int batch, s
  * trajectory risk (Eq. 7): the mean conf over M_t and the churn, the
  * fraction of rows of M_t that had a previous prediction whose argmax
  * changed.
- *   logits        bf16 [total_rows][V]; only masked rows are read
+ *   logits        bf16 [total_rows][V]; only masked rows are read.  May be
+ *                 device memory or pinned host memory that the device can
+ *                 address (cudaHostAlloc / a pinned allocation on a system
+ *                 with unified addressing): the kernels then read the masked
+ *                 rows over the host link and nothing else crosses it.
  *   V             vocabulary size, a multiple of 8
  *   cu_resp_dev   int32 [batch+1]: request b owns rows cu[b]..cu[b+1]-1;
  *                 cu[batch] <= total_rows

@@ -140,3 +140,24 @@ def test_full_size_first_step(davet, name):
     w = workloads.make(name)
     s = State(w.resp, w.V, w.k)
     s.step(davet, workloads.logits(w, 0))
+
+
+def test_host_mapped_logits_match_device_logits(davet):
+    """Logits in pinned host memory (read by the kernels over the host link,
+    masked rows only) give bit-identical results to the same logits in device
+    memory, over three steps of an 8B-class vocabulary."""
+    resp, V, k = [40, 7, 81], workloads.VOCAB_8B, 3
+    a, b = State(resp, V, k), State(resp, V, k)
+    for t in range(3):
+        lg = workloads.normal_bf16((a.R, V), 900 + t, 2 ** 0.5)
+        host = lg.pin_memory()
+        for st, src in ((a, lg.cuda()), (b, host)):
+            d = st.d
+            ws = torch.zeros(max(davet.davet_unmask_topk_workspace(st.R, V, st.B), 256), dtype=torch.uint8,
+                             device="cuda")
+            davet.davet_unmask_topk(src, V, d["cu"], st.B, st.R, k, d["masked"], d["tokens"], d["argmax"],
+                                    d["conf"], d["committed"], d["stats"], ws)
+        torch.cuda.synchronize()
+        assert davet.davet_device_status() == (0, 0)
+        for key in ("masked", "tokens", "argmax", "conf", "committed", "stats"):
+            assert torch.equal(a.d[key], b.d[key]), (t, key)
