@@ -46,11 +46,12 @@ def attention_source_hash() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, fused: bool = True):
     """DRAM bytes per attention launch from the committed ncu summary of this
     workload's pass, or None when the summary is missing or was taken on
     different kernel sources."""
-    path = os.path.join(ROOT, "profiles", f"attention_{workload}_pass_traffic.txt")
+    kind = "view_attention" if fused else "attention"
+    path = os.path.join(ROOT, "profiles", f"{kind}_{workload}_pass_traffic.txt")
     try:
         kv = {}
         for line in open(path):
@@ -147,7 +148,7 @@ def run_ours(args, rank, world, local_rank):
     w = workloads.make(args.config)
     if rank > 0:
         w.seed = w.seed + 1000 * rank  # each replica gets its own batch
-    pl = Pipeline(w, dev, lib)
+    pl = Pipeline(w, dev, lib, fused=not getattr(args, "unfused", False))
     feats = [workloads.features(w, b) for b in range(w.batch)]
     text = workloads.text_rows(w)
     pl.load_inputs(feats, text)
@@ -221,9 +222,13 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0:
         peaks = measured_peaks()
         value = whole_job_rate(w.T * args.steps, world, total_s)
-        launches_per_pass = w.batch + w.T * 4  # pyramid per request; gather, attention, 2 unmask kernels per step
-        attn_flops_launch = comp["attention"]["flops"] / comp["attention"]["launches"]
-        attn_ms = comp["attention"]["ms"] / comp["attention"]["launches"]
+        # per request the view-block build (pyramid + fill kernels) or the
+        # pyramid; per step the fused view attention (or gather and attention)
+        # and the two unmask kernels
+        launches_per_pass = (2 * w.batch + w.T * 3) if pl.fused else (w.batch + w.T * 4)
+        akey = "view_attention" if pl.fused else "attention"
+        attn_flops_launch = comp[akey]["flops"] / comp[akey]["launches"]
+        attn_ms = comp[akey]["ms"] / comp[akey]["launches"]
         achieved = attn_flops_launch / (attn_ms * 1e-3) / 1e12
         out = {
             "metric": METRIC,
@@ -260,14 +265,14 @@ def run_ours(args, rank, world, local_rank):
                 for k, v in comp.items()
             },
             "roofline": {
-                "kernel": "step_attention",
+                "kernel": "view_attention (fused gather and step attention)" if pl.fused else "step_attention",
                 "bound": "tensor",
                 "achieved": round(achieved, 2),
                 "peak": peaks["bf16_tflops"],
                 "unit": "TFLOP/s",
                 "frac": round(achieved / peaks["bf16_tflops"], 4),
                 "peak_source": f"{peaks['source']} bf16 burst (MEASURED_PEAKS.json)",
-                "traffic": profiled_traffic(w.name),
+                "traffic": profiled_traffic(w.name, pl.fused),
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
                 "flops_per_launch": attn_flops_launch,
             },
@@ -310,11 +315,14 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
         pl.reset_state()
         timed("pyramid", pl.build_pyramids)
         for t in range(w.T):
-            timed("gather", lambda t=t: pl.gather(t))
-            timed("attention", pl.attention)
+            if pl.fused:
+                timed("view_attention", lambda t=t: pl.view_attention(t))
+            else:
+                timed("gather", lambda t=t: pl.gather(t))
+                timed("attention", pl.attention)
             timed("unmask", lambda t=t: pl.unmask(t, pool[t % P]))
 
-    totals = {"pyramid": 0.0, "gather": 0.0, "attention": 0.0, "unmask": 0.0}
+    totals = {"pyramid": 0.0, "gather": 0.0, "attention": 0.0, "unmask": 0.0, "view_attention": 0.0}
     mode = "graph"
     if probe is not None:
         try:
@@ -344,17 +352,22 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
     gbytes = sum(w.gather_bytes(t) for t in range(w.T))
     ubytes = sum(w.unmask_bytes(t) for t in range(w.T))
     pbytes = w.pyramid_bytes()
-    return {
+    out = {
         "timing_mode": mode,
         "pyramid": {"launches": w.batch, "ms": ms["pyramid"], "bytes": pbytes,
                     "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9},
-        "gather": {"launches": w.T, "ms": ms["gather"], "bytes": gbytes,
-                   "GBps": gbytes / (ms["gather"] * 1e-3) / 1e9},
-        "attention": {"launches": w.T, "ms": ms["attention"], "flops": flops,
-                      "TFLOPs": flops / (ms["attention"] * 1e-3) / 1e12},
-        "unmask": {"launches": 2 * w.T, "ms": ms["unmask"], "bytes": ubytes,
-                   "GBps": ubytes / (ms["unmask"] * 1e-3) / 1e9},
     }
+    if pl.fused:
+        out["view_attention"] = {"launches": w.T, "ms": ms["view_attention"], "flops": flops,
+                                 "TFLOPs": flops / (ms["view_attention"] * 1e-3) / 1e12}
+    else:
+        out["gather"] = {"launches": w.T, "ms": ms["gather"], "bytes": gbytes,
+                         "GBps": gbytes / (ms["gather"] * 1e-3) / 1e9}
+        out["attention"] = {"launches": w.T, "ms": ms["attention"], "flops": flops,
+                            "TFLOPs": flops / (ms["attention"] * 1e-3) / 1e12}
+    out["unmask"] = {"launches": 2 * w.T, "ms": ms["unmask"], "bytes": ubytes,
+                     "GBps": ubytes / (ms["unmask"] * 1e-3) / 1e9}
+    return out
 
 
 def run_e2e(args, pl, w, dev, stream, world):
@@ -598,6 +611,7 @@ def run_profile(args):
     pl.build_pyramids()
     pl.gather(t)
     fn = {"pyramid": pl.build_pyramids, "gather": lambda: pl.gather(t), "attention": pl.attention,
+          "view_attention": lambda: pl.view_attention(t),
           "unmask": lambda: (pl.reset_state(), pl.unmask(t, lg))}[args.profile]
     for _ in range(args.warmup + args.steps):
         fn()
@@ -659,7 +673,9 @@ def main(argv=None):
     ap.add_argument("--logit-pool", type=int, default=0, help="cap on distinct device logit buffers")
     ap.add_argument("--e2e-mode", choices=["mapped", "copy"], default="mapped",
                     help="e2e logits: read from pinned host memory by the kernel, or copied to the device")
-    ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "unmask"], default=None,
+    ap.add_argument("--unfused", action="store_true",
+                    help="pack each step with davet_gather_view, then davet_step_attention (instead of the fused call)")
+    ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)
     args = ap.parse_args(argv)

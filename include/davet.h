@@ -11,6 +11,9 @@
  *   davet_gather_view     the step input [view || prompt || answer] (Eq. 5),
  *                         the view a pooled level or the mixed view
  *   davet_step_attention  bidirectional attention over it (Sec. 3.1, Eq. 1)
+ *   davet_build_views     every view once as a contiguous [view || text] block
+ *   davet_view_attention  the gather and the attention fused: attention reads
+ *                         each request's step sequence from its view block
  *   davet_unmask_topk     argmax, confidence and confidence-ranked commit
  *                         (Sec. 3.1, Eq. 1-2) plus the mean confidence and
  *                         churn that drive the trajectory risk (Eq. 7)
@@ -27,8 +30,8 @@
  *    aligned.
  *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
  *    call only enqueues work on that stream and returns without waiting.
- *    davet_build_pyramid, davet_gather_view, davet_step_attention and
- *    davet_unmask_topk never synchronize the host, so they can be captured in
+ *    davet_build_pyramid, davet_gather_view, davet_step_attention,
+ *    davet_view_attention and davet_unmask_topk never synchronize the host, so they can be captured in
  *    a CUDA graph once each has run at least once on the device outside of a
  *    capture (the first call per device resolves a few device addresses).
  *  - Host-visible argument checks run before anything is enqueued and return
@@ -201,6 +204,73 @@ davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* t
  */
 davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev, int batch,
                                   int64_t max_total_rows, int H, int D, float scale, void* out, void* stream);
+
+/*
+ * View blocks (host-only helpers and the build).  In the view-block layout a
+ * request keeps every evidence view once as a contiguous block
+ *     [ view rows (n_tiles * rows_per_tile[v]) || its text_rows prompt and
+ *       answer rows ]
+ * for views v = 0..n_views-1: the pooled levels 0..n_levels-1 (Sec. 4.3,
+ * rows as in davet_pyramid_layout) and, when mixed_stride != 0, the mixed
+ * view as view n_levels (davet_mixed_view_rows).  A step's input for view v
+ * (Eq. 5) is then one run of rows, which davet_view_attention reads directly.
+ *
+ * davet_view_rows: rows_per_tile (int [n_views], nullable) and n_views (int*,
+ * nullable) for this geometry.
+ * davet_view_layout: block_row0 (int64 [n_views + 1], nullable): first row of
+ * each block within the request's buffer; [n_views] is the buffer's rows.
+ */
+davet_status davet_view_rows(int grid, int n_levels, int mixed_level, int mixed_stride, int* rows_per_tile,
+                             int* n_views);
+davet_status davet_view_layout(int grid, int n_levels, int mixed_level, int mixed_stride, int n_tiles, int text_rows,
+                               int64_t* block_row0);
+
+/*
+ * Builds one request's view blocks (Sec. 4.3: all views constructed once
+ * before denoising): the pooled levels as davet_build_pyramid defines them
+ * (level l at the start of block l), the mixed view's rows, and a copy of the
+ * request's text rows in every block.
+ *   feat   bf16 [n_tiles][grid][grid][C]; if feat == buf the encoding is
+ *          already in place at the start of block 0, otherwise it is copied
+ *          there (feat must not overlap buf then)
+ *   buf    bf16 [block_row0[n_views]][C], the request's buffer
+ *   text   bf16 [text_rows][C], the prompt and answer rows; must not overlap
+ *          buf (nullable when text_rows == 0)
+ * Enqueues two kernels on `stream`.
+ */
+davet_status davet_build_views(const void* feat, void* buf, const void* text, int n_tiles, int grid, int n_levels,
+                               int mixed_level, int mixed_stride, int text_rows, int C, void* stream);
+
+/*
+ * davet_gather_view followed by davet_step_attention in one kernel (Eq. 5,
+ * then Sec. 3.1, Eq. 1), without the packed step input: request b's sequence
+ * [view || prompt || answer] for its step view is the view block that
+ * davet_build_views laid out, and the attention kernel reads its query, key
+ * and value rows straight from it.  out and cu_seqlens_dev are what
+ * davet_gather_view + davet_step_attention produce for the same views.
+ *   store            bf16 [store_rows][3][H][D]: every request's view-block
+ *                    buffer (C = 3*H*D)
+ *   buf_row0_dev     int64 [batch]: first store row of request b's buffer
+ *   tiles_dev, prompt_len_dev, resp_len_dev  int32 [batch]; request b's
+ *                    blocks carry prompt_len + resp_len text rows
+ *   view_dev         int32 [batch]: the step's view of each request (a level,
+ *                    or n_levels for the mixed view)
+ *   grid, n_levels, mixed_level, mixed_stride   the view geometry
+ *   H, D, scale, out           as for davet_step_attention
+ *   cu_seqlens_dev   int32 [batch+1] output, as davet_gather_view writes it
+ *   max_total_rows   capacity of out in packed rows
+ *   batch            0..256
+ * Device-side checks: a view outside [0, n_views) or a negative count sets
+ * DAVET_DEV_ARG and the request contributes no rows; a sequence running past
+ * store_rows sets DAVET_DEV_ARG (those rows read as zeros); a total above
+ * max_total_rows sets DAVET_DEV_CAPACITY and cu_seqlens is clamped.
+ */
+davet_status davet_view_attention(const void* store, int64_t store_rows, const int64_t* buf_row0_dev,
+                                  const int32_t* tiles_dev, const int32_t* prompt_len_dev,
+                                  const int32_t* resp_len_dev, const int32_t* view_dev, int batch, int grid,
+                                  int n_levels, int mixed_level, int mixed_stride, int H, int D, float scale,
+                                  void* out, int32_t* cu_seqlens_dev, int64_t max_total_rows, void* stream);
+
 
 /* ------------------------------------------------------------ unmasking */
 

@@ -23,8 +23,17 @@
 // memory, so key tiles may straddle request boundaries and the buffer end.
 // With few items (short sequences) the host selects one query tile per item
 // so that more SMs get work.
+//
+// Fused variant (davet_view_attention, FUSED = true): the step input is never
+// packed.  Each request keeps every evidence view as a contiguous block
+// [view rows || prompt rows || answer rows] (davet_build_views), so a
+// request's sequence for its step view is one run of store rows: every CTA
+// derives the requests' view lengths and block starts on the device, and the
+// producer loads query, key and value tiles from those runs exactly as the
+// packed variant loads them from the packed input.
 #include <algorithm>
 #include <cstdio>
+#include <cstring>
 #include <mutex>
 
 #include "common.cuh"
@@ -38,6 +47,8 @@ constexpr int NS = 2;            // K/V pipeline stages
 constexpr int kThreads = 320;    // 2 softmax warpgroups + TMA warp + MMA warp
 constexpr int kWarpTma = 8, kWarpMma = 9;
 constexpr int kMaxBatch = 1024;  // requests per call
+constexpr int kFusedMaxBatch = 256;  // requests per call of the fused variant
+constexpr int kMaxLevels = 5;
 constexpr int kLptMaxBatch = 256;
 constexpr int kChunkBytes = 128 * 128;  // 128 rows x 128 B (64 bf16) swizzled chunk
 constexpr uint32_t kTmemCols = 512;
@@ -46,9 +57,10 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units
 __host__ __device__ constexpr uint32_t col_s(int t) { return t * 128u; }
 __host__ __device__ constexpr uint32_t col_o(int t) { return 256u + t * 128u; }
 
-template <int D>
+template <int D, bool FUSED>
 struct Smem {
   static constexpr int KC = D / 64;
+  static constexpr int kFB = FUSED ? kFusedMaxBatch : 1;
   alignas(1024) uint8_t q[2][KC][kChunkBytes];
   alignas(1024) uint8_t k[NS][KC][kChunkBytes];
   alignas(1024) uint8_t v[NS][KC][kChunkBytes];
@@ -64,9 +76,24 @@ struct Smem {
   int32_t req_len[kMaxBatch];
   int32_t order[kMaxBatch];   // request index of the i-th scheduled request
   int32_t cum[kMaxBatch + 1]; // items before the i-th scheduled request
+  // fused variant: first store row of request b's sequence for its view
+  int64_t f_base[kFB];
+};
+
+struct FusedView {
+  long long n_rows;         // rows of the store
+  const int64_t* buf_row0;  // first store row of each request's view blocks
+  const int32_t* tiles;
+  const int32_t* prompt;
+  const int32_t* resp;
+  const int32_t* level;     // view index per request
+  int n_views;
+  int rows_per_tile[kMaxLevels + 1];  // view rows per tile of each view
+  int32_t* cu_out;
 };
 
 struct Params {
+  FusedView fv;
   const int32_t* cu;
   int batch;
   int H;
@@ -107,6 +134,7 @@ __device__ __forceinline__ void trace_event(unsigned long long* t, unsigned regi
 #endif
 
 struct Item {
+  int b;                              // request
   int start, len, q0, h, nkv, ntile;  // q0: first query row of the item within the request
   int kv0;  // key tile the item starts from (key tiles are visited cyclically)
 
@@ -121,8 +149,8 @@ struct Item {
 // 1 = key, 2 = value) of head h.
 __device__ __forceinline__ int h_coord(int slot, int h, int H) { return slot * H + h; }
 
-template <int D>
-__device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H, int qtiles) {
+template <typename S>
+__device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) {
   // largest i with cum[i] <= item
   int lo = 0, hi = s.n_req - 1;
   while (lo < hi) {
@@ -135,6 +163,7 @@ __device__ __forceinline__ Item decode(const Smem<D>& s, int item, int H, int qt
   const int rows_per_item = BM * qtiles;
   const int nq = (len + rows_per_item - 1) / rows_per_item;
   Item it;
+  it.b = b;
   it.start = s.req_start[b];
   it.len = len;
   it.h = local / nq;
@@ -154,12 +183,14 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
   return __all_sync(0xffffffffu, ok);
 }
 
-template <int D>
+template <int D, bool FUSED>
 __global__ void __launch_bounds__(kThreads, 1)
     attention_kernel(const __grid_constant__ CUtensorMap tmap, Params prm) {
   constexpr int KC = D / 64;
   extern __shared__ uint8_t smem_raw[];
-  Smem<D>& s = *reinterpret_cast<Smem<D>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  using SM = Smem<D, FUSED>;
+  SM& s = *reinterpret_cast<SM*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const FusedView& fv = prm.fv;
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -194,7 +225,42 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();  // cu_seqlens and qkv come from the previous kernel
 
   // ---------------------------------------------------------- schedule
-  if (tid == 0) {
+  if (FUSED && tid == 0) {
+    // view lengths and packed starts, as davet_gather_view computes them, and
+    // where each request's sequence starts in the store: its view block
+    bool bad = false;
+    long long run = 0;
+    int n = 0;
+    for (int b = 0; b < prm.batch; ++b) {
+      const int v = fv.level[b], nt = fv.tiles[b], pl = fv.prompt[b], rl = fv.resp[b];
+      long long nvis = 0, base = fv.buf_row0[b];
+      const long long text = static_cast<long long>(max(pl, 0)) + max(rl, 0);
+      if (v < 0 || v >= fv.n_views || nt < 0 || pl < 0 || rl < 0) {
+        bad = true;
+        base = -1;
+      } else {
+        for (int u = 0; u < v; ++u) base += static_cast<long long>(nt) * fv.rows_per_tile[u] + text;
+        nvis = static_cast<long long>(nt) * fv.rows_per_tile[v];
+      }
+      const long long len = base >= 0 ? nvis + text : 0;
+      if (base >= 0 && base + len > fv.n_rows) bad = true;  // rows past the store read as zeros
+      const long long a = min(run, static_cast<long long>(prm.max_rows));
+      const long long e = min(run + len, static_cast<long long>(prm.max_rows));
+      run += len;
+      s.req_start[b] = static_cast<int32_t>(a);
+      s.req_len[b] = static_cast<int32_t>(e - a);
+      s.f_base[b] = base;
+      if (e > a) s.order[n++] = b;
+      if (blockIdx.x == 0) fv.cu_out[b] = static_cast<int32_t>(a);
+    }
+    if (blockIdx.x == 0) {
+      fv.cu_out[prm.batch] = static_cast<int32_t>(min(run, static_cast<long long>(prm.max_rows)));
+      if (bad) raise_error(prm.err, DEV_ERR_ARG);
+      if (run > prm.max_rows) raise_error(prm.err, DEV_ERR_CAPACITY);
+    }
+    s.n_req = n;
+  }
+  if (!FUSED && tid == 0) {
     bool bad = false;
     int prev_end = 0;
     int n = 0;
@@ -265,21 +331,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kWarpTma) {
     // ------------------------------------------------------ TMA producer
+    // rows of the item's request: packed input (cu) or its view block
     if (lane == 0) {
       ATTN_TRACE_DECL;
       uint32_t it = 0, wi = 0;
       bool ok = true;
       for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
         const Item w = decode(s, item, H, qtiles);
+        const long long src0 = FUSED ? s.f_base[w.b] : w.start;
         if (wi > 0) ok = mbar_wait(&s.q_empty, (wi - 1) & 1, prm.err, abort_flag);
         if (!ok) break;
         mbar_arrive_expect_tx(&s.q_full, w.ntile * KC * kChunkBytes);
         for (int t = 0; t < w.ntile; ++t)
           for (int c = 0; c < KC; ++c)
-            tma_load_3d(s.q[t][c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), w.start + w.q0 + t * BM);
+            tma_load_3d(s.q[t][c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), src0 + w.q0 + t * BM);
         for (int j = 0; j < w.nkv; ++j, ++it) {
           const int st = it % NS;
-          const int row = w.start + w.key_tile(j) * BN;
+          const int row = static_cast<int>(src0 + w.key_tile(j) * BN);
           // K of stage st is free once the S MMAs of the tile that used it completed
           if (it >= NS) ok = mbar_wait(&s.k_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
           if (!ok) break;
@@ -377,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (more) {
             ok = mbar_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
             if (!ok) break;
-            ATTN_TRACE(1, 11, it);
+              ATTN_TRACE(1, 11, it);
             tc_fence_after();
             issue_s(0, st1);
             if (w.ntile == 1) {
@@ -598,19 +666,22 @@ EncodeTiledFn get_encode_fn() {
 
 struct DeviceInfo {
   int sms = 0;
-  bool attr_set[2] = {false, false};
+  bool attr_set[4] = {false, false, false, false};
 };
 DeviceInfo g_dev[64];
 std::mutex g_dev_mu;
 
-template <int D>
-davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_rows, int H, float scale, void* out,
-                    cudaStream_t stream) {
+// Launches the packed variant (FUSED = false: qkv is the packed input, cu its
+// boundaries) or the fused one (FUSED = true: qkv is the row store of view
+// blocks, fv describes the requests; cu is unused).
+template <int D, bool FUSED>
+davet_status launch(const void* qkv, const int32_t* cu, const attn::FusedView& fv, int batch, int64_t max_rows, int H,
+                    float scale, void* out, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e);
   if (dev < 0 || dev >= 64) return DAVET_ERR_UNSUPPORTED;
-  const size_t smem = sizeof(attn::Smem<D>) + 1024;
+  const size_t smem = sizeof(attn::Smem<D, FUSED>) + 1024;
   {
     std::lock_guard<std::mutex> g(g_dev_mu);
     DeviceInfo& di = g_dev[dev];
@@ -618,9 +689,9 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
       e = cudaDeviceGetAttribute(&di.sms, cudaDevAttrMultiProcessorCount, dev);
       if (e != cudaSuccess) return cuda_fail(e);
     }
-    const int slot = D == 128 ? 1 : 0;
+    const int slot = (D == 128 ? 1 : 0) + (FUSED ? 2 : 0);
     if (!di.attr_set[slot]) {
-      e = cudaFuncSetAttribute(attn::attention_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      e = cudaFuncSetAttribute(attn::attention_kernel<D, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(smem));
       if (e != cudaSuccess) return cuda_fail(e);
       di.attr_set[slot] = true;
@@ -630,10 +701,11 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   if (!err) return DAVET_ERR_CUDA;
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return DAVET_ERR_CUDA;
-
+  // packed variant: the packed input; fused: the row store of view blocks
   CUtensorMap tmap;
+  const int64_t map_rows = FUSED ? fv.n_rows : max_rows;
   const cuuint64_t gdim[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(3 * H),
-                              static_cast<cuuint64_t>(max_rows)};
+                              static_cast<cuuint64_t>(std::max<int64_t>(map_rows, 1))};
   const cuuint64_t gstride[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(3) * H * D * 2};
   const cuuint32_t box[3] = {64, 1, 128};
   const cuuint32_t estride[3] = {1, 1, 1};
@@ -643,6 +715,7 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   if (cr != CUDA_SUCCESS) return DAVET_ERR_INVALID_ARG;
 
   attn::Params prm;
+  prm.fv = fv;
   prm.cu = cu;
   prm.batch = batch;
   prm.H = H;
@@ -657,7 +730,7 @@ davet_status launch(const void* qkv, const int32_t* cu, int batch, int64_t max_r
   const int64_t items_bound = ((max_rows + attn::BM - 1) / attn::BM + batch) * static_cast<int64_t>(H);
   const int grid = static_cast<int>(std::min<int64_t>(items_bound, g_dev[dev].sms));
   if (grid <= 0) return DAVET_OK;
-  e = davet::launch(attn::attention_kernel<D>, dim3(grid), dim3(attn::kThreads), smem, stream, tmap, prm);
+  e = davet::launch(attn::attention_kernel<D, FUSED>, dim3(grid), dim3(attn::kThreads), smem, stream, tmap, prm);
   return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }
 
@@ -683,6 +756,44 @@ extern "C" davet_status davet_step_attention(const void* qkv, const int32_t* cu_
   if (batch > attn::kMaxBatch) return DAVET_ERR_UNSUPPORTED;
   if (max_total_rows > (int64_t(1) << 30) || static_cast<int64_t>(3) * H > 65535) return DAVET_ERR_UNSUPPORTED;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  return D == 128 ? launch<128>(qkv, cu_seqlens_dev, batch, max_total_rows, H, scale, out, st)
-                  : launch<64>(qkv, cu_seqlens_dev, batch, max_total_rows, H, scale, out, st);
+  const attn::FusedView none{};
+  return D == 128 ? launch<128, false>(qkv, cu_seqlens_dev, none, batch, max_total_rows, H, scale, out, st)
+                  : launch<64, false>(qkv, cu_seqlens_dev, none, batch, max_total_rows, H, scale, out, st);
+}
+
+extern "C" davet_status davet_view_attention(const void* store, int64_t store_rows, const int64_t* buf_row0_dev,
+                                             const int32_t* tiles_dev, const int32_t* prompt_len_dev,
+                                             const int32_t* resp_len_dev, const int32_t* view_dev, int batch,
+                                             int grid, int n_levels, int mixed_level, int mixed_stride, int H, int D,
+                                             float scale, void* out, int32_t* cu_seqlens_dev, int64_t max_total_rows,
+                                             void* stream) {
+  using namespace davet;
+  if (batch < 0 || max_total_rows < 0 || H < 1 || !(scale > 0.f) || store_rows < 0) return DAVET_ERR_INVALID_ARG;
+  int rpt[attn::kMaxLevels + 1];
+  int n_views = 0;
+  const davet_status ls = davet_view_rows(grid, n_levels, mixed_level, mixed_stride, rpt, &n_views);
+  if (ls != DAVET_OK) return ls;
+  if (D != 64 && D != 128) return DAVET_ERR_UNSUPPORTED;
+  if (batch > attn::kFusedMaxBatch) return DAVET_ERR_UNSUPPORTED;
+  if (max_total_rows > (int64_t(1) << 30) || static_cast<int64_t>(3) * H > 65535) return DAVET_ERR_UNSUPPORTED;
+  if (store_rows > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
+  if (!cu_seqlens_dev) return DAVET_ERR_INVALID_ARG;
+  if (batch == 0) return DAVET_OK;
+  if (!store || !buf_row0_dev || !tiles_dev || !prompt_len_dev || !resp_len_dev || !view_dev || !out)
+    return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(store) | reinterpret_cast<uintptr_t>(out)) & 15u) return DAVET_ERR_INVALID_ARG;
+  attn::FusedView fv{};
+  fv.n_rows = store_rows;
+  fv.buf_row0 = buf_row0_dev;
+  fv.tiles = tiles_dev;
+  fv.prompt = prompt_len_dev;
+  fv.resp = resp_len_dev;
+  fv.level = view_dev;
+  fv.n_views = n_views;
+  for (int v = 0; v <= attn::kMaxLevels; ++v) fv.rows_per_tile[v] = v < n_views ? rpt[v] : 0;
+  fv.cu_out = cu_seqlens_dev;
+  if (max_total_rows == 0) return DAVET_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return D == 128 ? launch<128, true>(store, nullptr, fv, batch, max_total_rows, H, scale, out, st)
+                  : launch<64, true>(store, nullptr, fv, batch, max_total_rows, H, scale, out, st);
 }

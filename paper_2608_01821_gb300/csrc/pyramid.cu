@@ -319,33 +319,27 @@ extern "C" davet_status davet_pyramid_layout(int grid, int n_levels, int n_tiles
   return DAVET_OK;
 }
 
-extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C,
-                                            float* pyr_f32, void* stream) {
-  using namespace davet;
-  using namespace davet::pyr;
-  if (n_tiles < 0 || grid < 1 || n_levels < 1 || C < 8) return DAVET_ERR_INVALID_ARG;
-  if (n_levels > kMaxLevels || grid > 65536) return DAVET_ERR_UNSUPPORTED;
-  if (C % 8 != 0) return DAVET_ERR_INVALID_ARG;
-  if (n_tiles == 0) return DAVET_OK;
-  if (!feat || !pyr) return DAVET_ERR_INVALID_ARG;
-  if ((reinterpret_cast<uintptr_t>(feat) | reinterpret_cast<uintptr_t>(pyr) |
-       reinterpret_cast<uintptr_t>(pyr_f32)) & 15u)
-    return DAVET_ERR_INVALID_ARG;
+namespace davet {
+namespace pyr {
 
+// Enqueues the pyramid build with level l's rows starting at row off[l] of
+// pyr (level 0 at off[0]; rows of a level are tile-major, row-major within a
+// tile) and `extent` rows in all; arguments already checked by the caller.
+davet_status enqueue(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C, float* pyr_f32,
+                     const int64_t* off, int64_t extent, cudaStream_t st) {
   Geom g;
-  int64_t off[kMaxLevels + 1];
   int side[kMaxLevels];
-  davet_pyramid_layout(grid, n_levels, n_tiles, side, off);
+  davet_pyramid_layout(grid, n_levels, n_tiles, side, nullptr);
   for (int l = 0; l < kMaxLevels; ++l) g.side[l] = l < n_levels ? side[l] : 1;
-  for (int l = 0; l <= kMaxLevels; ++l) g.off[l] = l <= n_levels ? off[l] : off[n_levels];
+  for (int l = 0; l <= kMaxLevels; ++l) g.off[l] = l < n_levels ? off[l] : extent;
   g.n_tiles = n_tiles;
   g.C8 = C / 8;
   g.copy0 = feat != pyr;
   if (g.copy0) {
     // feat and the pyramid must not overlap when level 0 is copied
     const uintptr_t f0 = reinterpret_cast<uintptr_t>(feat), p0 = reinterpret_cast<uintptr_t>(pyr);
-    const uintptr_t f1 = f0 + static_cast<uintptr_t>(off[1]) * C * 2;
-    const uintptr_t p1 = p0 + static_cast<uintptr_t>(off[n_levels]) * C * 2;
+    const uintptr_t f1 = f0 + static_cast<uintptr_t>(n_tiles) * grid * grid * C * 2;
+    const uintptr_t p1 = p0 + static_cast<uintptr_t>(extent) * C * 2;
     if (f0 < p1 && p0 < f1) return DAVET_ERR_INVALID_ARG;
   }
 
@@ -361,7 +355,6 @@ extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_t
     threads = 256;
     blocks = std::min<long long>((total + threads - 1) / threads, 152LL * 64);
   }
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   const uint4* f = static_cast<const uint4*>(feat);
   uint4* p = static_cast<uint4*>(pyr);
   float4* p32 = reinterpret_cast<float4*>(pyr_f32);
@@ -375,4 +368,24 @@ extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_t
   }
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
+}
+
+}  // namespace pyr
+}  // namespace davet
+
+extern "C" davet_status davet_build_pyramid(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C,
+                                            float* pyr_f32, void* stream) {
+  using namespace davet;
+  using namespace davet::pyr;
+  if (n_tiles < 0 || grid < 1 || n_levels < 1 || C < 8) return DAVET_ERR_INVALID_ARG;
+  if (n_levels > kMaxLevels || grid > 65536) return DAVET_ERR_UNSUPPORTED;
+  if (C % 8 != 0) return DAVET_ERR_INVALID_ARG;
+  if (n_tiles == 0) return DAVET_OK;
+  if (!feat || !pyr) return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(feat) | reinterpret_cast<uintptr_t>(pyr) |
+       reinterpret_cast<uintptr_t>(pyr_f32)) & 15u)
+    return DAVET_ERR_INVALID_ARG;
+  int64_t off[kMaxLevels + 1];
+  davet_pyramid_layout(grid, n_levels, n_tiles, nullptr, off);
+  return enqueue(feat, pyr, n_tiles, grid, n_levels, C, pyr_f32, off, off[n_levels], static_cast<cudaStream_t>(stream));
 }

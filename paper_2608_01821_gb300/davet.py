@@ -69,6 +69,11 @@ def _declare(lib):
         "davet_gather_view": (_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _vp,
                                      _vp, _i64, _vp]),
         "davet_step_attention": (_int, [_vp, _vp, _int, _i64, _int, _int, _f32, _vp, _vp]),
+        "davet_view_rows": (_int, [_int, _int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_int)]),
+        "davet_view_layout": (_int, [_int, _int, _int, _int, _int, _int, ctypes.POINTER(_i64)]),
+        "davet_build_views": (_int, [_vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _int, _vp]),
+        "davet_view_attention": (_int, [_vp, _i64, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _int, _int,
+                                        _int, _f32, _vp, _vp, _i64, _vp]),
         "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_unmask_topk": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
                                      _vp]),
@@ -141,6 +146,31 @@ class Davet:
         self._check("davet_step_attention",
                     self.lib.davet_step_attention(_ptr(qkv), _ptr(cu_seqlens), batch, max_total_rows, H, D,
                                                   float(scale), _ptr(out), _stream(stream)))
+
+    def davet_view_layout(self, grid: int, n_levels: int, mixed_level: int, mixed_stride: int, n_tiles: int,
+                          text_rows: int) -> list[int]:
+        nv = _int(0)
+        self._check("davet_view_rows", self.lib.davet_view_rows(grid, n_levels, mixed_level, mixed_stride, None,
+                                                                 ctypes.byref(nv)))
+        off = (_i64 * (nv.value + 1))()
+        self._check("davet_view_layout", self.lib.davet_view_layout(grid, n_levels, mixed_level, mixed_stride,
+                                                                     n_tiles, text_rows, off))
+        return list(off)
+
+    def davet_build_views(self, feat, buf, text, n_tiles: int, grid: int, n_levels: int, mixed_level: int,
+                          mixed_stride: int, text_rows: int, C: int, stream=None):
+        self._check("davet_build_views",
+                    self.lib.davet_build_views(_ptr(feat), _ptr(buf), _ptr(text), n_tiles, grid, n_levels,
+                                               mixed_level, mixed_stride, text_rows, C, _stream(stream)))
+
+    def davet_view_attention(self, store, store_rows: int, buf_row0, tiles, prompt_len, resp_len, view, batch: int,
+                             grid: int, n_levels: int, mixed_level: int, mixed_stride: int, H: int, D: int,
+                             scale: float, out, cu_seqlens, max_total_rows: int, stream=None):
+        self._check("davet_view_attention",
+                    self.lib.davet_view_attention(_ptr(store), store_rows, _ptr(buf_row0), _ptr(tiles),
+                                                  _ptr(prompt_len), _ptr(resp_len), _ptr(view), batch, grid,
+                                                  n_levels, mixed_level, mixed_stride, H, D, float(scale), _ptr(out),
+                                                  _ptr(cu_seqlens), max_total_rows, _stream(stream)))
 
     def davet_unmask_topk_workspace(self, total_rows: int, V: int, batch: int) -> int:
         n = _sz(0)

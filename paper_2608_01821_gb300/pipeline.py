@@ -1,13 +1,20 @@
 """Device-resident state of one DAVET batch and the per-step call sequence.
 
 Host orchestration only: this module allocates the buffers a batch needs
-(pyramids, packed step input, attention output, answer state, workspace) as
-torch CUDA tensors and issues the four library calls in order.  It performs no
-arithmetic of its own.
+(pyramids or view blocks, step input, attention output, answer state,
+workspace) as torch CUDA tensors and issues the library calls in order.  It
+performs no arithmetic of its own.
 
-Per request the pyramid buffer is level-major; its level-0 rows are where the
-visual encoding is written, so the pyramid build reads the encoding in place
-and writes only the pooled levels.
+Two layouts:
+  fused (default)  each request's buffer holds view blocks [view || text]
+                   (davet_build_views), and a step is davet_view_attention,
+                   which reads each request's sequence from the block of its
+                   step view, then the unmasking;
+  unfused          each request's buffer is its level-major pyramid, text
+                   rows live apart, and a step is davet_gather_view (packing
+                   the step input), davet_step_attention, then the unmasking.
+In both, the encoding is written where level 0 lives (the first rows of the
+request's buffer), so the build reads it in place.
 """
 from __future__ import annotations
 
@@ -18,25 +25,38 @@ from .workloads import Workload
 
 
 class Pipeline:
-    def __init__(self, w: Workload, device="cuda", lib=None):
+    def __init__(self, w: Workload, device="cuda", lib=None, fused: bool = True):
         self.w = w
         self.dev = torch.device(device)
         self.lib = lib if lib is not None else _davet.load()
         C, B = w.C, w.batch
         self.sides = w.level_sides()
-        # pyramids: one allocation, request b at row pyr_row0[b]
-        rows = [w.pyramid_rows(b) for b in range(B)]
-        self.pyr_row0 = [0]
+        self.fused = fused
+        mixed = w.mixed_args
+        text_rows = [p + r for p, r in zip(w.prompt, w.resp)]
+        # one allocation; request b's buffer starts at row buf_row0[b]
+        if fused:
+            self.blocks = [self.lib.davet_view_layout(w.grid, w.n_levels, *mixed, w.tiles[b], text_rows[b])
+                           for b in range(B)]
+            rows = [blk[-1] for blk in self.blocks]
+        else:
+            rows = [w.pyramid_rows(b) for b in range(B)]
+        self.buf_row0 = [0]
         for r in rows:
-            self.pyr_row0.append(self.pyr_row0[-1] + r)
-        self.pyr = torch.empty((self.pyr_row0[-1], C), dtype=torch.bfloat16, device=self.dev)
-        self.pyr_views = [self.pyr[self.pyr_row0[b]:self.pyr_row0[b + 1]] for b in range(B)]
-        self.pyr_ptrs = torch.tensor([v.data_ptr() for v in self.pyr_views], dtype=torch.int64, device=self.dev)
+            self.buf_row0.append(self.buf_row0[-1] + r)
+        n_buf = self.buf_row0[-1]
+        self.store = torch.empty((max(n_buf, 1), C), dtype=torch.bfloat16, device=self.dev)
+        self.bufs = [self.store[self.buf_row0[b]:self.buf_row0[b + 1]] for b in range(B)]
+        self.buf_row0_dev = torch.tensor(self.buf_row0[:-1], dtype=torch.int64, device=self.dev)
+        # text rows (unfused: gathered from here; fused: copied into every block)
         self.text = torch.empty((max(w.total_text(), 1), C), dtype=torch.bfloat16, device=self.dev)
+        self.pyr_views = self.bufs  # unfused: the level-major pyramids
+        self.pyr_ptrs = torch.tensor([v.data_ptr() for v in self.bufs], dtype=torch.int64, device=self.dev)
         self.tiles = torch.tensor(w.tiles, dtype=torch.int32, device=self.dev)
         self.prompt = torch.tensor(w.prompt, dtype=torch.int32, device=self.dev)
         self.resp = torch.tensor(w.resp, dtype=torch.int32, device=self.dev)
         self.text_off = torch.from_numpy(w.text_offsets()).to(self.dev)
+        self.text_off_host = w.text_offsets()
         self.schedule = torch.from_numpy(w.schedule).to(self.dev).contiguous()
         self.max_rows = w.max_total_rows()
         self.packed = torch.empty((self.max_rows, C), dtype=torch.bfloat16, device=self.dev)
@@ -55,9 +75,22 @@ class Pipeline:
 
     # -------------------------------------------------------------- inputs
     def level0(self, b: int):
-        """Rows of request b's encoding inside its pyramid buffer."""
+        """Rows of request b's encoding inside its buffer (level 0 comes first
+        in both layouts)."""
         n = self.w.tiles[b] * self.w.grid * self.w.grid
-        return self.pyr_views[b][:n]
+        return self.bufs[b][:n]
+
+    def pyramid_cpu(self, b: int):
+        """Request b's pooled levels as a level-major bf16 CPU tensor (for
+        checks), from either layout."""
+        w = self.w
+        if not self.fused:
+            return self.bufs[b].cpu()
+        parts = []
+        for lvl, g in enumerate(self.sides):
+            r0 = self.blocks[b][lvl]
+            parts.append(self.bufs[b][r0:r0 + w.tiles[b] * g * g])
+        return torch.cat(parts).cpu()
 
     def load_inputs(self, feats, text, non_blocking=False):
         """feats: per-request bf16 [tiles, G, G, C]; text: bf16 [sum(P+R), C]."""
@@ -73,16 +106,29 @@ class Pipeline:
 
     # ---------------------------------------------------------------- path
     def build_pyramids(self, stream=None):
+        """The pyramids (unfused) or every view block (fused), once per batch."""
         w = self.w
         for b in range(w.batch):
-            v = self.pyr_views[b]
-            self.lib.davet_build_pyramid(v, v, w.tiles[b], w.grid, w.n_levels, w.C, None, stream)
+            v = self.bufs[b]
+            if self.fused:
+                t0 = int(self.text_off_host[b])
+                n = w.prompt[b] + w.resp[b]
+                self.lib.davet_build_views(v, v, self.text[t0:t0 + n] if n else None, w.tiles[b], w.grid, w.n_levels,
+                                           *w.mixed_args, n, w.C, stream)
+            else:
+                self.lib.davet_build_pyramid(v, v, w.tiles[b], w.grid, w.n_levels, w.C, None, stream)
 
     def gather(self, t: int, stream=None):
         w = self.w
         self.lib.davet_gather_view(self.pyr_ptrs, self.tiles, self.text, self.text_off, self.prompt, self.resp,
                                    self.schedule[t], w.batch, w.grid, w.n_levels, *w.mixed_args, w.C,
                                    self.packed, self.cu, self.max_rows, stream)
+
+    def view_attention(self, t: int, stream=None):
+        w = self.w
+        self.lib.davet_view_attention(self.store, self.store.shape[0], self.buf_row0_dev, self.tiles, self.prompt,
+                                      self.resp, self.schedule[t], w.batch, w.grid, w.n_levels, *w.mixed_args, w.H,
+                                      w.D, w.scale, self.attn_out, self.cu, self.max_rows, stream)
 
     def attention(self, stream=None):
         w = self.w
@@ -96,6 +142,9 @@ class Pipeline:
                                    self.workspace, self.workspace.numel(), stream)
 
     def step(self, t: int, logits, stream=None):
-        self.gather(t, stream)
-        self.attention(stream)
+        if self.fused:
+            self.view_attention(t, stream)
+        else:
+            self.gather(t, stream)
+            self.attention(stream)
         self.unmask(t, logits, stream)

@@ -83,6 +83,20 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_step_attention(null, p, 1, 128, 4, 64, f(0.1), p, null) == INV
     assert lib.davet_step_attention(p, p, 2000, 128, 4, 64, f(0.1), p, null) == UNS
     assert lib.davet_step_attention(p, p, 0, 128, 4, 64, f(0.1), p, null) == 0  # empty batch
+    # fused view attention: batch above its limit, bad head dim, null store
+    assert lib.davet_view_attention(p, 10, p, p, p, p, p, 300, 27, 4, 0, 0, 4, 64, f(0.1), p, p, 100, null) == UNS
+    assert lib.davet_view_attention(p, 10, p, p, p, p, p, 1, 27, 4, 0, 0, 4, 96, f(0.1), p, p, 100, null) == UNS
+    assert lib.davet_view_attention(null, 10, p, p, p, p, p, 1, 27, 4, 0, 0, 4, 64, f(0.1), p, p, 100, null) == INV
+    assert lib.davet_view_attention(p, 10, p, p, p, p, p, 1, 27, 4, 5, 3, 4, 64, f(0.1), p, p, 100, null) == INV
+    # view blocks: layout helpers against the pyramid layout plus text rows
+    off = (ctypes.c_int64 * 6)()
+    assert lib.davet_view_layout(27, 4, 2, 3, 2, 50, off) == 0
+    assert list(off)[:6] == [0, 2 * 729 + 50, 2 * 729 + 2 * 196 + 100, 2 * (729 + 196 + 49) + 150,
+                             2 * (729 + 196 + 49 + 16) + 200, 2 * (729 + 196 + 49 + 16 + 130) + 250]
+    nv = ctypes.c_int(0)
+    assert lib.davet_view_rows(27, 4, 0, 0, None, ctypes.byref(nv)) == 0 and nv.value == 4
+    assert lib.davet_view_layout(27, 4, 5, 3, 2, 50, off) == INV
+    assert lib.davet_build_views(p, p, null, 1, 27, 4, 0, 0, 5, 16, null) == INV  # text rows without text
     # gather: bad levels count, batch too large
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 0, 0, 16, p, p, 100, null) == INV
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 0, 0, 16, p, p, 100, null) == UNS
