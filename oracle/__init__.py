@@ -23,6 +23,14 @@ Parity status of each function (what pins it is listed in the tests under
   unmask    pinned (closed-form confidences, tie rules, brute-force top-k)
   policy    pinned (Eq. 7-9 special cases, envelope mean and ordering
             invariants, Table D "High" step counts)
+  prune     pinned (stable library sort, nesting, identity at full
+            retention, NaN and tie rules); the score is an input (the paper
+            does not define it)
+  merge     pinned (constant tiles, single-cell top level = tile mean,
+            partition and nesting invariants, row = member mean in fp64,
+            per-round greedy choices against an independent fp64 cosine,
+            hand-worked 4x4 example); the matching rule is a reading
+            (bipartite matching rounds), the paper prints none
 """
 from __future__ import annotations
 
@@ -51,7 +59,7 @@ def build(force: bool = False) -> str:
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".tmp{os.getpid()}"
         subprocess.check_call(
-            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-Wall",
+            ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared", "-fopenmp", "-Wall",
              _SRC, "-o", tmp, "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
@@ -65,6 +73,7 @@ def _load():
             lib = ctypes.CDLL(_LIB)
             lib.oracle_level_sides.restype = ctypes.c_int64
             lib.oracle_mixed_view.restype = ctypes.c_int64
+            lib.oracle_merge_round.restype = ctypes.c_int
             lib.oracle_policy_risk.restype = ctypes.c_double
             lib.oracle_policy_budget.restype = ctypes.c_double
             lib.oracle_policy_view.restype = ctypes.c_int
@@ -151,6 +160,77 @@ def mixed_view(pyr_bf16, n_tiles: int, grid: int, n_levels: int, coarse_level: i
                                   _ptr(out, _c_u16p))
     assert n == rows
     return out
+
+
+
+def view_rows_per_tile(grid: int, n_levels: int, mixed=None) -> list[int]:
+    """Rows per tile of every view: the pooled levels, then the mixed view."""
+    rows = [g * g for g in level_sides(grid, n_levels)]
+    if mixed is not None:
+        rows.append(mixed_rows_per_tile(grid, n_levels, *mixed))
+    return rows
+
+
+# ---------------------------------------------------------------- realizers
+def prune_keep(score, n_tiles: int, grid: int, rows_per_tile) -> list[np.ndarray]:
+    """Nested pruning (Sec. 4.3, Sec. 5.3): per view, int32 [n_tiles, m_v] of
+    the kept token indices of every tile (raster order)."""
+    s = np.ascontiguousarray(np.asarray(score, dtype=np.float32).reshape(-1))
+    assert s.size == n_tiles * grid * grid
+    m = np.ascontiguousarray(rows_per_tile, dtype=np.int32)
+    keep = np.empty(int(n_tiles * m.sum()), dtype=np.int32)
+    _load().oracle_prune_keep(_ptr(s, ctypes.POINTER(ctypes.c_float)), n_tiles, grid, len(m), _ptr(m, _c_i32p),
+                              _ptr(keep, _c_i32p))
+    out, o = [], 0
+    for mv in m:
+        out.append(keep[o: o + n_tiles * mv].reshape(n_tiles, mv))
+        o += n_tiles * mv
+    return out
+
+
+def prune_views(feat_bf16, score, n_tiles: int, grid: int, rows_per_tile, C: int) -> list[np.ndarray]:
+    """Rows of every pruned view: uint16 [n_tiles * m_v, C] per view."""
+    f = _as_u16(feat_bf16).reshape(n_tiles, grid * grid, C)
+    return [np.concatenate([f[t, k[t]] for t in range(n_tiles)]) if n_tiles else np.empty((0, C), np.uint16)
+            for k in prune_keep(score, n_tiles, grid, rows_per_tile)]
+
+
+def merge_views(feat_bf16, n_tiles: int, grid: int, n_levels: int, C: int, c0: int, Cs: int):
+    """Hierarchical similarity merging (Sec. 4.3, Sec. 5.3).
+
+    Returns (levels, assign): levels[l] is uint16 [n_tiles * G_l^2, C] (level
+    0 is the encoding itself) and assign is int32 [n_levels, n_tiles, grid^2],
+    the level-l token each level-0 token belongs to."""
+    f = _as_u16(feat_bf16).reshape(-1)
+    assert f.size == n_tiles * grid * grid * C
+    sides = level_sides(grid, n_levels)
+    rows = sum(n_tiles * g * g for g in sides[1:])
+    out = np.empty((max(rows, 1), C), dtype=np.uint16)
+    assign = np.empty((n_levels, n_tiles, grid * grid), dtype=np.int32)
+    _load().oracle_merge_views(_ptr(f, _c_u16p), n_tiles, grid, n_levels, C, c0, Cs, _ptr(out, _c_u16p),
+                               _ptr(assign, _c_i32p))
+    levels, o = [f.reshape(-1, C).copy()], 0
+    for g in sides[1:]:
+        levels.append(out[o: o + n_tiles * g * g])
+        o += n_tiles * g * g
+    return levels, assign
+
+
+def merge_round(feat_bf16, C: int, c0: int, Cs: int, tok, n: int, r: int):
+    """One bipartite matching round of one tile (Sec. 4.3 merging reading).
+
+    feat: the tile's level-0 rows [n0, C]; tok: int32 [n0], the current token
+    of every level-0 row.  Returns (new tok, new n, best sim [ceil(n/2)],
+    matched B index [ceil(n/2)])."""
+    f = _as_u16(feat_bf16).reshape(-1)
+    n0 = f.size // C
+    t = np.ascontiguousarray(tok, dtype=np.int32).copy()
+    nA = (n + 1) // 2
+    best = np.empty(max(nA, 1), dtype=np.float32)
+    best_b = np.empty(max(nA, 1), dtype=np.int32)
+    m = _load().oracle_merge_round(_ptr(f, _c_u16p), n0, C, c0, Cs, _ptr(t, _c_i32p), n, r,
+                                   _ptr(best, ctypes.POINTER(ctypes.c_float)), _ptr(best_b, _c_i32p))
+    return t, int(m), best[:nA], best_b[:nA]
 
 
 def gather(pyrs, tiles, text_bf16, text_off, prompt_len, resp_len, level,

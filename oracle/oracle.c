@@ -28,6 +28,17 @@
  *   oracle_policy_*      Sec. 4.2 / Eq. 6-8 and Sec. 4.3 / Eq. 9: phase
  *                        profile, normalizer, evidence envelope, trajectory
  *                        risk, envelope interpolation, thirds quantization.
+ *   oracle_prune_keep    Sec. 4.3 / Sec. 5.3: nested visual-token pruning,
+ *                        the kept tokens of every view for a given score.
+ *   oracle_merge_views   Sec. 4.3 / Sec. 5.3: hierarchical similarity merging
+ *                        (bipartite matching rounds level by level).  Its
+ *                        merge decisions are taken in binary32 with a fixed
+ *                        operation order (fused multiply-add chains in
+ *                        ascending channel order, correctly rounded square
+ *                        root and division), the precision the CUDA kernels
+ *                        decide in, so both sides take the same decisions;
+ *                        the file is compiled without contraction of
+ *                        separate multiplies and adds.
  *
  * Parallelism: OpenMP over independent outer loops only (tiles, requests x
  * heads, rows); each inner computation is the sequential definition.
@@ -512,4 +523,256 @@ int64_t oracle_mixed_view(const uint16_t *pyr, int n_tiles, int grid, int n_leve
                 memcpy(out + row * C, pyr + ((int64_t)t * grid * grid + (int64_t)y * grid + x) * C, (size_t)C * 2);
     }
     return row;
+}
+
+/* ------------------------------------------------------ pruning realizer */
+
+/*
+ * Order key of an importance score: larger scores first, a NaN below every
+ * number, equal scores by ascending token index (the sort is then total).
+ */
+typedef struct {
+    float s;
+    int32_t i;
+} scored_t;
+
+static int scored_cmp(const void *a, const void *b)
+{
+    const scored_t *x = (const scored_t *)a, *y = (const scored_t *)b;
+    const int xn = isnan(x->s), yn = isnan(y->s);
+    if (xn != yn) return xn ? 1 : -1;
+    if (!xn && x->s != y->s) return x->s > y->s ? -1 : 1;
+    return x->i < y->i ? -1 : (x->i > y->i);
+}
+
+/*
+ * Nested visual-token pruning (Sec. 4.3 "compatible evidence realizers":
+ * pruning varies the retention ratio; Sec. 5.3 / Table 2).  The importance
+ * score is not specified by the paper and is an input here: score[t][i] for
+ * token i (raster order) of tile t.  Reading: view v keeps, per tile, the
+ * rows_per_tile[v] highest-scoring tokens (ties by smaller index, NaN last)
+ * in raster order, so each view is a subset of every larger one.
+ * keep: the kept token indices, view-major then tile-major,
+ *       keep[sum_{u<v} n_tiles*m_u + t*m_v + j]  (m_v = rows_per_tile[v]).
+ */
+void oracle_prune_keep(const float *score, int n_tiles, int grid, int n_views, const int32_t *rows_per_tile,
+                       int32_t *keep)
+{
+    const int n = grid * grid;
+    int64_t base[33];
+    base[0] = 0;
+    for (int v = 0; v < n_views; ++v) base[v + 1] = base[v] + (int64_t)n_tiles * rows_per_tile[v];
+#pragma omp parallel for schedule(dynamic)
+    for (int t = 0; t < n_tiles; ++t) {
+        scored_t *s = malloc(sizeof(scored_t) * (size_t)n);
+        int32_t *rank = malloc(sizeof(int32_t) * (size_t)n);
+        for (int i = 0; i < n; ++i) {
+            s[i].s = score[(int64_t)t * n + i];
+            s[i].i = i;
+        }
+        qsort(s, (size_t)n, sizeof *s, scored_cmp);
+        for (int p = 0; p < n; ++p) rank[s[p].i] = p;
+        for (int v = 0; v < n_views; ++v) {
+            int32_t *k = keep + base[v] + (int64_t)t * rows_per_tile[v];
+            int j = 0;
+            for (int i = 0; i < n; ++i)
+                if (rank[i] < rows_per_tile[v]) k[j++] = i;
+        }
+        free(rank);
+        free(s);
+    }
+}
+
+/* ------------------------------------------------------ merging realizer */
+
+static float bf16_to_f32(uint16_t h)
+{
+    uint32_t u = ((uint32_t)h) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+/* binary32 -> bfloat16, round to nearest, ties to even (finite inputs). */
+static uint16_t f32_to_bf16_rne(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7f800000u) == 0x7f800000u) return (uint16_t)((u >> 16) | ((u & 0xffffu) ? 0x40u : 0u));
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+/*
+ * Feature sums of the current tokens: S[j][c] = sum over the level-0 tokens
+ * i with tok[i] == j, in ascending i, of x_i[c0 + c] (binary32, one rounded
+ * addition per member, starting from the first member's value).
+ */
+static void member_sums(const uint16_t *x0, int n0, const int32_t *tok, int n, int C, int c0, int Cs, float *S,
+                        int32_t *size)
+{
+    for (int j = 0; j < n; ++j) size[j] = 0;
+    for (int i = 0; i < n0; ++i) {
+        const int j = tok[i];
+        float *s = S + (int64_t)j * Cs;
+        const uint16_t *x = x0 + (int64_t)i * C + c0;
+        if (size[j] == 0)
+            for (int c = 0; c < Cs; ++c) s[c] = bf16_to_f32(x[c]);
+        else
+            for (int c = 0; c < Cs; ++c) s[c] = s[c] + bf16_to_f32(x[c]);
+        ++size[j];
+    }
+}
+
+/* Inverse norm 1/sqrt(sum_c s_c^2) with the squares accumulated by fused
+ * multiply-adds in ascending c; a zero vector gets 0. */
+static float inv_norm(const float *s, int Cs)
+{
+    float n2 = 0.0f;
+    for (int c = 0; c < Cs; ++c) n2 = fmaf(s[c], s[c], n2);
+    return n2 > 0.0f ? 1.0f / sqrtf(n2) : 0.0f;
+}
+
+/*
+ * One bipartite matching round over the n current tokens of one tile
+ * (token merging by bipartite soft matching, Bolya et al. 2023, as the
+ * aggregation step).  Positions 0, 2, 4, ... form set A and 1, 3, 5, ... set
+ * B.  Each a in A is matched to the b in B of highest cosine similarity
+ *   sim(a, b) = (dot(S_a, S_b) * inv_a) * inv_b,
+ * dot accumulated by fused multiply-adds in ascending channel order (ties
+ * go to the smaller b).  The r members of A with the highest matched
+ * similarity (ties to the smaller position) are merged into their match; the
+ * survivors keep their relative order.  Updates tok and returns n - r.
+ */
+static int merge_round(const uint16_t *x0, int n0, int32_t *tok, int n, int r, int C, int c0, int Cs, float *S,
+                       int32_t *size, float *inv, float *best, int32_t *best_b, int32_t *newpos)
+{
+    member_sums(x0, n0, tok, n, C, c0, Cs, S, size);
+    for (int j = 0; j < n; ++j) inv[j] = inv_norm(S + (int64_t)j * Cs, Cs);
+    const int nA = (n + 1) / 2, nB = n / 2;
+    for (int a = 0; a < nA; ++a) {
+        const float *sa = S + (int64_t)(2 * a) * Cs;
+        best[a] = 0.0f;
+        best_b[a] = -1;
+        for (int b = 0; b < nB; ++b) {
+            const float *sb = S + (int64_t)(2 * b + 1) * Cs;
+            float dot = 0.0f;
+            for (int c = 0; c < Cs; ++c) dot = fmaf(sa[c], sb[c], dot);
+            const float sim = (dot * inv[2 * a]) * inv[2 * b + 1];
+            if (best_b[a] < 0 || sim > best[a]) {
+                best[a] = sim;
+                best_b[a] = b;
+            }
+        }
+    }
+    /* merged[a] <=> fewer than r members of A rank before a */
+    int32_t *merged = newpos + n; /* scratch of nA entries after newpos */
+    for (int a = 0; a < nA; ++a) {
+        int before = 0;
+        for (int o = 0; o < nA; ++o)
+            if (best[o] > best[a] || (best[o] == best[a] && o < a)) ++before;
+        merged[a] = before < r;
+    }
+    int kept = 0;
+    for (int p = 0; p < n; ++p) {
+        const int gone = (p % 2 == 0) && merged[p / 2];
+        newpos[p] = gone ? -1 : kept++;
+    }
+    for (int i = 0; i < n0; ++i) {
+        int p = tok[i];
+        if (p % 2 == 0 && merged[p / 2]) p = 2 * best_b[p / 2] + 1;
+        tok[i] = newpos[p];
+    }
+    return kept;
+}
+
+/* One matching round of one tile on its own (for the tests): tok is
+ * updated in place; best / best_b (nullable, ceil(n/2) entries) receive each
+ * member of A's matched similarity and B index.  Returns the new count. */
+int oracle_merge_round(const uint16_t *x0, int n0, int C, int c0, int Cs, int32_t *tok, int n, int r, float *best,
+                       int32_t *best_b)
+{
+    float *S = malloc(sizeof(float) * (size_t)n * (size_t)Cs);
+    int32_t *size = malloc(sizeof(int32_t) * (size_t)n);
+    float *inv = malloc(sizeof(float) * (size_t)n);
+    float *bs = malloc(sizeof(float) * (size_t)n);
+    int32_t *bb = malloc(sizeof(int32_t) * (size_t)n);
+    int32_t *newpos = malloc(sizeof(int32_t) * (size_t)(2 * n));
+    const int out = merge_round(x0, n0, tok, n, r, C, c0, Cs, S, size, inv, bs, bb, newpos);
+    for (int a = 0; a < (n + 1) / 2; ++a) {
+        if (best) best[a] = bs[a];
+        if (best_b) best_b[a] = bb[a];
+    }
+    free(newpos);
+    free(bb);
+    free(bs);
+    free(inv);
+    free(size);
+    free(S);
+    return out;
+}
+
+/*
+ * Hierarchical similarity merging (Sec. 4.3 "compatible evidence realizers":
+ * merging varies the aggregation strength; Sec. 5.3 / Table 2).  Reading:
+ * per tile, level 0 is the encoding; level l is built from level l-1 by
+ * bipartite matching rounds (merge_round) with r = min(n - G_l^2, ceil(n/2))
+ * until it holds G_l^2 tokens, the row count of the pooled level l, so the
+ * views have the pooled hierarchy's lengths.  Similarity is measured on
+ * channels [c0, c0 + Cs) of the token sums.  A merged token's row is the
+ * mean of the level-0 rows it absorbed: the binary32 sum of its members in
+ * ascending index, divided by their count (binary32 division), rounded to
+ * bf16 (nearest even).
+ * feat : bf16 bits [n_tiles][grid*grid][C]
+ * out  : bf16 bits, level-major then tile-major, levels 1..n_levels-1:
+ *        row(l, t, j) = sum_{1<=u<l} n_tiles*G_u^2 + t*G_l^2 + j
+ * assign (nullable): int32 [n_levels][n_tiles][grid*grid], the level-l token
+ *        index that level-0 token i belongs to (level 0: i itself)
+ */
+void oracle_merge_views(const uint16_t *feat, int n_tiles, int grid, int n_levels, int C, int c0, int Cs,
+                        uint16_t *out, int32_t *assign)
+{
+    int side[32];
+    oracle_level_sides(grid, n_levels, side);
+    const int n0 = grid * grid;
+    int64_t lbase[33];
+    lbase[1] = 0;
+    for (int l = 1; l < n_levels; ++l) lbase[l + 1] = lbase[l] + (int64_t)n_tiles * side[l] * side[l];
+#pragma omp parallel for schedule(dynamic)
+    for (int t = 0; t < n_tiles; ++t) {
+        const uint16_t *x0 = feat + (int64_t)t * n0 * C;
+        int32_t *tok = malloc(sizeof(int32_t) * (size_t)n0);
+        float *S = malloc(sizeof(float) * (size_t)n0 * (size_t)(Cs > C ? Cs : C));
+        int32_t *size = malloc(sizeof(int32_t) * (size_t)n0);
+        float *inv = malloc(sizeof(float) * (size_t)n0);
+        float *best = malloc(sizeof(float) * (size_t)n0);
+        int32_t *best_b = malloc(sizeof(int32_t) * (size_t)n0);
+        int32_t *newpos = malloc(sizeof(int32_t) * (size_t)(2 * n0));
+        for (int i = 0; i < n0; ++i) tok[i] = i;
+        if (assign)
+            for (int i = 0; i < n0; ++i) assign[(int64_t)t * n0 + i] = i;
+        int n = n0;
+        for (int l = 1; l < n_levels; ++l) {
+            const int target = side[l] * side[l];
+            while (n > target) {
+                const int nA = (n + 1) / 2;
+                const int r = n - target < nA ? n - target : nA;
+                n = merge_round(x0, n0, tok, n, r, C, c0, Cs, S, size, inv, best, best_b, newpos);
+            }
+            member_sums(x0, n0, tok, n, C, 0, C, S, size);
+            for (int j = 0; j < n; ++j)
+                for (int c = 0; c < C; ++c)
+                    out[(lbase[l] + (int64_t)t * target + j) * C + c] =
+                        f32_to_bf16_rne(S[(int64_t)j * C + c] / (float)size[j]);
+            if (assign)
+                for (int i = 0; i < n0; ++i) assign[((int64_t)l * n_tiles + t) * n0 + i] = tok[i];
+        }
+        free(newpos);
+        free(best_b);
+        free(best);
+        free(inv);
+        free(size);
+        free(S);
+        free(tok);
+    }
 }
