@@ -12,6 +12,8 @@
  *                         the view a pooled level or the mixed view
  *   davet_step_attention  bidirectional attention over it (Sec. 3.1, Eq. 1)
  *   davet_build_views     every view once as a contiguous [view || text] block
+ *   davet_build_views_pruned, davet_build_views_merged   the same blocks from
+ *                         the pruning and merging realizers (Sec. 4.3, 5.3)
  *   davet_view_attention  the gather and the attention fused: attention reads
  *                         each request's step sequence from its view block
  *   davet_unmask_topk     argmax, confidence and confidence-ranked commit
@@ -240,6 +242,60 @@ davet_status davet_view_layout(int grid, int n_levels, int mixed_level, int mixe
  */
 davet_status davet_build_views(const void* feat, void* buf, const void* text, int n_tiles, int grid, int n_levels,
                                int mixed_level, int mixed_stride, int text_rows, int C, void* stream);
+
+/*
+ * Alternative evidence realizers (Sec. 4.3 "compatible evidence realizers":
+ * pruning varies the retention ratio, merging the aggregation strength;
+ * Sec. 5.3 / Table 2 runs the same allocation policy over pooling, pruning and
+ * merging).  Each builds the same view blocks as davet_build_views -- the
+ * same views, rows per tile (davet_view_rows), layout (davet_view_layout)
+ * and text rows -- so davet_view_attention reads them unchanged; only the
+ * rows of the views differ.  feat, buf, text and the geometry arguments are
+ * as for davet_build_views; grid <= 64 and n_tiles <= 65535 (else
+ * DAVET_ERR_UNSUPPORTED).
+ *
+ * davet_build_views_pruned -- nested visual-token pruning.  The paper leaves
+ * the importance score open; it is an input:
+ *   score  fp32 [n_tiles][grid*grid], device, the score of each token (raster
+ *          order) of each tile; a NaN ranks below every number
+ * View v keeps, per tile, the davet_view_rows(v) highest-scoring tokens
+ * (equal scores by ascending index) in raster order, so every view is a
+ * subset of each larger one; the mixed view, if any, is the one of that
+ * length.  DAVET_ERR_INVALID_ARG if a view has more rows per tile than a tile
+ * has tokens.  Enqueues two kernels.
+ *
+ * davet_build_views_merged -- hierarchical similarity merging.  Level 0 is
+ * the encoding; level l is built from level l-1 by bipartite matching rounds
+ * (positions 0, 2, 4, ... form set A, 1, 3, 5, ... set B; each member of A is
+ * matched to the member of B of highest cosine similarity, ties to the
+ * smaller B; the r = min(n - G_l^2, ceil(n/2)) best-matched members of A,
+ * ties to the smaller position, merge into their match; survivors keep their
+ * order) until it holds G_l^2 tokens, the pooled level's count.  Similarity
+ * is measured on channels [sim_c0, sim_c0 + sim_C) of the token's feature
+ * sum; each merged row is the mean of the level-0 rows it absorbed.  All of
+ * it is binary32 in a fixed order: feature sums add the members in ascending
+ * level-0 index, dot products and squared norms are fused multiply-add
+ * chains in ascending channel order, 1/|s| is a correctly rounded square
+ * root then division (0 for a zero vector), sim = (dot * 1/|a|) * 1/|b|, a
+ * row is sum / count correctly rounded then rounded to bf16 (nearest even).
+ * The mixed view, if any, is the merged coarse level plus the level-0
+ * lattice, as for pooling.  Inputs must be finite.
+ *   sim_c0, sim_C   similarity channels: sim_c0 % 8 == 0, sim_C % 32 == 0,
+ *                   sim_c0 + sim_C <= C
+ *   assign          int32 [n_levels][n_tiles][grid*grid], device, nullable:
+ *                   the level-l token each level-0 token belongs to
+ *   workspace       device, 256-byte aligned, davet_merge_workspace_bytes
+ *                   bytes; not read before it is written
+ * Enqueues four launches per round and one per level on `stream`.
+ */
+davet_status davet_build_views_pruned(const void* feat, const float* score, void* buf, const void* text, int n_tiles,
+                                      int grid, int n_levels, int mixed_level, int mixed_stride, int text_rows, int C,
+                                      void* stream);
+davet_status davet_merge_workspace_bytes(int n_tiles, int grid, int n_levels, int sim_C, size_t* bytes);
+davet_status davet_build_views_merged(const void* feat, void* buf, const void* text, int n_tiles, int grid,
+                                      int n_levels, int mixed_level, int mixed_stride, int text_rows, int C,
+                                      int sim_c0, int sim_C, int32_t* assign, void* workspace,
+                                      size_t workspace_bytes, void* stream);
 
 /*
  * davet_gather_view followed by davet_step_attention in one kernel (Eq. 5,

@@ -97,6 +97,14 @@ davet_status enqueue(const void* feat, void* pyr, int n_tiles, int grid, int n_l
                      const int64_t* off, int64_t extent, cudaStream_t st);
 }
 
+// Internal entry shared by the view-block builds (views.cu): fills every
+// block's text rows and, when compose_mixed, the mixed view's rows from the
+// coarse level's block and the level-0 lattice.
+namespace views {
+davet_status enqueue_fill(void* buf, const void* text, int n_tiles, int grid, int n_levels, int mixed_level,
+                          int mixed_stride, int text_rows, int C, bool compose_mixed, cudaStream_t st);
+}
+
 // ------------------------------------------------------------------ bf16
 __device__ __forceinline__ float bf16lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }

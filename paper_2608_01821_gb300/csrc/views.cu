@@ -83,6 +83,43 @@ __global__ void __launch_bounds__(kThreads) fill_kernel(Fill f) {
   }
 }
 
+
+davet_status enqueue_fill(void* buf, const void* text, int n_tiles, int grid, int n_levels, int mixed_level,
+                          int mixed_stride, int text_rows, int C, bool compose_mixed, cudaStream_t st) {
+  int rpt[kMaxViews];
+  int nv = 0;
+  const davet_status ls = davet_view_rows(grid, n_levels, mixed_level, mixed_stride, rpt, &nv);
+  if (ls != DAVET_OK) return ls;
+  int64_t block0[kMaxViews + 1];
+  davet_view_layout(grid, n_levels, mixed_level, mixed_stride, n_tiles, text_rows, block0);
+  Fill f;
+  f.buf = static_cast<uint4*>(buf);
+  f.text = static_cast<const uint4*>(text);
+  f.C8 = C / 8;
+  f.n_tiles = n_tiles;
+  f.text_rows = text_rows;
+  f.n_views = nv;
+  for (int v = 0; v <= kMaxViews; ++v) f.block0[v] = v <= nv ? block0[v] : block0[nv];
+  for (int v = 0; v < kMaxViews; ++v) f.rpt[v] = v < nv ? rpt[v] : 0;
+  int side[5];
+  davet_pyramid_layout(grid, n_levels, 0, side, nullptr);
+  f.mixed_view = mixed_stride != 0 ? n_levels : -1;
+  f.coarse = mixed_stride != 0 ? mixed_level : 0;
+  f.stride = mixed_stride;
+  f.lat_n = mixed_stride != 0 ? (grid - mixed_stride / 2 + mixed_stride - 1) / mixed_stride : 1;
+  f.mrows = mixed_stride != 0 ? rpt[n_levels] : 1;
+  f.g0 = grid;
+  f.gc = side[f.coarse];
+  f.n_mixed_rows = compose_mixed && mixed_stride != 0 ? static_cast<long long>(n_tiles) * f.mrows : 0;
+  f.n_rows = f.n_mixed_rows + static_cast<long long>(text_rows) * nv;
+  if (f.n_rows == 0) return DAVET_OK;
+  const long long tasks = f.n_rows * ((f.C8 + kChunk - 1) / kChunk);
+  const long long blocks = std::min<long long>((tasks + kThreads / 32 - 1) / (kThreads / 32), 152LL * 8);
+  const cudaError_t e = launch(fill_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, st, f);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
 }  // namespace views
 }  // namespace davet
 
@@ -144,30 +181,5 @@ extern "C" davet_status davet_build_views(const void* feat, void* buf, const voi
     const davet_status e = pyr::enqueue(feat, buf, n_tiles, grid, n_levels, C, nullptr, block0, block0[nv], st);
     if (e != DAVET_OK) return e;
   }
-  Fill f;
-  f.buf = static_cast<uint4*>(buf);
-  f.text = static_cast<const uint4*>(text);
-  f.C8 = C / 8;
-  f.n_tiles = n_tiles;
-  f.text_rows = text_rows;
-  f.n_views = nv;
-  for (int v = 0; v <= kMaxViews; ++v) f.block0[v] = v <= nv ? block0[v] : block0[nv];
-  for (int v = 0; v < kMaxViews; ++v) f.rpt[v] = v < nv ? rpt[v] : 0;
-  int side[5];
-  davet_pyramid_layout(grid, n_levels, 0, side, nullptr);
-  f.mixed_view = mixed_stride != 0 ? n_levels : -1;
-  f.coarse = mixed_stride != 0 ? mixed_level : 0;
-  f.stride = mixed_stride;
-  f.lat_n = mixed_stride != 0 ? (grid - mixed_stride / 2 + mixed_stride - 1) / mixed_stride : 1;
-  f.mrows = mixed_stride != 0 ? rpt[n_levels] : 1;
-  f.g0 = grid;
-  f.gc = side[f.coarse];
-  f.n_mixed_rows = mixed_stride != 0 ? static_cast<long long>(n_tiles) * f.mrows : 0;
-  f.n_rows = f.n_mixed_rows + static_cast<long long>(text_rows) * nv;
-  if (f.n_rows == 0) return DAVET_OK;
-  const long long tasks = f.n_rows * ((f.C8 + kChunk - 1) / kChunk);
-  const long long blocks = std::min<long long>((tasks + kThreads / 32 - 1) / (kThreads / 32), 152LL * 8);
-  const cudaError_t e = launch(fill_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, st, f);
-  if (e != cudaSuccess) return cuda_fail(e);
-  return check_launch();
+  return views::enqueue_fill(buf, text, n_tiles, grid, n_levels, mixed_level, mixed_stride, text_rows, C, true, st);
 }

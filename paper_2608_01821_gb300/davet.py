@@ -72,6 +72,10 @@ def _declare(lib):
         "davet_view_rows": (_int, [_int, _int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_int)]),
         "davet_view_layout": (_int, [_int, _int, _int, _int, _int, _int, ctypes.POINTER(_i64)]),
         "davet_build_views": (_int, [_vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _int, _vp]),
+        "davet_build_views_pruned": (_int, [_vp, _vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _int, _vp]),
+        "davet_merge_workspace_bytes": (_int, [_int, _int, _int, _int, ctypes.POINTER(_sz)]),
+        "davet_build_views_merged": (_int, [_vp, _vp, _vp, _int, _int, _int, _int, _int, _int, _int, _int, _int,
+                                            _vp, _vp, _sz, _vp]),
         "davet_view_attention": (_int, [_vp, _i64, _vp, _vp, _vp, _vp, _vp, _int, _int, _int, _int, _int, _int,
                                         _int, _f32, _vp, _vp, _i64, _vp]),
         "davet_unmask_topk_workspace": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
@@ -162,6 +166,30 @@ class Davet:
         self._check("davet_build_views",
                     self.lib.davet_build_views(_ptr(feat), _ptr(buf), _ptr(text), n_tiles, grid, n_levels,
                                                mixed_level, mixed_stride, text_rows, C, _stream(stream)))
+
+    def davet_build_views_pruned(self, feat, score, buf, text, n_tiles: int, grid: int, n_levels: int,
+                                 mixed_level: int, mixed_stride: int, text_rows: int, C: int, stream=None):
+        self._check("davet_build_views_pruned",
+                    self.lib.davet_build_views_pruned(_ptr(feat), _ptr(score), _ptr(buf), _ptr(text), n_tiles, grid,
+                                                      n_levels, mixed_level, mixed_stride, text_rows, C,
+                                                      _stream(stream)))
+
+    def davet_merge_workspace_bytes(self, n_tiles: int, grid: int, n_levels: int, sim_C: int) -> int:
+        n = _sz(0)
+        self._check("davet_merge_workspace_bytes",
+                    self.lib.davet_merge_workspace_bytes(n_tiles, grid, n_levels, sim_C, ctypes.byref(n)))
+        return int(n.value)
+
+    def davet_build_views_merged(self, feat, buf, text, n_tiles: int, grid: int, n_levels: int, mixed_level: int,
+                                 mixed_stride: int, text_rows: int, C: int, sim_c0: int, sim_C: int, assign=None,
+                                 workspace=None, workspace_bytes: int = 0, stream=None):
+        if workspace is not None and not isinstance(workspace, int) and workspace_bytes == 0:
+            workspace_bytes = workspace.numel() * workspace.element_size()
+        self._check("davet_build_views_merged",
+                    self.lib.davet_build_views_merged(_ptr(feat), _ptr(buf), _ptr(text), n_tiles, grid, n_levels,
+                                                      mixed_level, mixed_stride, text_rows, C, sim_c0, sim_C,
+                                                      _ptr(assign), _ptr(workspace), workspace_bytes,
+                                                      _stream(stream)))
 
     def davet_view_attention(self, store, store_rows: int, buf_row0, tiles, prompt_len, resp_len, view, batch: int,
                              grid: int, n_levels: int, mixed_level: int, mixed_stride: int, H: int, D: int,

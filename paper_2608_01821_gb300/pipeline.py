@@ -15,6 +15,11 @@ Two layouts:
                    the step input), davet_step_attention, then the unmasking.
 In both, the encoding is written where level 0 lives (the first rows of the
 request's buffer), so the build reads it in place.
+
+The fused layout takes one of three evidence realizers (Sec. 4.3, 5.3):
+"pool" (structured pooling, the default), "prune" (nested pruning by a
+per-token score the caller loads) or "merge" (hierarchical similarity
+merging on the key channels); all three give the same view lengths.
 """
 from __future__ import annotations
 
@@ -25,8 +30,13 @@ from .workloads import Workload
 
 
 class Pipeline:
-    def __init__(self, w: Workload, device="cuda", lib=None, fused: bool = True):
+    REALIZERS = ("pool", "prune", "merge")
+
+    def __init__(self, w: Workload, device="cuda", lib=None, fused: bool = True, realizer: str = "pool"):
+        if realizer not in self.REALIZERS or (realizer != "pool" and not fused):
+            raise ValueError(f"realizer {realizer!r} needs the fused layout and one of {self.REALIZERS}")
         self.w = w
+        self.realizer = realizer
         self.dev = torch.device(device)
         self.lib = lib if lib is not None else _davet.load()
         C, B = w.C, w.batch
@@ -72,6 +82,13 @@ class Pipeline:
         self.stats = torch.zeros((w.T, B, 2), dtype=torch.float32, device=self.dev)
         ws = self.lib.davet_unmask_topk_workspace(R, w.V, B)
         self.workspace = torch.zeros(max(ws, 256), dtype=torch.uint8, device=self.dev)
+        # realizer inputs: per-token scores (prune), a workspace (merge)
+        self.scores = [torch.zeros((t, w.grid * w.grid), dtype=torch.float32, device=self.dev) for t in w.tiles]
+        self.merge_ws = None
+        if realizer == "merge":
+            mw = max(self.lib.davet_merge_workspace_bytes(t, w.grid, w.n_levels, w.sim_channels()[1])
+                     for t in w.tiles)
+            self.merge_ws = torch.empty(max(mw, 256), dtype=torch.uint8, device=self.dev)
 
     # -------------------------------------------------------------- inputs
     def level0(self, b: int):
@@ -92,12 +109,16 @@ class Pipeline:
             parts.append(self.bufs[b][r0:r0 + w.tiles[b] * g * g])
         return torch.cat(parts).cpu()
 
-    def load_inputs(self, feats, text, non_blocking=False):
-        """feats: per-request bf16 [tiles, G, G, C]; text: bf16 [sum(P+R), C]."""
+    def load_inputs(self, feats, text, non_blocking=False, scores=None):
+        """feats: per-request bf16 [tiles, G, G, C]; text: bf16 [sum(P+R), C];
+        scores (pruning realizer): per-request fp32 [tiles, G*G]."""
         for b, f in enumerate(feats):
             self.level0(b).copy_(f.reshape(-1, self.w.C), non_blocking=non_blocking)
         if self.w.total_text():
             self.text[: self.w.total_text()].copy_(text, non_blocking=non_blocking)
+        if scores is not None:
+            for b, s in enumerate(scores):
+                self.scores[b].copy_(s.reshape(self.scores[b].shape), non_blocking=non_blocking)
 
     def reset_state(self):
         self.masked.fill_(1)
@@ -113,8 +134,15 @@ class Pipeline:
             if self.fused:
                 t0 = int(self.text_off_host[b])
                 n = w.prompt[b] + w.resp[b]
-                self.lib.davet_build_views(v, v, self.text[t0:t0 + n] if n else None, w.tiles[b], w.grid, w.n_levels,
-                                           *w.mixed_args, n, w.C, stream)
+                text = self.text[t0:t0 + n] if n else None
+                geo = (w.tiles[b], w.grid, w.n_levels, *w.mixed_args, n, w.C)
+                if self.realizer == "pool":
+                    self.lib.davet_build_views(v, v, text, *geo, stream)
+                elif self.realizer == "prune":
+                    self.lib.davet_build_views_pruned(v, self.scores[b], v, text, *geo, stream)
+                else:
+                    self.lib.davet_build_views_merged(v, v, text, *geo, *w.sim_channels(), None, self.merge_ws,
+                                                      stream=stream)
             else:
                 self.lib.davet_build_pyramid(v, v, w.tiles[b], w.grid, w.n_levels, w.C, None, stream)
 

@@ -87,7 +87,7 @@ def derive_seed(*parts: int) -> int:
 
 
 # tensor kinds for derive_seed
-KIND_FEAT, KIND_TEXT, KIND_LOGITS, KIND_QKV = 1, 2, 3, 4
+KIND_FEAT, KIND_TEXT, KIND_LOGITS, KIND_QKV, KIND_SCORE = 1, 2, 3, 4, 5
 
 
 @dataclasses.dataclass
@@ -142,6 +142,11 @@ class Workload:
         coarse, s = self.mixed
         n = len(range(s // 2, self.grid, s))
         return self.level_sides()[coarse] ** 2 + n * n
+
+    def sim_channels(self) -> tuple[int, int]:
+        """(first channel, count) the merging realizer measures similarity on:
+        the key slice [H*D, 2*H*D) of each packed [q | k | v] row."""
+        return self.H * self.D, self.H * self.D
 
     def n_views(self) -> int:
         return self.n_levels + (1 if self.mixed else 0)
@@ -274,6 +279,15 @@ def text_rows(w: Workload):
     parts = [normal_bf16((w.prompt[b] + w.resp[b], w.C), derive_seed(w.seed, KIND_TEXT, b))
              for b in range(w.batch)]
     return torch.cat(parts, 0)
+
+
+def token_scores(w: Workload, b: int):
+    """Importance score of every visual token of request b for the pruning
+    realizer (the paper leaves the score open): fp32 [tiles, G*G] ~ N(0,1)."""
+    import torch
+    g = torch.Generator(device="cpu")
+    g.manual_seed(derive_seed(w.seed, KIND_SCORE, b))
+    return torch.randn((w.tiles[b], w.grid * w.grid), generator=g, dtype=torch.float32)
 
 
 def logits(w: Workload, t: int):

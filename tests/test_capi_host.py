@@ -97,6 +97,25 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_view_rows(27, 4, 0, 0, None, ctypes.byref(nv)) == 0 and nv.value == 4
     assert lib.davet_view_layout(27, 4, 5, 3, 2, 50, off) == INV
     assert lib.davet_build_views(p, p, null, 1, 27, 4, 0, 0, 5, 16, null) == INV  # text rows without text
+    # realizers: pruning needs a score and cannot keep more rows than a tile has
+    assert lib.davet_build_views_pruned(p, null, p, null, 1, 27, 4, 0, 0, 0, 16, null) == INV
+    assert lib.davet_build_views_pruned(p, p, p, null, 1, 27, 4, 2, 1, 0, 16, null) == INV  # 49 + 729 rows
+    assert lib.davet_build_views_pruned(p, p, p, null, 1, 65, 4, 0, 0, 0, 16, null) == UNS
+    assert lib.davet_build_views_pruned(null, null, null, null, 0, 27, 4, 0, 0, 0, 16, null) == 0  # empty
+    # merging: similarity channels, workspace size, geometry limits
+    ws = ctypes.c_size_t(0)
+    assert lib.davet_merge_workspace_bytes(10, 27, 4, 4096, ctypes.byref(ws)) == 0 and ws.value > 0
+    ws10 = ws.value
+    assert lib.davet_merge_workspace_bytes(1, 27, 4, 4096, ctypes.byref(ws)) == 0 and ws.value < ws10
+    assert lib.davet_merge_workspace_bytes(1, 27, 4, 48, ctypes.byref(ws)) == INV
+    assert lib.davet_merge_workspace_bytes(1, 65, 4, 64, ctypes.byref(ws)) == UNS
+    mw = ctypes.c_void_p(1 << 24)
+    assert lib.davet_build_views_merged(p, p, null, 1, 27, 4, 0, 0, 0, 128, 0, 48, null, mw, ws10, null) == INV
+    assert lib.davet_build_views_merged(p, p, null, 1, 27, 4, 0, 0, 0, 128, 104, 32, null, mw, ws10, null) == INV
+    assert lib.davet_build_views_merged(p, p, null, 1, 27, 4, 0, 0, 0, 128, 4, 32, null, mw, ws10, null) == INV
+    assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, mw, 1024, null) == INV
+    assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, null, ws10, null) == INV
+    assert lib.davet_build_views_merged(null, null, null, 0, 27, 4, 0, 0, 0, 128, 0, 32, null, null, 0, null) == 0
     # gather: bad levels count, batch too large
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 0, 0, 16, p, p, 100, null) == INV
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 0, 0, 16, p, p, 100, null) == UNS
