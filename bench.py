@@ -148,10 +148,12 @@ def run_ours(args, rank, world, local_rank):
     w = workloads.make(args.config)
     if rank > 0:
         w.seed = w.seed + 1000 * rank  # each replica gets its own batch
-    pl = Pipeline(w, dev, lib, fused=not getattr(args, "unfused", False))
+    realizer = getattr(args, "realizer", "pool")
+    pl = Pipeline(w, dev, lib, fused=not getattr(args, "unfused", False), realizer=realizer)
     feats = [workloads.features(w, b) for b in range(w.batch)]
     text = workloads.text_rows(w)
-    pl.load_inputs(feats, text)
+    scores = [workloads.token_scores(w, b) for b in range(w.batch)] if realizer == "prune" else None
+    pl.load_inputs(feats, text, scores=scores)
     torch.cuda.synchronize()
 
     # step logits: a pool of distinct device buffers, step t uses t % P
@@ -222,10 +224,10 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0:
         peaks = measured_peaks()
         value = whole_job_rate(w.T * args.steps, world, total_s)
-        # per request the view-block build (pyramid + fill kernels) or the
+        # per request the view-block build (realizer + fill kernels) or the
         # pyramid; per step the fused view attention (or gather and attention)
         # and the two unmask kernels
-        launches_per_pass = (2 * w.batch + w.T * 3) if pl.fused else (w.batch + w.T * 4)
+        launches_per_pass = build_launches(w, pl.realizer, pl.fused) + w.T * (3 if pl.fused else 4)
         akey = "view_attention" if pl.fused else "attention"
         attn_flops_launch = comp[akey]["flops"] / comp[akey]["launches"]
         attn_ms = comp[akey]["ms"] / comp[akey]["launches"]
@@ -258,6 +260,7 @@ def run_ours(args, rank, world, local_rank):
                 "timing": "CUDA events per pass on the launching stream; one CUDA graph per pass",
                 "l2": f"{L2_FLUSH_BYTES >> 20} MiB write between timed passes (not timed)",
                 "logit_pool": P,
+                "realizer": pl.realizer,
             },
             "components": {
                 k: ({kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in v.items()}
@@ -282,6 +285,39 @@ def run_ours(args, rank, world, local_rank):
             "wall_s_timed": round(wall, 3),
         }
     return out
+
+
+def merge_round_count(grid: int, n_levels: int) -> int:
+    """Bipartite matching rounds the merging realizer runs per tile: level l
+    is reached from n tokens by rounds of r = min(n - G_l^2, ceil(n/2))."""
+    sides, g = [], grid
+    for _ in range(n_levels):
+        sides.append(g)
+        g = (g + 1) // 2
+    n, rounds = grid * grid, 0
+    for g in sides[1:]:
+        while n > g * g:
+            n -= min(n - g * g, (n + 1) // 2)
+            rounds += 1
+    return rounds
+
+
+def build_launches(w, realizer: str, fused: bool) -> int:
+    """Kernels the view construction of one pass launches (all requests)."""
+    if not fused:
+        return sum(1 for t in w.tiles if t > 0)
+    n = 0
+    for b in range(w.batch):
+        has_text = w.prompt[b] + w.resp[b] > 0
+        if w.tiles[b] > 0:
+            if realizer == "merge":
+                R = merge_round_count(w.grid, w.n_levels)
+                n += 1 + 3 * R + (w.n_levels - 1)  # init, rounds, level rows
+            else:
+                n += 1  # pyramid or pruning kernel
+        if has_text or (w.mixed and realizer != "prune" and w.tiles[b] > 0):
+            n += 1  # text (and mixed) fill
+    return n
 
 
 def kernel_times(pl, w, pool, P, stream, reps=3):
@@ -352,11 +388,19 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
     gbytes = sum(w.gather_bytes(t) for t in range(w.T))
     ubytes = sum(w.unmask_bytes(t) for t in range(w.T))
     pbytes = w.pyramid_bytes()
-    out = {
-        "timing_mode": mode,
-        "pyramid": {"launches": w.batch, "ms": ms["pyramid"], "bytes": pbytes,
-                    "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9},
-    }
+    nb = build_launches(w, pl.realizer, pl.fused)
+    if pl.realizer == "pool":
+        out = {
+            "timing_mode": mode,
+            "pyramid": {"launches": nb, "ms": ms["pyramid"], "bytes": pbytes,
+                        "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9},
+        }
+    else:
+        out = {
+            "timing_mode": mode,
+            "views_build": {"realizer": pl.realizer, "launches": nb, "ms": ms["pyramid"],
+                            "ms_per_request": ms["pyramid"] / max(w.batch, 1)},
+        }
     if pl.fused:
         out["view_attention"] = {"launches": w.T, "ms": ms["view_attention"], "flops": flops,
                                  "TFLOPs": flops / (ms["view_attention"] * 1e-3) / 1e12}
@@ -386,6 +430,8 @@ def run_e2e(args, pl, w, dev, stream, world):
     from paper_2608_01821_gb300 import workloads
     feats = [workloads.features(w, b).pin_memory() for b in range(w.batch)]
     text = workloads.text_rows(w).pin_memory()
+    scores = ([workloads.token_scores(w, b).pin_memory() for b in range(w.batch)] if pl.realizer == "prune"
+              else None)
     P = 4
     host_logits = [workloads.logits(w, t).pin_memory() for t in range(P)]
     NB = 3
@@ -395,6 +441,8 @@ def run_e2e(args, pl, w, dev, stream, world):
     tokens_host = torch.empty(w.total_resp, dtype=torch.int32).pin_memory()
     logit_rows = sum(w.masked_rows(t) for t in range(w.T)) if mapped else w.T * w.total_resp
     h2d = sum(f.numel() * 2 for f in feats) + text.numel() * 2 + logit_rows * w.V * 2
+    if scores is not None:
+        h2d += sum(x.numel() * 4 for x in scores)
     d2h = w.total_resp * 4
     copy_stream = torch.cuda.Stream(device=dev)
     ready = [torch.cuda.Event() for _ in range(NB)]
@@ -411,7 +459,7 @@ def run_e2e(args, pl, w, dev, stream, world):
 
     def one_mapped():
         pl.reset_state()
-        pl.load_inputs(feats, text, non_blocking=True)
+        pl.load_inputs(feats, text, non_blocking=True, scores=scores)
         pl.build_pyramids()
         for t in range(w.T):
             pl.step(t, host_logits[t % P])
@@ -423,7 +471,7 @@ def run_e2e(args, pl, w, dev, stream, world):
         for t in range(min(NB, w.T)):
             issue_copy(t)
         pl.reset_state()
-        pl.load_inputs(feats, text, non_blocking=True)
+        pl.load_inputs(feats, text, non_blocking=True, scores=scores)
         pl.build_pyramids()
         for t in range(w.T):
             slot = t % NB
@@ -604,8 +652,10 @@ def run_profile(args):
     dev = torch.device("cuda", 0)
     lib = davet.load()
     w = workloads.make(args.config)
-    pl = Pipeline(w, dev, lib)
-    pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w))
+    realizer = getattr(args, "realizer", "pool")
+    pl = Pipeline(w, dev, lib, realizer=realizer)
+    pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w),
+                   scores=[workloads.token_scores(w, b) for b in range(w.batch)] if realizer == "prune" else None)
     t = args.profile_step
     lg = workloads.logits_device(w, t, dev)
     pl.build_pyramids()
@@ -678,6 +728,8 @@ def main(argv=None):
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)
+    ap.add_argument("--realizer", choices=["pool", "prune", "merge"], default="pool",
+                    help="evidence realizer of the view blocks (Sec. 4.3): pooling (default), pruning or merging")
     args = ap.parse_args(argv)
     rank, world, local = dist_env()
     if args.profile:

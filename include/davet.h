@@ -286,7 +286,7 @@ davet_status davet_build_views(const void* feat, void* buf, const void* text, in
  *                   the level-l token each level-0 token belongs to
  *   workspace       device, 256-byte aligned, davet_merge_workspace_bytes
  *                   bytes; not read before it is written
- * Enqueues four launches per round and one per level on `stream`.
+ * Enqueues three launches per round and one per level on `stream`.
  */
 davet_status davet_build_views_pruned(const void* feat, const float* score, void* buf, const void* text, int n_tiles,
                                       int grid, int n_levels, int mixed_level, int mixed_stride, int text_rows, int C,

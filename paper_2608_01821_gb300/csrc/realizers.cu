@@ -12,21 +12,24 @@
 // 4 KB row chunk.  The sort is repeated by each CTA of a tile; it is a few
 // microseconds, and it saves a workspace and a launch.
 //
-// Merging: bipartite matching rounds per level, each round three or four
-// launches over all tiles of the request:
+// Merging: bipartite matching rounds per level, each round three launches
+// over all tiles of the request:
 //   sum_kernel    feature sums S of the current tokens (members in ascending
 //                 level-0 index, binary32) over the similarity channels;
-//   norm_kernel   1/|S| per token (fused multiply-add chain, then correctly
-//                 rounded square root and division);
 //   sim_kernel    the A x B cosine block (A = even, B = odd positions): a
-//                 64 x 64 register-blocked fp32 product whose every output
-//                 accumulates its channels in ascending order with fused
-//                 multiply-adds, then the row-wise best match per B block;
+//                 register-blocked fp32 product over channel stages streamed
+//                 into shared memory by a cp.async ring, every output
+//                 accumulating its channels in ascending order with fused
+//                 multiply-adds; the squared-norm chains of the staged rows
+//                 run alongside (then a correctly rounded square root and
+//                 division), and each A row's best match per B block is
+//                 written out.  The block shape is chosen per round (64, 32
+//                 or 16 rows a side) so that small late rounds still spread
+//                 over the SMs;
 //   select_kernel one CTA per tile: best match over the B blocks, the r
 //                 best-matched members of A, the new token of every level-0
 //                 token, and the member lists of the new tokens (stable).
-// The first round reads the encoding (bf16) directly instead of sums.  When a
-// level is complete, sum_kernel writes its rows as member means (bf16).
+// When a level is complete, sum_kernel writes its rows as member means (bf16).
 // The merge decisions are taken in binary32 with this fixed operation order
 // on purpose: the products are CUDA-core fused multiply-adds rather than
 // tensor-core MMAs, whose internal accumulation order is not specified, so
@@ -178,21 +181,35 @@ __global__ void __launch_bounds__(kThreads) prune_kernel(Prune p) {
 //   tok     int32 [n_tiles][n0]      current token of each level-0 token
 //   start   int32 [n_tiles][n0 + 1]  member-list offsets of the current tokens
 //   members int32 [n_tiles][n0]      level-0 indices, ascending per token
-//   inv     f32   [n_tiles][n0]      1/|S| of each current token
 //   best    Best  [n_tiles][bblk][nA] best match of each member of A per B block
-//   S       f32   [n_tiles][s_rows][Cs] similarity-channel sums (rounds 2+)
+//   S       f32   [n_tiles][n0][Cs]  similarity-channel sums of the current tokens
 struct Best {
   float s;
   int b;
 };
 
+// Similarity block shapes: TM x TM members of A by B per CTA, RM x RM
+// products per thread, KC channels per pipeline stage, STAGES stages.
+template <int TM_, int RM_, int KC_, int STAGES_>
+struct SimShape {
+  static constexpr int TM = TM_, RM = RM_, KC = KC_, STAGES = STAGES_;
+  static constexpr int NT = (TM / RM) * (TM / RM);
+  static constexpr int PITCH = KC + 4;  // floats per staged row: 16-byte aligned, 4-bank offset per row
+  static constexpr int CHUNKS = TM * KC / 4 / NT;  // 16-byte copies per operand per thread per stage
+  static constexpr size_t SMEM = static_cast<size_t>(STAGES) * 2 * TM * PITCH * 4 + 2 * TM * 4;
+  static_assert(NT >= 2 * TM, "the norm chains need one thread per staged row");
+  static_assert(TM * KC / 4 % NT == 0, "stage copies must divide evenly");
+};
+using SimLarge = SimShape<64, 4, 32, 3>;
+using SimMid = SimShape<32, 4, 32, 4>;
+using SimSmall = SimShape<16, 2, 32, 6>;
+
 struct Plan {
   int n0, n_levels;
   int side[5];
   std::vector<int> n, r, level;  // per round: tokens before, merged, level it builds
-  int s_rows;                    // rows of S (largest n of a round after the first)
   int nA_max, bblk_max;
-  size_t off_tok, off_start, off_members, off_inv, off_best, off_S, bytes;
+  size_t off_tok, off_start, off_members, off_best, off_S, bytes;
 };
 
 inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -203,7 +220,6 @@ inline Plan make_plan(int n_tiles, int grid, int n_levels, int Cs) {
   P.n_levels = n_levels;
   davet_pyramid_layout(grid, n_levels, 0, P.side, nullptr);
   int n = P.n0;
-  P.s_rows = 0;
   P.nA_max = 1;
   P.bblk_max = 1;
   for (int l = 1; l < n_levels; ++l) {
@@ -211,12 +227,11 @@ inline Plan make_plan(int n_tiles, int grid, int n_levels, int Cs) {
     while (n > target) {
       const int nA = (n + 1) / 2, nB = n / 2;
       const int r = std::min(n - target, nA);
-      if (!P.n.empty()) P.s_rows = std::max(P.s_rows, n);
       P.n.push_back(n);
       P.r.push_back(r);
       P.level.push_back(l);
       P.nA_max = std::max(P.nA_max, nA);
-      P.bblk_max = std::max(P.bblk_max, (nB + 63) / 64);
+      P.bblk_max = std::max(P.bblk_max, (nB + SimSmall::TM - 1) / SimSmall::TM);
       n -= r;
     }
   }
@@ -228,12 +243,10 @@ inline Plan make_plan(int n_tiles, int grid, int n_levels, int Cs) {
   o = align256(o + T * (P.n0 + 1) * 4);
   P.off_members = o;
   o = align256(o + T * P.n0 * 4);
-  P.off_inv = o;
-  o = align256(o + T * P.n0 * 4);
   P.off_best = o;
   o = align256(o + T * P.bblk_max * P.nA_max * sizeof(Best));
   P.off_S = o;
-  o = align256(o + T * static_cast<size_t>(P.s_rows) * Cs * 4);
+  o = align256(o + (P.n.empty() ? 0 : T * static_cast<size_t>(P.n0) * Cs * 4));
   P.bytes = o;
   return P;
 }
@@ -246,10 +259,8 @@ struct MergeArgs {
   int32_t* tok;
   int32_t* start;
   int32_t* members;
-  float* inv;
   Best* best;
   float* S;
-  int s_rows;
   int n, nA, nB, bblk, r;
 };
 
@@ -270,139 +281,129 @@ __global__ void __launch_bounds__(kThreads) init_kernel(MergeArgs a, int32_t* as
   }
 }
 
-// 1/|S_j| for the n current tokens of every tile.  BF: the tokens are the
-// level-0 rows themselves (first round), read from the encoding.
-template <bool BF>
-__global__ void __launch_bounds__(kThreads) norm_kernel(MergeArgs a) {
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// One stage of the A and B rows of this CTA: TM rows x KC channels each,
+// 16-byte cp.async copies (rows past the set end are zero-filled).
+template <class SH>
+__device__ __forceinline__ void sim_stage(const MergeArgs& a, const float* St, int a0, int b0, int k0,
+                                          float* sa, float* sb) {
+  constexpr int CPR = SH::KC / 4;  // 16-byte chunks per staged row
+#pragma unroll
+  for (int u = 0; u < SH::CHUNKS; ++u) {
+    const int q = threadIdx.x + u * SH::NT;
+    const int row = q / CPR, c = q % CPR;
+    const bool va = a0 + row < a.nA, vb = b0 + row < a.nB;
+    const float* pa = St + static_cast<long long>(va ? 2 * (a0 + row) : 0) * a.Cs + k0 + c * 4;
+    const float* pb = St + static_cast<long long>(vb ? 2 * (b0 + row) + 1 : 0) * a.Cs + k0 + c * 4;
+    cp_async16(smem_u32(sa + row * SH::PITCH + c * 4), pa, va ? 16 : 0);
+    cp_async16(smem_u32(sb + row * SH::PITCH + c * 4), pb, vb ? 16 : 0);
+  }
+}
+
+// A x B cosine block (A = even, B = odd positions) of one tile: every
+// product accumulates its channels in ascending order by fused multiply-adds;
+// threads 0..TM-1 (2*TM-1) also run the squared-norm chains of the staged A
+// (B) rows over the same stages.  Then each A row's best match in the block.
+// Thread (ty, tx) owns rows ty + i*(TM/RM) of A and tx + j*(TM/RM) of B.
+template <class SH>
+__global__ void __launch_bounds__(SH::NT) sim_kernel(MergeArgs a) {
+  extern __shared__ __align__(16) float sm[];
+  float* sA = sm;                                        // [STAGES][TM][PITCH]
+  float* sB = sA + SH::STAGES * SH::TM * SH::PITCH;      // [STAGES][TM][PITCH]
+  float* invA = sB + SH::STAGES * SH::TM * SH::PITCH;    // [TM]
+  float* invB = invA + SH::TM;                           // [TM]
+  constexpr int TD = SH::TM / SH::RM;
   pdl_launch_dependents();
   pdl_wait();
-  const long long total = static_cast<long long>(a.n_tiles) * a.n;
-  for (long long q = static_cast<long long>(blockIdx.x) * kThreads + threadIdx.x; q < total;
-       q += static_cast<long long>(gridDim.x) * kThreads) {
-    const int t = static_cast<int>(q / a.n), j = static_cast<int>(q % a.n);
-    float n2 = 0.0f;
-    if constexpr (BF) {
-      const uint4* row = a.feat + (static_cast<long long>(t) * a.n0 + j) * a.C8 + a.c0_8;
-      for (int u = 0; u < a.Cs / 8; ++u) {
-        const uint4 x = row[u];
-        const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+  const int t = blockIdx.z;
+  const int a0 = blockIdx.x * SH::TM, b0 = blockIdx.y * SH::TM;
+  const int tx = threadIdx.x % TD, ty = threadIdx.x / TD;
+  const float* St = a.S + static_cast<long long>(t) * a.n0 * a.Cs;
+  const int nk = a.Cs / SH::KC;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float lo = bf16lo(w[e]), hi = bf16hi(w[e]);
-          n2 = __fmaf_rn(lo, lo, n2);
-          n2 = __fmaf_rn(hi, hi, n2);
-        }
-      }
-    } else {
-      const float4* row =
-          reinterpret_cast<const float4*>(a.S + (static_cast<long long>(t) * a.s_rows + j) * a.Cs);
-      for (int u = 0; u < a.Cs / 4; ++u) {
-        const float4 x = row[u];
+  for (int s = 0; s < SH::STAGES - 1; ++s) {
+    if (s < nk) sim_stage<SH>(a, St, a0, b0, s * SH::KC, sA + s * SH::TM * SH::PITCH, sB + s * SH::TM * SH::PITCH);
+    cp_async_commit();
+  }
+  float acc[SH::RM][SH::RM];
+#pragma unroll
+  for (int i = 0; i < SH::RM; ++i)
+#pragma unroll
+    for (int j = 0; j < SH::RM; ++j) acc[i][j] = 0.0f;
+  float n2 = 0.0f;
+  const bool chainA = threadIdx.x < SH::TM, chainB = !chainA && threadIdx.x < 2 * SH::TM;
+  const int crow = chainA ? threadIdx.x : threadIdx.x - SH::TM;
+  for (int kb = 0; kb < nk; ++kb) {
+    cp_async_wait_group<SH::STAGES - 2>();
+    __syncthreads();
+    {  // refill the stage consumed last iteration
+      const int kn = kb + SH::STAGES - 1;
+      const int sn = kn % SH::STAGES;
+      if (kn < nk)
+        sim_stage<SH>(a, St, a0, b0, kn * SH::KC, sA + sn * SH::TM * SH::PITCH, sB + sn * SH::TM * SH::PITCH);
+      cp_async_commit();
+    }
+    const float* A = sA + (kb % SH::STAGES) * SH::TM * SH::PITCH;
+    const float* B = sB + (kb % SH::STAGES) * SH::TM * SH::PITCH;
+    if (chainA || chainB) {
+      const float* row = (chainA ? A : B) + crow * SH::PITCH;
+#pragma unroll 4
+      for (int k = 0; k < SH::KC; k += 4) {
+        const float4 x = *reinterpret_cast<const float4*>(row + k);
         n2 = __fmaf_rn(x.x, x.x, n2);
         n2 = __fmaf_rn(x.y, x.y, n2);
         n2 = __fmaf_rn(x.z, x.z, n2);
         n2 = __fmaf_rn(x.w, x.w, n2);
       }
     }
-    a.inv[static_cast<long long>(t) * a.n0 + j] = n2 > 0.0f ? __fdiv_rn(1.0f, __fsqrt_rn(n2)) : 0.0f;
-  }
-}
-
-// A x B similarity block of 64 members of A by 64 of B, 256 threads each
-// holding 4 x 4 products; channels staged 32 at a time in shared memory
-// (transposed, [channel][row]).  Then each row's best match in this B block.
-constexpr int kSimTile = 64;
-constexpr int kSimK = 32;
-constexpr int kSimPitch = kSimTile + 4;
-
-template <bool BF>
-__device__ __forceinline__ void sim_load(const MergeArgs& a, int t, int pos, bool valid, int k0, int cg,
-                                         float (&v)[8]) {
-  if (!valid) {
+#pragma unroll 1
+    for (int k = 0; k < SH::KC; k += 4) {
+      float4 x[SH::RM], y[SH::RM];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = 0.0f;
-    return;
-  }
-  if constexpr (BF) {
-    const uint4 x = a.feat[(static_cast<long long>(t) * a.n0 + pos) * a.C8 + a.c0_8 + (k0 + cg * 8) / 8];
-    v[0] = bf16lo(x.x); v[1] = bf16hi(x.x);
-    v[2] = bf16lo(x.y); v[3] = bf16hi(x.y);
-    v[4] = bf16lo(x.z); v[5] = bf16hi(x.z);
-    v[6] = bf16lo(x.w); v[7] = bf16hi(x.w);
-  } else {
-    const float4* s =
-        reinterpret_cast<const float4*>(a.S + (static_cast<long long>(t) * a.s_rows + pos) * a.Cs + k0 + cg * 8);
-    const float4 x = s[0], y = s[1];
-    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
-    v[4] = y.x; v[5] = y.y; v[6] = y.z; v[7] = y.w;
-  }
-}
-
-template <bool BF>
-__global__ void __launch_bounds__(kThreads) sim_kernel(MergeArgs a) {
-  __shared__ __align__(16) float As[kSimK][kSimPitch];
-  __shared__ __align__(16) float Bs[kSimK][kSimPitch];
-  pdl_launch_dependents();
-  pdl_wait();
-  const int t = blockIdx.z;
-  const int a0 = blockIdx.x * kSimTile, b0 = blockIdx.y * kSimTile;
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  // loader: row = tid % 64 (a warp covers 32 consecutive rows), 8 channels
-  const int lrow = threadIdx.x & 63, cg = threadIdx.x >> 6;
-  const bool va = a0 + lrow < a.nA, vb = b0 + lrow < a.nB;
-  const int pa = 2 * (a0 + lrow), pb = 2 * (b0 + lrow) + 1;
-  float acc[4][4];
+      for (int i = 0; i < SH::RM; ++i) x[i] = *reinterpret_cast<const float4*>(A + (ty + i * TD) * SH::PITCH + k);
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+      for (int j = 0; j < SH::RM; ++j) y[j] = *reinterpret_cast<const float4*>(B + (tx + j * TD) * SH::PITCH + k);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-  float ra[8], rb[8];
-  sim_load<BF>(a, t, pa, va, 0, cg, ra);
-  sim_load<BF>(a, t, pb, vb, 0, cg, rb);
-  for (int k0 = 0; k0 < a.Cs; k0 += kSimK) {
+      for (int i = 0; i < SH::RM; ++i)
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      As[cg * 8 + e][lrow] = ra[e];
-      Bs[cg * 8 + e][lrow] = rb[e];
+        for (int j = 0; j < SH::RM; ++j) {
+          acc[i][j] = __fmaf_rn(x[i].x, y[j].x, acc[i][j]);
+          acc[i][j] = __fmaf_rn(x[i].y, y[j].y, acc[i][j]);
+          acc[i][j] = __fmaf_rn(x[i].z, y[j].z, acc[i][j]);
+          acc[i][j] = __fmaf_rn(x[i].w, y[j].w, acc[i][j]);
+        }
     }
-    __syncthreads();
-    if (k0 + kSimK < a.Cs) {
-      sim_load<BF>(a, t, pa, va, k0 + kSimK, cg, ra);
-      sim_load<BF>(a, t, pb, vb, k0 + kSimK, cg, rb);
-    }
-#pragma unroll 8
-    for (int k = 0; k < kSimK; ++k) {
-      const float4 x = *reinterpret_cast<const float4*>(&As[k][ty * 4]);
-      const float4 y = *reinterpret_cast<const float4*>(&Bs[k][tx * 4]);
-      const float xa[4] = {x.x, x.y, x.z, x.w}, yb[4] = {y.x, y.y, y.z, y.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = __fmaf_rn(xa[i], yb[j], acc[i][j]);
-    }
-    __syncthreads();
   }
-  const float* inv = a.inv + static_cast<long long>(t) * a.n0;
+  cp_async_wait_group<0>();
+  if (chainA || chainB) (chainA ? invA : invB)[crow] = n2 > 0.0f ? __fdiv_rn(1.0f, __fsqrt_rn(n2)) : 0.0f;
+  __syncthreads();
+  // best match of each owned A row among the owned B columns, then across
+  // the TD threads sharing the row (ties to the smaller b)
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int ai = a0 + ty * 4 + i;
-    const float ia = ai < a.nA ? inv[2 * ai] : 0.0f;
+  for (int i = 0; i < SH::RM; ++i) {
+    const int ra = ty + i * TD;
+    const int ai = a0 + ra;
     float bs = 0.0f;
     int bb = -1;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int bj = b0 + tx * 4 + j;
+    for (int j = 0; j < SH::RM; ++j) {
+      const int rb = tx + j * TD;
+      const int bj = b0 + rb;
       if (ai < a.nA && bj < a.nB) {
-        const float s = __fmul_rn(__fmul_rn(acc[i][j], ia), inv[2 * bj + 1]);
-        if (bb < 0 || s > bs) {
-          bs = s;
+        const float sc = __fmul_rn(__fmul_rn(acc[i][j], invA[ra]), invB[rb]);
+        if (bb < 0 || sc > bs || (sc == bs && bj < bb)) {
+          bs = sc;
           bb = bj;
         }
       }
     }
-    // best over the 16 lanes of this row group (ties to the smaller b)
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) {
+    for (int o = TD / 2; o > 0; o >>= 1) {
       const float os = __shfl_xor_sync(0xffffffffu, bs, o);
       const int ob = __shfl_xor_sync(0xffffffffu, bb, o);
       if (ob >= 0 && (bb < 0 || os > bs || (os == bs && ob < bb))) {
@@ -552,7 +553,7 @@ __global__ void __launch_bounds__(kThreads) sum_kernel(MergeArgs a, uint4* out, 
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[e] = k == m0 ? v[e] : __fadd_rn(acc[e], v[e]);
       }
-      reinterpret_cast<float4*>(a.S + (static_cast<long long>(t) * a.s_rows + j) * a.Cs)[g] =
+      reinterpret_cast<float4*>(a.S + (static_cast<long long>(t) * a.n0 + j) * a.Cs)[g] =
           make_float4(acc[0], acc[1], acc[2], acc[3]);
     }
   }
@@ -686,10 +687,8 @@ extern "C" davet_status davet_build_views_merged(const void* feat, void* buf, co
     a.tok = reinterpret_cast<int32_t*>(ws + P.off_tok);
     a.start = reinterpret_cast<int32_t*>(ws + P.off_start);
     a.members = reinterpret_cast<int32_t*>(ws + P.off_members);
-    a.inv = reinterpret_cast<float*>(ws + P.off_inv);
     a.best = reinterpret_cast<Best*>(ws + P.off_best);
     a.S = reinterpret_cast<float*>(ws + P.off_S);
-    a.s_rows = P.s_rows;
     a.n = P.n0;
     a.nA = a.nB = a.bblk = a.r = 0;
     uint4* out = static_cast<uint4*>(buf);
@@ -708,25 +707,34 @@ extern "C" davet_status davet_build_views_merged(const void* feat, void* buf, co
     cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(std::max<size_t>(max_sel, 1024)));
     if (e != cudaSuccess) return cuda_fail(e);
+    e = cudaFuncSetAttribute(sim_kernel<SimLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(SimLarge::SMEM));
+    if (e != cudaSuccess) return cuda_fail(e);
     for (size_t k = 0; k < P.n.size(); ++k) {
       a.n = P.n[k];
       a.r = P.r[k];
       a.nA = (a.n + 1) / 2;
       a.nB = a.n / 2;
-      a.bblk = (a.nB + kSimTile - 1) / kSimTile;
       const long long tok_work = static_cast<long long>(n_tiles) * a.n;
-      const dim3 sg((a.nA + kSimTile - 1) / kSimTile, a.bblk, n_tiles);
-      if (k == 0) {
-        s = ok(launch(norm_kernel<true>, dim3(grid_for(tok_work, kThreads)), dim3(kThreads), 0, st, a));
-        if (s != DAVET_OK) return s;
-        s = ok(launch(sim_kernel<true>, sg, dim3(kThreads), 0, st, a));
+      s = ok(launch(sum_kernel<false>, dim3(grid_for(tok_work * (sim_C / 4), kThreads)), dim3(kThreads), 0, st, a,
+                    static_cast<uint4*>(nullptr), 0LL, a.n));
+      if (s != DAVET_OK) return s;
+      // the largest block shape that still gives about two CTAs per SM
+      auto ctas = [&](int tm) {
+        return static_cast<long long>((a.nA + tm - 1) / tm) * ((a.nB + tm - 1) / tm) * n_tiles;
+      };
+      if (ctas(SimLarge::TM) >= 2 * 152) {
+        a.bblk = (a.nB + SimLarge::TM - 1) / SimLarge::TM;
+        s = ok(launch(sim_kernel<SimLarge>, dim3((a.nA + SimLarge::TM - 1) / SimLarge::TM, a.bblk, n_tiles),
+                      dim3(SimLarge::NT), SimLarge::SMEM, st, a));
+      } else if (ctas(SimMid::TM) >= 2 * 152) {
+        a.bblk = (a.nB + SimMid::TM - 1) / SimMid::TM;
+        s = ok(launch(sim_kernel<SimMid>, dim3((a.nA + SimMid::TM - 1) / SimMid::TM, a.bblk, n_tiles),
+                      dim3(SimMid::NT), SimMid::SMEM, st, a));
       } else {
-        s = ok(launch(sum_kernel<false>, dim3(grid_for(tok_work * (sim_C / 4), kThreads)), dim3(kThreads), 0, st,
-                      a, static_cast<uint4*>(nullptr), 0LL, a.n));
-        if (s != DAVET_OK) return s;
-        s = ok(launch(norm_kernel<false>, dim3(grid_for(tok_work, kThreads)), dim3(kThreads), 0, st, a));
-        if (s != DAVET_OK) return s;
-        s = ok(launch(sim_kernel<false>, sg, dim3(kThreads), 0, st, a));
+        a.bblk = (a.nB + SimSmall::TM - 1) / SimSmall::TM;
+        s = ok(launch(sim_kernel<SimSmall>, dim3((a.nA + SimSmall::TM - 1) / SimSmall::TM, a.bblk, n_tiles),
+                      dim3(SimSmall::NT), SimSmall::SMEM, st, a));
       }
       if (s != DAVET_OK) return s;
       s = ok(launch(select_kernel, dim3(n_tiles), dim3(kSelThreads), select_smem(P.n0, a.nA, a.n, a.r), st, a));
