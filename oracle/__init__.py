@@ -26,6 +26,11 @@ Parity status of each function (what pins it is listed in the tests under
   prune     pinned (stable library sort, nesting, identity at full
             retention, NaN and tie rules); the score is an input (the paper
             does not define it)
+  layer     pinned (rms_norm and silu against torch's library functions,
+            rotary identities: position 0, pair norms, relative position,
+            the first pair's angle; a zero layer is the identity, equal
+            queries and keys give each request's mean value, a single-row
+            request attends to itself); numpy fp64 in ``oracle/layer.py``
   merge     pinned (constant tiles, single-cell top level = tile mean,
             partition and nesting invariants, row = member mean in fp64,
             per-round greedy choices against an independent fp64 cosine,
