@@ -21,6 +21,9 @@
  *                         churn that drive the trajectory risk (Eq. 7)
  *   davet_policy_*        the allocation policy that picks each step's view
  *                         (Sec. 4.2, Eq. 6-8; Sec. 4.3, Eq. 9)
+ *   davet_linear, davet_rmsnorm, davet_rope_table, davet_embed_answers
+ *                         the dense part of a full backbone layer step
+ *                         (tcgen05 GEMM with fused epilogues)
  *
  * Conventions shared by every entry point:
  *  - Pointers named *_dev, and every tensor argument, are DEVICE pointers on
@@ -451,6 +454,60 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
                                        int64_t total_rows, int k, uint8_t* masked_dev, int32_t* tokens_dev,
                                        int32_t* argmax_dev, float* conf_dev, int32_t* committed_dev,
                                        float* stats_dev, void* stream);
+
+/*
+ * Full-layer step (the dense part of one denoising step of the backbone;
+ * Sec. 3.1: each step runs the bidirectional transformer over [v_t || q ||
+ * y]).  The paper does not print the backbone; the layer here is a
+ * pre-normalization decoder layer without a causal mask: RMS normalization,
+ * QKV projection with rotary position embedding, davet_step_attention,
+ * output projection added to the residual stream, RMS normalization, a
+ * gated (SiLU) MLP added to the residual stream; a final normalization of
+ * the answer rows and the LM head give the logits davet_unmask_topk reads.
+ *
+ * davet_linear -- out = epilogue(A . W^T) on the tensor cores (tcgen05,
+ * bf16 operands, fp32 accumulation, bf16 output).
+ *   A        bf16 [M][K], row-major; W bf16 [N][K], row-major (a linear
+ *            layer's weight); K % 64 == 0, N % 256 == 0; 16-byte aligned
+ *   out      bf16 [M][N] (epilogue 2: [M][N/2]); must not overlap A or W
+ *   epilogue 0 store; 1 out = residual + A.W^T (residual bf16 [M][N], may be
+ *            out itself); 2 gated MLP: W holds gate and up rows in alternating
+ *            blocks of 128 (rows [256j, 256j+128) gate block j, the next 128
+ *            the up block j), out[:, 128j + c] = silu(gate) * up;
+ *            3 rotary embedding of columns [0, rope_cols) (query and key
+ *            heads of head_dim columns; pairs (d, d + head_dim/2) rotated by
+ *            the angle of the row's position in its request, row - cu[b] for
+ *            cu_seqlens[b] <= row < cu_seqlens[b+1]), the rest stored as is
+ *   cu_seqlens, batch, rope_cols, head_dim (64 or 128), rope_table
+ *            (davet_rope_table, [max_pos][head_dim/2] float2), max_pos:
+ *            epilogue 3 only (nullable otherwise); a position >= max_pos is
+ *            clamped and flags DAVET_DEV_ARG
+ * One persistent kernel on `stream`.
+ *
+ * davet_rope_table -- table[p][d] = (cos, sin)(p * theta^(-2d/head_dim)),
+ * fp32, for p < max_pos and d < head_dim/2 (computed in fp64 on the device).
+ *
+ * davet_rmsnorm -- out = x / sqrt(mean(x^2) + eps) * gamma per row (fp32
+ * sums, bf16 out); x, out bf16 [M][C], gamma bf16 [C], C % 8 == 0.  With
+ * cu_resp (int32 [batch+1], the answer-row boundaries) the M = total answer
+ * rows are the last cu_resp[b+1] - cu_resp[b] rows of each request's rows
+ * (cu_seqlens) and are written packed, in request order.
+ *
+ * davet_embed_answers -- writes the answer rows of the packed step input from
+ * an embedding table: row cu_seqlens[b+1] - n_b + i (n_b answer rows of
+ * request b) becomes table[tokens[cu_resp[b] + i]], or table[mask_id] while
+ * the token is still masked (< 0); a token >= V uses mask_id and flags
+ * DAVET_DEV_ARG.  table bf16 [V][C]; x bf16 [rows][C].
+ */
+davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
+                          const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols, int head_dim,
+                          const void* rope_table, int max_pos, void* stream);
+davet_status davet_rope_table(int max_pos, int head_dim, double theta, void* table, void* stream);
+davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
+                           const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, void* stream);
+davet_status davet_embed_answers(const void* table, int V, int C, const int32_t* tokens, int mask_id,
+                                 const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, int64_t total_resp,
+                                 void* x, void* stream);
 
 #ifdef __cplusplus
 }

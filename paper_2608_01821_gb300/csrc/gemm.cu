@@ -1,0 +1,543 @@
+// gemm.cu -- the dense projections of a full transformer layer (QKV, output,
+// gated MLP, LM head) as one tcgen05 GEMM with fused epilogues:
+//   out[M, N'] = epilogue(A[M, K] . W[N, K]^T)
+// A and W are row-major bf16 with K contiguous (W as a linear layer's weight).
+//
+// Persistent, warp-specialized, one CTA per SM, 192 threads:
+//   warp 0     TMA producer: 128 x 64 tiles of A and 256 x 64 tiles of W
+//              (128-byte swizzle) into a 4-stage ring;
+//   warp 1     owns TMEM (512 columns: two 128 x 256 fp32 accumulators) and
+//              issues the MMAs (one thread, M = 128, N = 256, K = 16 each);
+//   warps 2-5  epilogue: thread r of the four warps owns accumulator row r,
+//              reads it from TMEM 32 columns at a time and writes bf16 rows;
+//              it runs on one accumulator while the MMAs fill the other.
+// Output tiles are visited m-fastest, so the CTAs working at the same time
+// share one 256-row block of W through L2.
+// Epilogues: plain store; residual add (out = residual + product, in place
+// allowed); gated MLP (W holds gate and up rows interleaved in blocks of
+// 128: columns [0,128) of each tile are the gate, [128,256) the up
+// projection; out = silu(gate) * up, half as many columns); rotary position
+// embedding on the query and key columns (pairs (d, d + D/2) of each head,
+// angle from a cos/sin table indexed by the row's position in its request).
+#include <algorithm>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace davet {
+namespace gemm {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int kThreads = 192;
+constexpr int kWarpTma = 0, kWarpMma = 1;  // warps 2-5: epilogue
+constexpr int kTmemCols = 512;
+constexpr uint32_t kStageA = BM * BK * 2;  // 16 KB
+constexpr uint32_t kStageB = BN * BK * 2;  // 32 KB
+
+enum : int { EPI_STORE = 0, EPI_RESIDUAL = 1, EPI_SWIGLU = 2, EPI_ROPE = 3 };
+
+struct Smem {
+  alignas(1024) uint8_t a[STAGES][kStageA];
+  alignas(1024) uint8_t b[STAGES][kStageB];
+  uint64_t full[STAGES], empty[STAGES];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t fin;
+  uint32_t tmem;
+  int abort;
+};
+
+struct Params {
+  long long M;
+  int N, K;
+  int tiles_m, tiles_n;
+  uint16_t* out;
+  int ldo;  // output row stride (elements)
+  const uint16_t* residual;
+  int epi;
+  // rotary embedding
+  const int32_t* cu;  // int32 [batch + 1] request row boundaries
+  int batch;
+  int rope_cols;  // columns [0, rope_cols) are query and key heads
+  int head_dim;
+  int max_pos;
+  const float2* rope;  // [max_pos][head_dim / 2] (cos, sin)
+  unsigned* err;
+};
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned* err, volatile int* abort_flag) {
+  const bool ok = mbar_wait(bar, parity, err, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
+
+__device__ __forceinline__ float silu(float g) { return g / (1.0f + __expf(-g)); }
+
+__device__ __forceinline__ void store32(uint16_t* dst, const float (&v)[32]) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    uint4 w;
+    w.x = pack_bf16x2(v[8 * u + 0], v[8 * u + 1]);
+    w.y = pack_bf16x2(v[8 * u + 2], v[8 * u + 3]);
+    w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
+    w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
+    d4[u] = w;
+  }
+}
+
+__device__ __forceinline__ void load_acc32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  tmem_ld32(taddr, r);
+  tmem_wait_ld();
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  Smem& s = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int* abort_flag = &s.abort;
+
+  if (tid == 0) {
+    s.abort = 0;
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.acc_full[i], 1);
+      mbar_init(&s.acc_empty[i], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(&s.fin, 1);
+    fence_mbar_init();
+  }
+  if (warp == kWarpMma) {
+    tmem_alloc(&s.tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kWarpTma && lane == 0) {
+    tma_prefetch_desc(&tmap_a);
+    tma_prefetch_desc(&tmap_w);
+  }
+  pdl_launch_dependents();
+  pdl_wait();  // A (and the residual) come from the previous kernel
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s.tmem;
+  const int n_tiles = p.tiles_m * p.tiles_n;
+  const int nk = p.K / BK;
+
+  if (warp == kWarpTma) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+        const int m0 = (t % p.tiles_m) * BM, n0 = (t / p.tiles_m) * BN;
+        bool ok = true;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const uint32_t st = it % STAGES;
+          if (it >= STAGES && !mbar_wait(&s.empty[st], ((it / STAGES) - 1) & 1, p.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&s.full[st], kStageA + kStageB);
+          tma_load_2d(s.a[st], &tmap_a, &s.full[st], kb * BK, m0);
+          tma_load_2d(s.b[st], &tmap_w, &s.full[st], kb * BK, n0);
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == kWarpMma) {
+    if (lane == 0) {
+      constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN, false, false);
+      uint32_t it = 0, tc = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++tc) {
+        const uint32_t ab = tc & 1, use = tc >> 1;
+        if (use > 0 && !mbar_wait(&s.acc_empty[ab], (use - 1) & 1, p.err, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + ab * BN;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const uint32_t st = it % STAGES;
+          if (!mbar_wait(&s.full[st], (it / STAGES) & 1, p.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = sw128_desc(smem_u32(s.a[st]), 16, 1024);
+          const uint64_t db = sw128_desc(smem_u32(s.b[st]), 16, 1024);
+          if (kb == 0)
+            umma_ss_imm<false>(d, da, db, kIdesc);
+          else
+            umma_ss_imm<true>(d, da, db, kIdesc);
+          umma_ss_imm<true>(d, da + 2, db + 2, kIdesc);
+          umma_ss_imm<true>(d, da + 4, db + 4, kIdesc);
+          umma_ss_imm<true>(d, da + 6, db + 6, kIdesc);
+          umma_commit(&s.empty[st]);
+        }
+        if (ok) umma_commit(&s.acc_full[ab]);
+      }
+      // every issued MMA completes before TMEM is released
+      umma_commit(&s.fin);
+      mbar_wait(&s.fin, 0, p.err, nullptr);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int r = 32 * q + lane;
+    uint32_t tc = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++tc) {
+      const uint32_t ab = tc & 1, use = tc >> 1;
+      if (!warp_wait(&s.acc_full[ab], use & 1, p.err, abort_flag)) break;
+      tc_fence_after();
+      const int m0 = (t % p.tiles_m) * BM, n0 = (t / p.tiles_m) * BN;
+      const long long row = static_cast<long long>(m0) + r;
+      const bool row_ok = row < p.M;
+      const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
+      if (p.epi == EPI_SWIGLU) {
+        uint16_t* dst = p.out + row * p.ldo + n0 / 2;
+#pragma unroll 1
+        for (int c = 0; c < BN / 2; c += 32) {
+          float g[32], u[32];
+          load_acc32(acc + c, g);
+          load_acc32(acc + BN / 2 + c, u);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) g[i] = silu(g[i]) * u[i];
+          if (row_ok) store32(dst + c, g);
+        }
+      } else if (p.epi == EPI_ROPE && n0 < p.rope_cols) {
+        // the row's position in its request
+        int pos = 0;
+        if (row_ok) {
+          int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
+          while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (p.cu[mid] <= row) lo = mid; else hi = mid;
+          }
+          pos = static_cast<int>(row - p.cu[lo]);
+          if (pos >= p.max_pos) {
+            raise_error(p.err, DEV_ERR_ARG);
+            pos = p.max_pos - 1;
+          }
+        }
+        const int half = p.head_dim / 2;
+        const float2* tab = p.rope + static_cast<long long>(pos) * half;
+        uint16_t* dst = p.out + row * p.ldo + n0;
+#pragma unroll 1
+        for (int hb = 0; hb < BN; hb += p.head_dim) {
+#pragma unroll 1
+          for (int c = 0; c < half; c += 32) {
+            float x[32], y[32];
+            load_acc32(acc + hb + c, x);
+            load_acc32(acc + hb + half + c, y);
+            if (row_ok) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const float2 cs = tab[c + i];
+                const float a = x[i], b = y[i];
+                x[i] = a * cs.x - b * cs.y;
+                y[i] = b * cs.x + a * cs.y;
+              }
+              store32(dst + hb + c, x);
+              store32(dst + hb + half + c, y);
+            }
+          }
+        }
+      } else {
+        uint16_t* dst = p.out + row * p.ldo + n0;
+        const uint16_t* res = p.epi == EPI_RESIDUAL ? p.residual + row * p.ldo + n0 : nullptr;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          load_acc32(acc + c, v);
+          if (row_ok) {
+            if (res) {
+              const uint4* r4 = reinterpret_cast<const uint4*>(res + c);
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const uint4 w = r4[u];
+                v[8 * u + 0] += bf16lo(w.x); v[8 * u + 1] += bf16hi(w.x);
+                v[8 * u + 2] += bf16lo(w.y); v[8 * u + 3] += bf16hi(w.y);
+                v[8 * u + 4] += bf16lo(w.z); v[8 * u + 5] += bf16hi(w.z);
+                v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
+              }
+            }
+            store32(dst + c, v);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.acc_empty[ab]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpMma) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// cos/sin table of the rotary embedding: tab[p][d] = (cos, sin)(p * theta^(-2d/D)).
+__global__ void rope_table_kernel(float2* tab, int max_pos, int half, double theta) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const long long total = static_cast<long long>(max_pos) * half;
+  for (long long q = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; q < total;
+       q += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int pos = static_cast<int>(q / half), d = static_cast<int>(q % half);
+    const double ang = pos * pow(theta, -static_cast<double>(d) / half);
+    tab[q] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
+  }
+}
+
+// Root-mean-square normalization of rows: one warp per row, fp32 sums.
+// ANSWERS: only the last resp_len[b] rows of each request (rows below
+// cu[b+1]), written packed in request order.
+template <bool ANSWERS>
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const uint16_t* __restrict__ x, long long M, int C,
+                                                      const uint16_t* __restrict__ gamma, float eps,
+                                                      uint16_t* __restrict__ out, const int32_t* cu,
+                                                      const int32_t* cu_resp, int batch) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  const int C8 = C / 8;
+  for (long long o = w0; o < M; o += nw) {
+    long long src = o;
+    if constexpr (ANSWERS) {
+      int lo = 0, hi = batch;  // request of answer row o: largest b with cu_resp[b] <= o
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (cu_resp[mid] <= o) lo = mid; else hi = mid;
+      }
+      const long long nresp = cu_resp[lo + 1] - cu_resp[lo];
+      src = cu[lo + 1] - nresp + (o - cu_resp[lo]);
+    }
+    const uint4* xr = reinterpret_cast<const uint4*>(x + src * C);
+    float ss = 0.f;
+    for (int c = lane; c < C8; c += 32) {
+      const uint4 v = xr[c];
+      const float f[8] = {bf16lo(v.x), bf16hi(v.x), bf16lo(v.y), bf16hi(v.y),
+                          bf16lo(v.z), bf16hi(v.z), bf16lo(v.w), bf16hi(v.w)};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    const float inv = rsqrtf(ss / static_cast<float>(C) + eps);
+    const uint4* gr = reinterpret_cast<const uint4*>(gamma);
+    uint4* orow = reinterpret_cast<uint4*>(out + o * C);
+    for (int c = lane; c < C8; c += 32) {
+      const uint4 v = xr[c], g = gr[c];
+      uint4 w;
+      w.x = pack_bf16x2(bf16lo(v.x) * inv * bf16lo(g.x), bf16hi(v.x) * inv * bf16hi(g.x));
+      w.y = pack_bf16x2(bf16lo(v.y) * inv * bf16lo(g.y), bf16hi(v.y) * inv * bf16hi(g.y));
+      w.z = pack_bf16x2(bf16lo(v.z) * inv * bf16lo(g.z), bf16hi(v.z) * inv * bf16hi(g.z));
+      w.w = pack_bf16x2(bf16lo(v.w) * inv * bf16lo(g.w), bf16hi(v.w) * inv * bf16hi(g.w));
+      orow[c] = w;
+    }
+  }
+}
+
+// Answer rows of the step input from the embedding table: row
+// cu[b+1] - resp[b] + i of request b is table[tokens[cu_resp[b] + i]], or
+// table[mask_id] while that position is still masked (token < 0).
+__global__ void __launch_bounds__(256) embed_answers_kernel(const uint16_t* __restrict__ table, int V, int C,
+                                                            const int32_t* __restrict__ tokens, int mask_id,
+                                                            const int32_t* cu, const int32_t* cu_resp, int batch,
+                                                            long long R, uint16_t* __restrict__ x,
+                                                            unsigned* err) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  const int C8 = C / 8;
+  for (long long o = w0; o < R; o += nw) {
+    int lo = 0, hi = batch;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (cu_resp[mid] <= o) lo = mid; else hi = mid;
+    }
+    const long long nresp = cu_resp[lo + 1] - cu_resp[lo];
+    const long long dst = cu[lo + 1] - nresp + (o - cu_resp[lo]);
+    int tok = tokens[o];
+    if (tok < 0) tok = mask_id;
+    if (tok >= V) {
+      if (lane == 0) raise_error(err, DEV_ERR_ARG);
+      tok = mask_id;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(table + static_cast<long long>(tok) * C);
+    uint4* d = reinterpret_cast<uint4*>(x + dst * C);
+    for (int c = lane; c < C8; c += 32) d[c] = src[c];
+  }
+}
+
+}  // namespace gemm
+}  // namespace davet
+
+using namespace davet;
+using namespace davet::gemm;
+
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2-D map over a row-major bf16 [rows][K] matrix, boxes of 64 x box_rows.
+bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(std::max<long long>(rows, 1))};
+  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(K) * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estride[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box, estride,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int g_sms[64] = {0};
+bool g_attr[64] = {false};
+std::mutex g_mu;
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
+                                     const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols,
+                                     int head_dim, const void* rope_table, int max_pos, void* stream) {
+  if (M < 0 || M > 0x7fffffffLL || K < BK || K % BK != 0 || N < BN || N % BN != 0) return DAVET_ERR_INVALID_ARG;
+  if (epilogue < EPI_STORE || epilogue > EPI_ROPE) return DAVET_ERR_INVALID_ARG;
+  if (M == 0) return DAVET_OK;
+  if (!A || !W || !out || !aligned16(A) || !aligned16(W) || !aligned16(out)) return DAVET_ERR_INVALID_ARG;
+  if (epilogue == EPI_RESIDUAL && (!residual || !aligned16(residual))) return DAVET_ERR_INVALID_ARG;
+  if (epilogue == EPI_ROPE) {
+    if (!cu_seqlens || batch < 1 || !rope_table || max_pos < 1 || (head_dim != 64 && head_dim != 128) ||
+        rope_cols < 0 || rope_cols % BN != 0 || rope_cols > N)
+      return DAVET_ERR_INVALID_ARG;
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= 64) return DAVET_ERR_UNSUPPORTED;
+  const size_t smem = sizeof(Smem) + 1024;
+  {
+    std::lock_guard<std::mutex> g(g_mu);
+    if (g_sms[dev] == 0) {
+      e = cudaDeviceGetAttribute(&g_sms[dev], cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return cuda_fail(e);
+    }
+    if (!g_attr[dev]) {
+      e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      if (e != cudaSuccess) return cuda_fail(e);
+      g_attr[dev] = true;
+    }
+  }
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  CUtensorMap ma, mw;
+  if (!make_map(&ma, A, M, K, BM) || !make_map(&mw, W, N, K, BN)) return DAVET_ERR_INVALID_ARG;
+  Params p;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.tiles_m = static_cast<int>((M + BM - 1) / BM);
+  p.tiles_n = N / BN;
+  p.out = static_cast<uint16_t*>(out);
+  p.ldo = epilogue == EPI_SWIGLU ? N / 2 : N;
+  p.residual = static_cast<const uint16_t*>(residual);
+  p.epi = epilogue;
+  p.cu = cu_seqlens;
+  p.batch = batch;
+  p.rope_cols = epilogue == EPI_ROPE ? rope_cols : 0;
+  p.head_dim = head_dim;
+  p.max_pos = max_pos;
+  p.rope = static_cast<const float2*>(rope_table);
+  p.err = err;
+  const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
+  if (tiles > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
+  const int grid = static_cast<int>(std::min<long long>(tiles, g_sms[dev]));
+  e = launch(gemm_kernel, dim3(grid), dim3(kThreads), smem, static_cast<cudaStream_t>(stream), ma, mw, p);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
+extern "C" davet_status davet_rope_table(int max_pos, int head_dim, double theta, void* table, void* stream) {
+  if (max_pos < 1 || (head_dim != 64 && head_dim != 128) || !(theta > 1.0) || !table) return DAVET_ERR_INVALID_ARG;
+  const long long total = static_cast<long long>(max_pos) * (head_dim / 2);
+  const int blocks = static_cast<int>(std::min<long long>((total + 255) / 256, 152LL * 8));
+  const cudaError_t e = launch(rope_table_kernel, dim3(blocks), dim3(256), 0, static_cast<cudaStream_t>(stream),
+                               static_cast<float2*>(table), max_pos, head_dim / 2, theta);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
+extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
+                                      const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, void* stream) {
+  if (M < 0 || C < 8 || C % 8 != 0 || !(eps >= 0.0f)) return DAVET_ERR_INVALID_ARG;
+  if (M == 0) return DAVET_OK;
+  if (!x || !gamma || !out || !aligned16(x) || !aligned16(gamma) || !aligned16(out)) return DAVET_ERR_INVALID_ARG;
+  const bool answers = cu_resp != nullptr;
+  if (answers && (!cu_seqlens || batch < 1)) return DAVET_ERR_INVALID_ARG;
+  const int blocks = static_cast<int>(std::min<long long>((M + 7) / 8, 152LL * 16));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const uint16_t* xs = static_cast<const uint16_t*>(x);
+  const uint16_t* gs = static_cast<const uint16_t*>(gamma);
+  uint16_t* os = static_cast<uint16_t*>(out);
+  const cudaError_t e =
+      answers ? launch(rmsnorm_kernel<true>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs, eps,
+                       os, cu_seqlens, cu_resp, batch)
+              : launch(rmsnorm_kernel<false>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs,
+                       eps, os, cu_seqlens, cu_resp, batch);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
+extern "C" davet_status davet_embed_answers(const void* table, int V, int C, const int32_t* tokens, int mask_id,
+                                            const int32_t* cu_seqlens, const int32_t* cu_resp, int batch,
+                                            int64_t total_resp, void* x, void* stream) {
+  if (V < 1 || C < 8 || C % 8 != 0 || mask_id < 0 || mask_id >= V || batch < 1 || total_resp < 0)
+    return DAVET_ERR_INVALID_ARG;
+  if (total_resp == 0) return DAVET_OK;
+  if (!table || !tokens || !cu_seqlens || !cu_resp || !x || !aligned16(table) || !aligned16(x))
+    return DAVET_ERR_INVALID_ARG;
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  const int blocks = static_cast<int>(std::min<long long>((total_resp + 7) / 8, 152LL * 16));
+  const cudaError_t e = launch(embed_answers_kernel, dim3(blocks), dim3(256), 0, static_cast<cudaStream_t>(stream),
+                               static_cast<const uint16_t*>(table), V, C, tokens, mask_id, cu_seqlens, cu_resp, batch,
+                               static_cast<long long>(total_resp), static_cast<uint16_t*>(x), err);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}

@@ -84,6 +84,10 @@ def _declare(lib):
         "davet_policy_envelope": (_int, [_int, _int, ctypes.c_double, ctypes.c_double, _vp, _int, _vp, _vp, _vp]),
         "davet_policy_step": (_int, [_int, _int, _vp, _vp, _vp, _int, ctypes.c_double, ctypes.POINTER(_i32), _vp,
                                      _vp, _vp]),
+        "davet_linear": (_int, [_vp, _i64, _int, _vp, _int, _vp, _int, _vp, _vp, _int, _int, _int, _vp, _int, _vp]),
+        "davet_rope_table": (_int, [_int, _int, ctypes.c_double, _vp, _vp]),
+        "davet_rmsnorm": (_int, [_vp, _i64, _int, _vp, _f32, _vp, _vp, _vp, _int, _vp]),
+        "davet_embed_answers": (_int, [_vp, _int, _int, _vp, _int, _vp, _vp, _int, _i64, _vp, _vp]),
         "davet_unmask_topk_noalloc": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp,
                                              _vp]),
     }
@@ -216,6 +220,32 @@ class Davet:
                                                _ptr(tokens), _ptr(argmax), _ptr(conf), _ptr(committed),
                                                _ptr(stats), _ptr(workspace), workspace_bytes, _stream(stream)))
 
+
+    EPI_STORE, EPI_RESIDUAL, EPI_SWIGLU, EPI_ROPE = 0, 1, 2, 3
+
+    def davet_linear(self, A, M: int, K: int, W, N: int, out, epilogue: int = 0, residual=None, cu_seqlens=None,
+                     batch: int = 0, rope_cols: int = 0, head_dim: int = 128, rope_table=None, max_pos: int = 0,
+                     stream=None):
+        self._check("davet_linear",
+                    self.lib.davet_linear(_ptr(A), M, K, _ptr(W), N, _ptr(out), epilogue, _ptr(residual),
+                                          _ptr(cu_seqlens), batch, rope_cols, head_dim, _ptr(rope_table), max_pos,
+                                          _stream(stream)))
+
+    def davet_rope_table(self, max_pos: int, head_dim: int, theta: float, table, stream=None):
+        self._check("davet_rope_table",
+                    self.lib.davet_rope_table(max_pos, head_dim, float(theta), _ptr(table), _stream(stream)))
+
+    def davet_rmsnorm(self, x, M: int, C: int, gamma, eps: float, out, cu_seqlens=None, cu_resp=None, batch: int = 0,
+                      stream=None):
+        self._check("davet_rmsnorm",
+                    self.lib.davet_rmsnorm(_ptr(x), M, C, _ptr(gamma), float(eps), _ptr(out), _ptr(cu_seqlens),
+                                           _ptr(cu_resp), batch, _stream(stream)))
+
+    def davet_embed_answers(self, table, V: int, C: int, tokens, mask_id: int, cu_seqlens, cu_resp, batch: int,
+                            total_resp: int, x, stream=None):
+        self._check("davet_embed_answers",
+                    self.lib.davet_embed_answers(_ptr(table), V, C, _ptr(tokens), mask_id, _ptr(cu_seqlens),
+                                                 _ptr(cu_resp), batch, total_resp, _ptr(x), _stream(stream)))
 
     def davet_policy_envelope(self, T: int, orientation: int, B: float, rho: float, demand, batch: int, lower,
                               upper, stream=None):

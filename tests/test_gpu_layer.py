@@ -1,0 +1,219 @@
+"""Parity of the full-layer kernels with the fp64 oracle (oracle/layer.py):
+the tcgen05 GEMM and its epilogues, RMS normalization, the embedding of the
+answer rows, and one whole layer.
+
+Tolerances: each kernel computes in fp32 and rounds its output to bf16
+once, so an output must lie within one bf16 rounding (2^-8 relative, two
+half-ulps) of the oracle's fp64 value on the same bf16 inputs, plus the fp32
+accumulation error, bounded by 1e-3 of the output's RMS; a whole layer (eight
+bf16 roundings between stages) must agree to 2% relative L2."""
+import numpy as np
+import pytest
+import torch
+
+from helpers import bits
+from oracle import layer as L
+
+pytestmark = pytest.mark.gpu
+
+THETA = 500000.0
+
+
+def rand_bf16(shape, seed, scale=1.0):
+    g = torch.Generator().manual_seed(seed)
+    return (torch.randn(shape, generator=g) * scale).to(torch.bfloat16)
+
+
+def f64(t):
+    return t.detach().cpu().double().numpy()
+
+
+def check_close(got, ref, what=""):
+    got = f64(got)
+    rms = np.sqrt((ref ** 2).mean()) + 1e-30
+    err = np.abs(got - ref)
+    lim = np.abs(ref) * 2.0 ** -8 + 1e-3 * rms
+    bad = err > lim
+    assert not bad.any(), f"{what}: {int(bad.sum())} of {bad.size} outside, worst {float((err - lim).max()):.3g}"
+
+
+def linear(davet, A, W, epi=0, residual=None, out_cols=None, **kw):
+    M, K = A.shape
+    N = W.shape[0]
+    out = torch.full((M + 3, out_cols or N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    if residual is not None and residual is not out:
+        out[:M].copy_(residual)
+        residual = out
+    davet.davet_linear(A, M, K, W, N, out, epi, residual, **kw)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    assert torch.isnan(out[M:].float()).all()
+    return out[:M]
+
+
+@pytest.mark.parametrize("M,K,N", [(1, 64, 256), (100, 256, 512), (128, 128, 256), (300, 512, 1024),
+                                   (1000, 4096, 768), (257, 1024, 2560)])
+def test_linear_store(davet, M, K, N):
+    A = rand_bf16((M, K), M + K).cuda()
+    W = rand_bf16((N, K), N + 7, K ** -0.5).cuda()
+    out = linear(davet, A, W)
+    check_close(out, f64(A) @ f64(W).T, f"{M}x{K}x{N}")
+
+
+def test_linear_residual_in_place(davet):
+    M, K, N = 333, 512, 768
+    A = rand_bf16((M, K), 1).cuda()
+    W = rand_bf16((N, K), 2, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 3).cuda()
+    ref = f64(R) + f64(A) @ f64(W).T
+    x = R.clone()
+    davet.davet_linear(A, M, K, W, N, x, davet.EPI_RESIDUAL, x)
+    torch.cuda.synchronize()
+    check_close(x, ref, "residual")
+
+
+def test_linear_gated_mlp(davet):
+    M, K, F = 200, 256, 768
+    A = rand_bf16((M, K), 4).cuda()
+    Wg = rand_bf16((F, K), 5, K ** -0.5)
+    Wu = rand_bf16((F, K), 6, K ** -0.5)
+    # interleave in blocks of 128 rows: gate block j, then up block j
+    Wgu = torch.stack([Wg.reshape(F // 128, 128, K), Wu.reshape(F // 128, 128, K)], 1).reshape(2 * F, K).cuda()
+    out = linear(davet, A, Wgu, davet.EPI_SWIGLU, out_cols=F)
+    a = f64(A)
+    check_close(out, L.silu(a @ f64(Wg).T) * (a @ f64(Wu).T), "swiglu")
+
+
+@pytest.mark.parametrize("D,H", [(128, 4), (64, 4)])
+def test_linear_rotary_qkv(davet, D, H):
+    HD = H * D
+    K = 256
+    cu = [0, 70, 71, 300, 300, 517]
+    M = cu[-1]
+    A = rand_bf16((M, K), 8).cuda()
+    W = rand_bf16((3 * HD, K), 9, K ** -0.5).cuda()
+    max_pos = 512
+    tab = torch.empty((max_pos, D // 2, 2), dtype=torch.float32, device="cuda")
+    davet.davet_rope_table(max_pos, D, THETA, tab)
+    cu_d = torch.tensor(cu, dtype=torch.int32, device="cuda")
+    out = linear(davet, A, W, davet.EPI_ROPE, cu_seqlens=cu_d, batch=len(cu) - 1, rope_cols=2 * HD, head_dim=D,
+                 rope_table=tab, max_pos=max_pos)
+    y = f64(A) @ f64(W).T
+    pos = L.positions(cu)
+    ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
+                          y[:, 2 * HD:]], axis=1)
+    check_close(out, ref, "rope")
+    # the table itself: fp32 rounding of the fp64 angles' cos and sin
+    ang = L.rope_angles(np.arange(max_pos), D, THETA)
+    t = tab.cpu().double().numpy()
+    assert np.abs(t[..., 0] - np.cos(ang)).max() < 1e-6 and np.abs(t[..., 1] - np.sin(ang)).max() < 1e-6
+
+
+def test_rope_position_past_the_table_is_flagged(davet):
+    D, H, K = 64, 4, 64
+    cu = torch.tensor([0, 40], dtype=torch.int32, device="cuda")
+    tab = torch.empty((16, D // 2, 2), dtype=torch.float32, device="cuda")
+    davet.davet_rope_table(16, D, THETA, tab)
+    A = rand_bf16((40, K), 10).cuda()
+    W = rand_bf16((3 * H * D, K), 11, K ** -0.5).cuda()
+    out = torch.empty((40, 3 * H * D), dtype=torch.bfloat16, device="cuda")
+    davet.davet_device_status(clear=True)
+    davet.davet_linear(A, 40, K, W, 3 * H * D, out, davet.EPI_ROPE, None, cu, 1, 2 * H * D, D, tab, 16)
+    torch.cuda.synchronize()
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags & 0x4
+
+
+def test_rmsnorm_rows_and_answer_rows(davet):
+    C = 4096
+    cu = [0, 50, 51, 200]
+    resp = [7, 1, 30]
+    cu_resp = np.concatenate([[0], np.cumsum(resp)]).astype(np.int32)
+    x = rand_bf16((cu[-1], C), 12, 3.0).cuda()
+    g = (1 + 0.1 * rand_bf16((C,), 13).float()).to(torch.bfloat16).cuda()
+    out = torch.empty_like(x)
+    davet.davet_rmsnorm(x, cu[-1], C, g, 1e-5, out)
+    torch.cuda.synchronize()
+    check_close(out, L.rmsnorm(f64(x), f64(g), 1e-5), "rmsnorm")
+    R = int(cu_resp[-1])
+    outa = torch.full((R + 2, C), float("nan"), dtype=torch.bfloat16, device="cuda")
+    davet.davet_rmsnorm(x, R, C, g, 1e-5, outa, torch.tensor(cu, dtype=torch.int32, device="cuda"),
+                        torch.from_numpy(cu_resp).cuda(), 3)
+    torch.cuda.synchronize()
+    rows = np.concatenate([np.arange(cu[b + 1] - resp[b], cu[b + 1]) for b in range(3)])
+    check_close(outa[:R], L.rmsnorm(f64(x)[rows], f64(g), 1e-5), "rmsnorm answers")
+    assert torch.isnan(outa[R:].float()).all()
+
+
+def test_embed_answers_bit_exact(davet):
+    V, C = 300, 256
+    table = rand_bf16((V, C), 14).cuda()
+    cu = torch.tensor([0, 10, 30, 31], dtype=torch.int32, device="cuda")
+    resp = [4, 0, 1]
+    cu_resp = torch.tensor([0, 4, 4, 5], dtype=torch.int32, device="cuda")
+    tokens = torch.tensor([-1, 17, 299, -1, 5], dtype=torch.int32, device="cuda")
+    x = rand_bf16((31, C), 15).cuda()
+    before = bits(x).copy()
+    davet.davet_embed_answers(table, V, C, tokens, 3, cu, cu_resp, 3, 5, x)
+    torch.cuda.synchronize()
+    got, tb = bits(x), bits(table)
+    want = before.copy()
+    for row, tok in zip([6, 7, 8, 9, 30], [3, 17, 299, 3, 5]):
+        want[row] = tb[tok]
+    assert np.array_equal(got, want)
+
+
+def test_one_layer_against_the_oracle(davet):
+    """A whole layer (tiny shapes: C = 256, 4 heads of 64, F = 768) on three
+    packed requests, kernel by kernel as the backbone step runs it."""
+    C, H, D, F = 256, 4, 64, 768
+    HD = H * D
+    cu = [0, 100, 101, 260]
+    N = cu[-1]
+    rng = np.random.default_rng(20)
+
+    def w(shape, fan_in):
+        return torch.from_numpy(rng.standard_normal(shape) / np.sqrt(fan_in)).to(torch.bfloat16)
+
+    g1 = torch.from_numpy(1 + 0.1 * rng.standard_normal(C)).to(torch.bfloat16)
+    g2 = torch.from_numpy(1 + 0.1 * rng.standard_normal(C)).to(torch.bfloat16)
+    wq, wk, wv, wo = w((HD, C), C), w((HD, C), C), w((HD, C), C), w((C, HD), HD)
+    wg, wu, wd = w((F, C), C), w((F, C), C), w((C, F), F)
+    x0 = torch.from_numpy(rng.standard_normal((N, C))).to(torch.bfloat16)
+    ref = L.layer(f64(x0), dict(g1=f64(g1), wq=f64(wq), wk=f64(wk), wv=f64(wv), wo=f64(wo), g2=f64(g2),
+                                wg=f64(wg), wu=f64(wu), wd=f64(wd)), cu, H, D, THETA, 1e-5)
+    dev = "cuda"
+    x = x0.to(dev)
+    wqkv = torch.cat([wq, wk, wv]).to(dev)
+    wgu = torch.stack([wg.reshape(F // 128, 128, C), wu.reshape(F // 128, 128, C)], 1).reshape(2 * F, C).to(dev)
+    cu_d = torch.tensor(cu, dtype=torch.int32, device=dev)
+    tab = torch.empty((512, D // 2, 2), dtype=torch.float32, device=dev)
+    davet.davet_rope_table(512, D, THETA, tab)
+    h = torch.empty((N, C), dtype=torch.bfloat16, device=dev)
+    qkv = torch.empty((N, 3 * HD), dtype=torch.bfloat16, device=dev)
+    att = torch.empty((N, HD), dtype=torch.bfloat16, device=dev)
+    a = torch.empty((N, F), dtype=torch.bfloat16, device=dev)
+    davet.davet_rmsnorm(x, N, C, g1.to(dev), 1e-5, h)
+    davet.davet_linear(h, N, C, wqkv, 3 * HD, qkv, davet.EPI_ROPE, None, cu_d, 3, 2 * HD, D, tab, 512)
+    davet.davet_step_attention(qkv, cu_d, 3, N, H, D, D ** -0.5, att)
+    davet.davet_linear(att, N, HD, wo.to(dev), C, x, davet.EPI_RESIDUAL, x)
+    davet.davet_rmsnorm(x, N, C, g2.to(dev), 1e-5, h)
+    davet.davet_linear(h, N, C, wgu, 2 * F, a, davet.EPI_SWIGLU)
+    davet.davet_linear(a, N, F, wd.to(dev), C, x, davet.EPI_RESIDUAL, x)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    got = f64(x)
+    rel = np.linalg.norm(got - ref) / np.linalg.norm(ref)
+    assert rel < 2e-2, rel
+
+
+def test_large_projection_sampled_rows(davet):
+    """The 8B-class QKV shape (921 rows, 4096 -> 12288) on sampled rows."""
+    M, K, N = 921, 4096, 12288
+    A = rand_bf16((M, K), 21).cuda()
+    W = rand_bf16((N, K), 22, K ** -0.5).cuda()
+    out = linear(davet, A, W)
+    rows = np.random.default_rng(5).choice(M, 48, replace=False)
+    rows = np.concatenate([rows, [0, 127, 128, M - 1]])
+    ref = f64(A)[rows] @ f64(W).T
+    check_close(out[torch.from_numpy(rows).cuda()], ref, "qkv 8B rows")
