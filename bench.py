@@ -287,6 +287,165 @@ def run_ours(args, rank, world, local_rank):
     return out
 
 
+def run_backbone(args, rank, world, local_rank):
+    """The full backbone step (`--model full`): every denoising step runs
+    `--layers` synthetic-weight layers over the step sequence, the LM head
+    over the answer rows and the unmasking, in one CUDA graph per pass."""
+    import torch
+
+    from paper_2608_01821_gb300 import davet, workloads
+    from paper_2608_01821_gb300.model import Backbone
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    lib = davet.load()
+    w = workloads.make(args.config)
+    if rank > 0:
+        w.seed = w.seed + 1000 * rank
+    bb = Backbone(w, args.layers, dev, lib)
+    feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C),
+                                   workloads.derive_seed(w.seed, workloads.KIND_FEAT, b)) for b in range(w.batch)]
+    prompts = [workloads.normal_bf16((w.prompt[b], bb.C), workloads.derive_seed(w.seed, workloads.KIND_TEXT, b))
+               for b in range(w.batch)]
+    bb.load_inputs(feats, prompts)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def one_pass(timed=None):
+        bb.reset_state()
+        bb.build_pyramids()
+        for t in range(w.T):
+            bb.step(t, timed=timed)
+
+    with torch.cuda.stream(stream):
+        one_pass()
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        one_pass()
+    torch.cuda.synchronize()
+    st, flags = lib.davet_device_status()
+    if st != 0:
+        raise RuntimeError(f"device error word {flags:#x} after warm-up")
+    for _ in range(args.warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks:
+        with torch.cuda.stream(stream):
+            for i in range(args.steps):
+                flush.fill_(i & 0xFF)
+                starts[i].record(stream)
+                graph.replay()
+                ends[i].record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    pass_ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    total_s = allreduce_max(sum(pass_ms) / 1e3, world, dev)
+    st, flags = lib.davet_device_status()
+    if st != 0:
+        raise RuntimeError(f"device error word {flags:#x} after the timed region")
+
+    # per-kind device time of one pass: a graph with an event pair around every call
+    calls = []
+
+    def timed(kind, fn):
+        a, b = torch.cuda.Event(enable_timing=True, external=True), torch.cuda.Event(enable_timing=True,
+                                                                                     external=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        calls.append((kind, a, b))
+
+    g2 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g2, stream=stream):
+        one_pass(timed)
+    g2.replay()
+    torch.cuda.synchronize()
+    kinds = {}
+    for kind, a, b in calls:
+        kinds[kind] = kinds.get(kind, 0.0) + a.elapsed_time(b)
+    n_gemm = sum(1 for k, _, _ in calls if k == "gemm")
+    gemm_flops = sum(bb.gemm_flops(t) for t in range(w.T))
+
+    # end to end: visual hidden states and prompt rows from pinned host memory,
+    # committed tokens back to the host, every pass
+    e2e = None
+    if not args.no_e2e:
+        pf = [f.pin_memory() for f in feats]
+        pp = [p.pin_memory() for p in prompts]
+        tok_host = torch.empty(w.total_resp, dtype=torch.int32).pin_memory()
+        n = max(1, min(args.steps, 3))
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            s0.record(stream)
+            for _ in range(n):
+                bb.load_inputs(pf, pp, non_blocking=True)
+                graph.replay()
+                tok_host.copy_(bb.tokens, non_blocking=True)
+            s1.record(stream)
+        torch.cuda.synchronize()
+        te = allreduce_max(s0.elapsed_time(s1) / 1e3, world, dev)
+        h2d = sum(f.numel() * 2 for f in pf) + sum(p.numel() * 2 for p in pp)
+        e2e = {"value": round(w.T * n * world / te, 3), "unit": "denoising steps/s", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(w.total_resp * 4), "passes": n}
+
+    if rank != 0:
+        return None
+    peaks = measured_peaks()
+    achieved = gemm_flops / (kinds["gemm"] * 1e-3) / 1e12
+    peak = peaks.get("bf16_tflops_sustained") or peaks["bf16_tflops"]
+    n_steps = w.T
+    return {
+        "metric": METRIC,
+        "value": round(whole_job_rate(w.T * args.steps, world, total_s), 3),
+        "unit": "denoising steps/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(statistics.mean(pass_ms), 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) visual hidden states and prompt rows; random N(0,1/fan_in) weights)",
+        "config": {
+            "workload": w.name,
+            "model": "full backbone step (synthetic weights)",
+            "layers": args.layers,
+            "hidden": bb.C,
+            "heads": w.H,
+            "head_dim": w.D,
+            "mlp": bb.F,
+            "vocab": w.V,
+            "batch": w.batch,
+            "denoising_steps_per_pass": n_steps,
+            "parallelism": f"replicas x{world} (independent requests)",
+            "timing": "CUDA events per pass on the launching stream; one CUDA graph per pass",
+            "l2": f"{L2_FLUSH_BYTES >> 20} MiB write between timed passes (not timed); weights stream from HBM",
+        },
+        "components": {k: {"ms_per_pass": round(v, 3), "share": round(v / sum(kinds.values()), 4)}
+                       for k, v in kinds.items()},
+        "roofline": {
+            "kernel": "davet_linear (tcgen05 GEMM, all projections and the LM head)",
+            "bound": "tensor",
+            "achieved": round(achieved, 2),
+            "peak": peak,
+            "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 4),
+            "peak_source": f"{peaks['source']} bf16 sustained (MEASURED_PEAKS.json)",
+            "traffic": None,
+            "flops_per_launch": gemm_flops / max(n_gemm, 1),
+        },
+        "clocks": clocks.summary(),
+        "gpu_launches": (w.batch + w.T * bb.launches_per_step()) * args.steps,
+        "e2e": e2e,
+    }
+
+
 def merge_round_count(grid: int, n_levels: int) -> int:
     """Bipartite matching rounds the merging realizer runs per tile: level l
     is reached from n tokens by rounds of r = min(n - G_l^2, ceil(n/2))."""
@@ -580,6 +739,35 @@ def oracle_sample(w, budget_s=20.0):
     return w.T / total, cores, desc, spent
 
 
+def backbone_oracle_sample(w, n_layers: int):
+    """The fp64 layer oracle on one layer of one step of the workload (its
+    first step's sequence), scaled to n_layers and the whole schedule by the
+    steps' GEMM work.  Returns (denoising steps/s, cores, description, s)."""
+    import numpy as np
+
+    import oracle
+    from oracle import layer as L
+    cores = oracle.max_threads()
+    C = w.H * w.D
+    F = 3 * C
+    rng = np.random.default_rng(0)
+    lens = w.step_lengths(0)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    x = rng.standard_normal((int(cu[-1]), C))
+    wts = dict(g1=np.ones(C), wq=rng.standard_normal((C, C)) / 64, wk=rng.standard_normal((C, C)) / 64,
+               wv=rng.standard_normal((C, C)) / 64, wo=rng.standard_normal((C, C)) / 64, g2=np.ones(C),
+               wg=rng.standard_normal((F, C)) / 64, wu=rng.standard_normal((F, C)) / 64,
+               wd=rng.standard_normal((C, F)) / 110)
+    t0 = time.perf_counter()
+    L.layer(x, wts, cu, w.H, w.D, 500000.0, 1e-5)
+    dt = time.perf_counter() - t0
+    rows0 = float(cu[-1])
+    per_step = [dt * n_layers * sum(w.step_lengths(t)) / rows0 for t in range(w.T)]
+    desc = (f"fp64 layer oracle (numpy): one layer of step 0 ({int(rows0)} rows) timed, scaled by rows to "
+            f"{n_layers} layers and the {w.T}-step schedule; LM head and unmasking not included")
+    return w.T / sum(per_step), cores, desc, dt
+
+
 def run_reference(args, rank, world):
     """The oracle arm: each timed step is one denoising step of the workload
     run by the fp64 CPU oracle (levels taken in schedule order, cycling
@@ -728,6 +916,10 @@ def main(argv=None):
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)
+    ap.add_argument("--model", choices=["core", "full"], default="core",
+                    help="core: the step-conditioning path (attention core); full: every step runs --layers "
+                         "synthetic-weight backbone layers and the LM head")
+    ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--realizer", choices=["pool", "prune", "merge"], default="pool",
                     help="evidence realizer of the view blocks (Sec. 4.3): pooling (default), pruning or merging")
     args = ap.parse_args(argv)
@@ -740,6 +932,19 @@ def main(argv=None):
             print(json.dumps(out), flush=True)
         return 0
     init_dist(world, "nccl")
+    if args.model == "full":
+        out = run_backbone(args, rank, world, local)
+        if rank == 0:
+            if not args.no_cpu_baseline:
+                from paper_2608_01821_gb300 import workloads
+                v, cores, desc, spent = backbone_oracle_sample(workloads.make(args.config), args.layers)
+                out["cpu_baseline"] = {"value": round(v, 6), "unit": "denoising steps/s", "cores": cores,
+                                       "kind": "oracle", "sample": desc, "cpu_seconds": round(spent, 1)}
+            print(json.dumps(out), flush=True)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return 0
     out = run_ours(args, rank, world, local)
     if rank == 0:
         if not args.no_cpu_baseline:

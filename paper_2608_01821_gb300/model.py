@@ -1,0 +1,189 @@
+"""Full backbone step with synthetic weights: host orchestration only.
+
+Every denoising step (Sec. 3.1, Eq. 1-2) runs the whole backbone over the
+step sequence [v_t || q || y^(t-1)]: the step's view rows and prompt rows
+come from the evidence pyramid and the text store (davet_gather_view), the
+answer rows are the embeddings of the current answer state (committed token
+or the mask token; davet_embed_answers); then `n_layers` pre-normalization
+layers (davet_rmsnorm, davet_linear with the rotary / residual / gated-MLP
+epilogues, davet_step_attention), the final normalization of the answer rows
+and the LM head give the logits that davet_unmask_topk commits from.  The
+rows carry hidden states of width C = H * D; the MLP width is 3C.
+
+Weights are random (no checkpoint is available): each matrix ~ N(0, 1/fan_in),
+normalization gains ~ 1 + N(0, 0.1^2), drawn on the device from torch
+generators seeded per tensor.  This module performs no arithmetic of its own.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import davet as _davet
+from .workloads import Workload, derive_seed
+
+KIND_WEIGHT = 16
+ROPE_THETA = 500000.0
+RMS_EPS = 1e-5
+
+
+class Backbone:
+    def __init__(self, w: Workload, n_layers: int, device="cuda", lib=None, mask_id: int | None = None):
+        self.w = w
+        self.L = n_layers
+        self.dev = torch.device(device)
+        self.lib = lib if lib is not None else _davet.load()
+        H, D = w.H, w.D
+        self.C = C = H * D
+        self.F = F = 3 * C
+        self.HD = H * D
+        self.V = w.V
+        self.mask_id = w.V - 1 if mask_id is None else mask_id
+        if C % 256 or F % 128 or w.V % 256:
+            raise ValueError("hidden width and vocabulary must be multiples of 256, the MLP width of 128")
+        dev = self.dev
+        seed = w.seed
+
+        def rnd(shape, k, std):
+            g = torch.Generator(device=dev)
+            g.manual_seed(derive_seed(seed, KIND_WEIGHT + k, 0))
+            return (torch.randn(shape, generator=g, device=dev, dtype=torch.float32) * std).to(torch.bfloat16)
+
+        def gain(k):
+            return (1.0 + rnd((C,), k, 0.1).float()).to(torch.bfloat16)
+
+        self.layers = []
+        for l in range(n_layers):
+            base = 16 * (l + 1)
+            wg = rnd((F, C), base + 4, C ** -0.5)
+            wu = rnd((F, C), base + 5, C ** -0.5)
+            self.layers.append(dict(
+                g1=gain(base + 0),
+                wqkv=rnd((3 * self.HD, C), base + 1, C ** -0.5),
+                wo=rnd((C, self.HD), base + 2, self.HD ** -0.5),
+                g2=gain(base + 3),
+                # gate and up rows interleaved in blocks of 128 (the gated-MLP epilogue's layout)
+                wgu=torch.stack([wg.reshape(F // 128, 128, C), wu.reshape(F // 128, 128, C)], 1)
+                .reshape(2 * F, C).contiguous(),
+                wd=rnd((C, F), base + 6, F ** -0.5),
+            ))
+            del wg, wu
+        self.gf = gain(1)
+        self.wlm = rnd((w.V, C), 2, C ** -0.5)
+        self.emb = rnd((w.V, C), 3, 1.0)
+
+        # the evidence pyramids of the hidden rows (level-major, one buffer per request) and the prompt rows
+        self.pyr = [torch.empty((max(w.tiles[b] * sum(g * g for g in w.level_sides()), 1), C), dtype=torch.bfloat16,
+                                device=dev) for b in range(w.batch)]
+        self.pyr_ptrs = torch.tensor([p.data_ptr() for p in self.pyr], dtype=torch.int64, device=dev)
+        self.text = torch.zeros((max(w.total_text(), 1), C), dtype=torch.bfloat16, device=dev)
+        self.tiles = torch.tensor(w.tiles, dtype=torch.int32, device=dev)
+        self.prompt = torch.tensor(w.prompt, dtype=torch.int32, device=dev)
+        self.resp = torch.tensor(w.resp, dtype=torch.int32, device=dev)
+        self.text_off = torch.from_numpy(w.text_offsets()).to(dev)
+        self.schedule = torch.from_numpy(w.schedule).to(dev).contiguous()
+        self.max_rows = w.max_total_rows()
+        R = w.total_resp
+        self.R = R
+        self.cu = torch.zeros(w.batch + 1, dtype=torch.int32, device=dev)
+        self.cu_resp = torch.from_numpy(w.cu_resp()).to(dev)
+        self.x = torch.empty((self.max_rows, C), dtype=torch.bfloat16, device=dev)
+        self.h = torch.empty((self.max_rows, C), dtype=torch.bfloat16, device=dev)
+        self.qkv = torch.empty((self.max_rows, 3 * self.HD), dtype=torch.bfloat16, device=dev)
+        self.att = torch.empty((self.max_rows, self.HD), dtype=torch.bfloat16, device=dev)
+        self.a = torch.empty((self.max_rows, F), dtype=torch.bfloat16, device=dev)
+        self.xa = torch.empty((max(R, 1), C), dtype=torch.bfloat16, device=dev)
+        self.logits = torch.empty((max(R, 1), w.V), dtype=torch.bfloat16, device=dev)
+        self.max_pos = max(max(w.seq_len(b, v) for v in range(w.n_views())) for b in range(w.batch))
+        self.rope = torch.empty((self.max_pos, D // 2, 2), dtype=torch.float32, device=dev)
+        self.lib.davet_rope_table(self.max_pos, D, ROPE_THETA, self.rope)
+        self.masked = torch.ones(R, dtype=torch.uint8, device=dev)
+        self.tokens = torch.full((R,), -1, dtype=torch.int32, device=dev)
+        self.argmax = torch.full((R,), -1, dtype=torch.int32, device=dev)
+        self.conf = torch.zeros(R, dtype=torch.float32, device=dev)
+        self.committed = torch.full((w.T, w.batch, w.k), -1, dtype=torch.int32, device=dev)
+        self.stats = torch.zeros((w.T, w.batch, 2), dtype=torch.float32, device=dev)
+        ws = self.lib.davet_unmask_topk_workspace(R, w.V, w.batch)
+        self.workspace = torch.zeros(max(ws, 256), dtype=torch.uint8, device=dev)
+
+    # -------------------------------------------------------------- inputs
+    def load_inputs(self, feats, prompts, non_blocking=False):
+        """feats: per-request bf16 [tiles, G, G, C] visual hidden states;
+        prompts: per-request bf16 [P_b, C] prompt embeddings."""
+        w = self.w
+        for b, f in enumerate(feats):
+            if w.tiles[b]:
+                self.pyr[b][: f.numel() // self.C].copy_(f.reshape(-1, self.C), non_blocking=non_blocking)
+        off = w.text_offsets()
+        for b, p in enumerate(prompts):
+            if w.prompt[b]:
+                self.text[int(off[b]): int(off[b]) + w.prompt[b]].copy_(p, non_blocking=non_blocking)
+
+    def reset_state(self):
+        self.masked.fill_(1)
+        self.tokens.fill_(-1)
+        self.argmax.fill_(-1)
+
+    def build_pyramids(self, stream=None):
+        w = self.w
+        for b in range(w.batch):
+            self.lib.davet_build_pyramid(self.pyr[b], self.pyr[b], w.tiles[b], w.grid, w.n_levels, self.C, None,
+                                         stream)
+
+    # ---------------------------------------------------------------- path
+    def rows(self, t: int) -> int:
+        """Rows of step t's packed sequence (the schedule is known on the host)."""
+        return int(sum(self.w.step_lengths(t)))
+
+    def forward(self, t: int, stream=None, timed=None):
+        """Step t's input rows and every layer; leaves the answer logits.
+        `timed(kind, fn)`, if given, runs each library call (for per-kernel
+        timing); kind is "input", "norm", "gemm" or "attention"."""
+        w, lib = self.w, self.lib
+        run = timed if timed is not None else (lambda kind, fn: fn())
+        N = self.rows(t)
+        C, HD, F = self.C, self.HD, self.F
+        run("input", lambda: lib.davet_gather_view(self.pyr_ptrs, self.tiles, self.text, self.text_off, self.prompt,
+                                                   self.resp, self.schedule[t], w.batch, w.grid, w.n_levels, 0, 0, C,
+                                                   self.x, self.cu, self.max_rows, stream))
+        run("input", lambda: lib.davet_embed_answers(self.emb, w.V, C, self.tokens, self.mask_id, self.cu,
+                                                     self.cu_resp, w.batch, self.R, self.x, stream))
+        for p in self.layers:
+            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g1"], RMS_EPS, self.h, stream=stream))
+            run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wqkv"], 3 * HD, self.qkv, lib.EPI_ROPE, None,
+                                                 self.cu, w.batch, 2 * HD, w.D, self.rope, self.max_pos, stream))
+            run("attention", lambda: lib.davet_step_attention(self.qkv, self.cu, w.batch, self.max_rows, w.H, w.D,
+                                                              w.scale, self.att, stream))
+            run("gemm", lambda: lib.davet_linear(self.att, N, HD, p["wo"], C, self.x, lib.EPI_RESIDUAL, self.x,
+                                                 stream=stream))
+            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g2"], RMS_EPS, self.h, stream=stream))
+            run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wgu"], 2 * F, self.a, lib.EPI_SWIGLU,
+                                                 stream=stream))
+            run("gemm", lambda: lib.davet_linear(self.a, N, F, p["wd"], C, self.x, lib.EPI_RESIDUAL, self.x,
+                                                 stream=stream))
+        run("norm", lambda: lib.davet_rmsnorm(self.x, self.R, C, self.gf, RMS_EPS, self.xa, self.cu, self.cu_resp,
+                                              w.batch, stream))
+        run("gemm", lambda: lib.davet_linear(self.xa, self.R, C, self.wlm, w.V, self.logits, stream=stream))
+
+    def step(self, t: int, stream=None, timed=None):
+        w = self.w
+        run = timed if timed is not None else (lambda kind, fn: fn())
+        self.forward(t, stream, timed)
+        run("unmask", lambda: self.lib.davet_unmask_topk(self.logits, w.V, self.cu_resp, w.batch, self.R, w.k,
+                                                         self.masked, self.tokens, self.argmax, self.conf,
+                                                         self.committed[t], self.stats[t], self.workspace,
+                                                         stream=stream))
+
+    # ---------------------------------------------------- accounting (host)
+    def gemm_flops(self, t: int) -> float:
+        """Tensor-core FLOPs of step t's projections and LM head."""
+        N = self.rows(t)
+        C, HD, F = self.C, self.HD, self.F
+        per_layer = 2.0 * N * C * (3 * HD) + 2.0 * N * HD * C + 2.0 * N * C * (2 * F) + 2.0 * N * F * C
+        return self.L * per_layer + 2.0 * self.R * C * self.w.V
+
+    def gemm_launches_per_step(self) -> int:
+        return 4 * self.L + 1
+
+    def launches_per_step(self) -> int:
+        # gather, embed, per layer 2 norms + 4 GEMMs + attention, final norm, LM head, 2 unmask kernels
+        return 2 + 7 * self.L + 2 + 2

@@ -1,0 +1,99 @@
+"""The full backbone step (paper_2608_01821_gb300/model.py) against the fp64
+layer oracle: step inputs [view || prompt || answer embeddings], n layers,
+final normalization and LM head; then a closed denoising loop."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import layer as L
+from paper_2608_01821_gb300 import workloads
+from paper_2608_01821_gb300.model import RMS_EPS, ROPE_THETA, Backbone
+
+pytestmark = pytest.mark.gpu
+
+
+def f64(t):
+    return t.detach().cpu().double().numpy()
+
+
+def oracle_inputs(bb, feats, prompts, t):
+    """Packed step input as the oracle builds it: the step's pooled view
+    (fp64 means rounded to bf16), the prompt rows, the mask embedding."""
+    w = bb.w
+    C = bb.C
+    rows, cu = [], [0]
+    sides = w.level_sides()
+    for b in range(w.batch):
+        lvl = int(w.schedule[t, b])
+        parts = []
+        if w.tiles[b]:
+            pyr = oracle.pyramid(feats[b], w.tiles[b], w.grid, w.n_levels, C)
+            off = oracle.level_offsets(w.grid, w.n_levels, w.tiles[b])
+            view = torch.from_numpy(pyr[off[lvl]:off[lvl + 1]]).to(torch.bfloat16)
+            parts.append(f64(view))
+        parts.append(f64(prompts[b]))
+        parts.append(np.repeat(f64(bb.emb[bb.mask_id:bb.mask_id + 1]), w.resp[b], axis=0))
+        x = np.concatenate(parts)
+        rows.append(x)
+        cu.append(cu[-1] + len(x))
+    return np.concatenate(rows), cu
+
+
+def layer_weights(p, F):
+    C = p["g1"].numel()
+    wqkv = f64(p["wqkv"])
+    HD = wqkv.shape[0] // 3
+    gu = f64(p["wgu"]).reshape(F // 128, 2, 128, C)
+    return dict(g1=f64(p["g1"]), wq=wqkv[:HD], wk=wqkv[HD:2 * HD], wv=wqkv[2 * HD:], wo=f64(p["wo"]), g2=f64(p["g2"]),
+                wg=gu[:, 0].reshape(F, C), wu=gu[:, 1].reshape(F, C), wd=f64(p["wd"]))
+
+
+@pytest.mark.parametrize("t", [0, 2, 5])
+def test_tiny_two_layer_step_logits(davet, t):
+    w = workloads.make("tiny")
+    bb = Backbone(w, 2, lib=davet)
+    feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C), 100 + b) for b in range(w.batch)]
+    prompts = [workloads.normal_bf16((w.prompt[b], bb.C), 200 + b) for b in range(w.batch)]
+    bb.load_inputs(feats, prompts)
+    bb.reset_state()
+    bb.build_pyramids()
+    bb.forward(t)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    x, cu = oracle_inputs(bb, feats, prompts, t)
+    assert list(bb.cu.cpu().numpy()) == cu
+    for p in bb.layers:
+        x = L.layer(x, layer_weights(p, bb.F), cu, w.H, w.D, ROPE_THETA, RMS_EPS)
+    ref = L.answer_logits(x, cu, w.resp, f64(bb.gf), f64(bb.wlm), RMS_EPS)
+    got = f64(bb.logits[: bb.R])
+    rel = np.linalg.norm(got - ref) / np.linalg.norm(ref)
+    assert rel < 3e-2, rel
+    # the committed choice follows the logits: argmax agreement on rows with a clear margin
+    top2 = np.sort(ref, axis=1)[:, -2:]
+    clear = (top2[:, 1] - top2[:, 0]) > 0.05 * np.abs(top2[:, 1])
+    assert (got.argmax(1)[clear] == ref.argmax(1)[clear]).all()
+
+
+def test_closed_loop_commits_every_position(davet):
+    """T steps of k commits: every answer position ends committed, each step
+    commits only still-masked positions, and every token is a vocabulary id
+    (the mask id never wins a commit only by chance, so it is not excluded)."""
+    w = workloads.make("tiny")
+    bb = Backbone(w, 1, lib=davet)
+    feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C), 300 + b) for b in range(w.batch)]
+    prompts = [workloads.normal_bf16((w.prompt[b], bb.C), 400 + b) for b in range(w.batch)]
+    bb.load_inputs(feats, prompts)
+    bb.reset_state()
+    bb.build_pyramids()
+    for t in range(w.T):
+        bb.step(t)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    committed = bb.committed.cpu().numpy()
+    assert (committed >= 0).all()
+    flat = committed.reshape(-1)
+    assert len(set(flat.tolist())) == len(flat) == w.T * w.k  # every position once
+    assert int(bb.masked.sum()) == w.total_resp - w.T * w.k
+    tok = bb.tokens.cpu().numpy()
+    assert ((tok[flat] >= 0) & (tok[flat] < w.V)).all()
