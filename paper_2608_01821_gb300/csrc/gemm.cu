@@ -100,6 +100,86 @@ __device__ __forceinline__ void load_acc32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The epilogue of one output row of a 256-column tile: `get(c, v)` fills
+// v[0..32) with the fp32 products of columns [c, c + 32) of the row (a
+// warp-collective TMEM load: every lane calls it), and the row's stores
+// happen only where row_ok.
+template <class Get>
+__device__ __forceinline__ void epilogue_row(const Params& p, long long row, bool row_ok, int n0, Get&& get) {
+  if (p.epi == EPI_SWIGLU) {
+    uint16_t* dst = p.out + row * p.ldo + n0 / 2;
+#pragma unroll 1
+    for (int c = 0; c < BN / 2; c += 32) {
+      float g[32], u[32];
+      get(c, g);
+      get(BN / 2 + c, u);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) g[i] = silu(g[i]) * u[i];
+      if (row_ok) store32(dst + c, g);
+    }
+  } else if (p.epi == EPI_ROPE && n0 < p.rope_cols) {
+    // the row's position in its request
+    int pos = 0;
+    if (row_ok) {
+      int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (p.cu[mid] <= row) lo = mid; else hi = mid;
+      }
+      pos = static_cast<int>(row - p.cu[lo]);
+      if (pos >= p.max_pos) {
+        raise_error(p.err, DEV_ERR_ARG);
+        pos = p.max_pos - 1;
+      }
+    }
+    const int half = p.head_dim / 2;
+    const float2* tab = p.rope + static_cast<long long>(pos) * half;
+    uint16_t* dst = p.out + row * p.ldo + n0;
+#pragma unroll 1
+    for (int hb = 0; hb < BN; hb += p.head_dim) {
+#pragma unroll 1
+      for (int c = 0; c < half; c += 32) {
+        float x[32], y[32];
+        get(hb + c, x);
+        get(hb + half + c, y);
+        if (row_ok) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float2 cs = tab[c + i];
+            const float a = x[i], b = y[i];
+            x[i] = a * cs.x - b * cs.y;
+            y[i] = b * cs.x + a * cs.y;
+          }
+          store32(dst + hb + c, x);
+          store32(dst + hb + half + c, y);
+        }
+      }
+    }
+  } else {
+    uint16_t* dst = p.out + row * p.ldo + n0;
+    const uint16_t* res = p.epi == EPI_RESIDUAL ? p.residual + row * p.ldo + n0 : nullptr;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      float v[32];
+      get(c, v);
+      if (row_ok) {
+        if (res) {
+          const uint4* r4 = reinterpret_cast<const uint4*>(res + c);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const uint4 w = r4[u];
+            v[8 * u + 0] += bf16lo(w.x); v[8 * u + 1] += bf16hi(w.x);
+            v[8 * u + 2] += bf16lo(w.y); v[8 * u + 3] += bf16hi(w.y);
+            v[8 * u + 4] += bf16lo(w.z); v[8 * u + 5] += bf16hi(w.z);
+            v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
+          }
+        }
+        store32(dst + c, v);
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p) {
   extern __shared__ uint8_t smem_raw[];
@@ -203,78 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const long long row = static_cast<long long>(m0) + r;
       const bool row_ok = row < p.M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
-      if (p.epi == EPI_SWIGLU) {
-        uint16_t* dst = p.out + row * p.ldo + n0 / 2;
-#pragma unroll 1
-        for (int c = 0; c < BN / 2; c += 32) {
-          float g[32], u[32];
-          load_acc32(acc + c, g);
-          load_acc32(acc + BN / 2 + c, u);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) g[i] = silu(g[i]) * u[i];
-          if (row_ok) store32(dst + c, g);
-        }
-      } else if (p.epi == EPI_ROPE && n0 < p.rope_cols) {
-        // the row's position in its request
-        int pos = 0;
-        if (row_ok) {
-          int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
-          while (hi - lo > 1) {
-            const int mid = (lo + hi) >> 1;
-            if (p.cu[mid] <= row) lo = mid; else hi = mid;
-          }
-          pos = static_cast<int>(row - p.cu[lo]);
-          if (pos >= p.max_pos) {
-            raise_error(p.err, DEV_ERR_ARG);
-            pos = p.max_pos - 1;
-          }
-        }
-        const int half = p.head_dim / 2;
-        const float2* tab = p.rope + static_cast<long long>(pos) * half;
-        uint16_t* dst = p.out + row * p.ldo + n0;
-#pragma unroll 1
-        for (int hb = 0; hb < BN; hb += p.head_dim) {
-#pragma unroll 1
-          for (int c = 0; c < half; c += 32) {
-            float x[32], y[32];
-            load_acc32(acc + hb + c, x);
-            load_acc32(acc + hb + half + c, y);
-            if (row_ok) {
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                const float2 cs = tab[c + i];
-                const float a = x[i], b = y[i];
-                x[i] = a * cs.x - b * cs.y;
-                y[i] = b * cs.x + a * cs.y;
-              }
-              store32(dst + hb + c, x);
-              store32(dst + hb + half + c, y);
-            }
-          }
-        }
-      } else {
-        uint16_t* dst = p.out + row * p.ldo + n0;
-        const uint16_t* res = p.epi == EPI_RESIDUAL ? p.residual + row * p.ldo + n0 : nullptr;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          float v[32];
-          load_acc32(acc + c, v);
-          if (row_ok) {
-            if (res) {
-              const uint4* r4 = reinterpret_cast<const uint4*>(res + c);
-#pragma unroll
-              for (int u = 0; u < 4; ++u) {
-                const uint4 w = r4[u];
-                v[8 * u + 0] += bf16lo(w.x); v[8 * u + 1] += bf16hi(w.x);
-                v[8 * u + 2] += bf16lo(w.y); v[8 * u + 3] += bf16hi(w.y);
-                v[8 * u + 4] += bf16lo(w.z); v[8 * u + 5] += bf16hi(w.z);
-                v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
-              }
-            }
-            store32(dst + c, v);
-          }
-        }
-      }
+      epilogue_row(p, row, row_ok, n0, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.acc_empty[ab]);
