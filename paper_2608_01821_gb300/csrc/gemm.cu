@@ -77,7 +77,8 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
   return __all_sync(0xffffffffu, ok);
 }
 
-__device__ __forceinline__ float silu(float g) { return g / (1.0f + __expf(-g)); }
+// silu(g) = g * sigmoid(g); the fast division is exact enough for a bf16 output
+__device__ __forceinline__ float silu(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
 __device__ __forceinline__ void store32(uint16_t* dst, const float (&v)[32]) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
@@ -298,6 +299,214 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ------------------------------------------------------------ 2-SM tiles
+// A cluster of two CTAs (a CTA pair on two SMs) computes a 256 x 256 tile
+// with tcgen05 MMAs of M = 256 issued by the even CTA: each CTA holds its
+// 128 rows of A and 128 of the tile's 256 rows of W, so each SM takes in half
+// the operand bytes per FLOP of the one-CTA tile.  Each CTA's TMEM holds the
+// accumulator of its 128 output rows; both CTAs run the epilogue on their own
+// rows, on one of two accumulators while the MMAs fill the other.  Both
+// producers' TMA copies complete on the even CTA's barrier; the MMA commits
+// arrive on both CTAs' barriers; the odd CTA's epilogue signals the even
+// CTA's accumulator barrier remotely.  The pair's TMEM allocation is
+// collective (both CTAs get the same columns); the kernel checks it.
+constexpr int ST2 = 6;
+constexpr uint32_t kStageB2 = BM * BK * 2;  // 128 rows of W: 16 KB
+constexpr uint32_t kTmemCols2 = 512;        // two 128 x 256 accumulators per CTA
+
+struct Smem2 {
+  alignas(1024) uint8_t a[ST2][kStageA];
+  alignas(1024) uint8_t b[ST2][kStageB2];
+  uint64_t full[ST2], empty[ST2];
+  uint64_t acc_full[2], acc_empty[2];
+  uint64_t fin;
+  uint32_t tmem;
+  int abort;
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void remote_arrive(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const void* tmap, uint32_t bar_cluster, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar_cluster), "r"(c0), "r"(c1)
+      : "memory");
+}
+template <bool ACC>
+__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc) {
+  if constexpr (ACC)
+    asm volatile("tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, 1;" ::"r"(d_tmem), "l"(a_desc), "l"(b_desc),
+                 "r"(idesc)
+                 : "memory");
+  else
+    asm volatile("tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, 0;" ::"r"(d_tmem), "l"(a_desc), "l"(b_desc),
+                 "r"(idesc)
+                 : "memory");
+}
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm2_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  Smem2& s = *reinterpret_cast<Smem2*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int* abort_flag = &s.abort;
+  const uint32_t rank = cluster_rank();
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+
+  if (tid == 0) {
+    s.abort = 0;
+    for (int i = 0; i < ST2; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.acc_full[i], 1);
+      mbar_init(&s.acc_empty[i], 8);  // four epilogue warps in each CTA of the pair
+    }
+    mbar_init(&s.fin, 1);
+    fence_mbar_init();
+  }
+  if (warp == kWarpMma) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s.tmem)),
+                 "r"(kTmemCols2)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  if (warp == kWarpTma && lane == 0) {
+    tma_prefetch_desc(&tmap_a);
+    tma_prefetch_desc(&tmap_w);
+  }
+  pdl_launch_dependents();
+  pdl_wait();
+  tc_fence_before();
+  cluster_sync_all();  // barriers initialized and TMEM allocated in both CTAs
+  tc_fence_after();
+  const uint32_t tmem = s.tmem;
+  if (tid == 0) {
+    // both CTAs must hold the accumulator at the same TMEM address
+    uint32_t lead;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(lead) : "r"(map_to_rank(&s.tmem, 0)) : "memory");
+    if (lead != tmem) {
+      raise_error(p.err, DEV_ERR_ARG);
+      s.abort = 1;
+    }
+  }
+  __syncthreads();
+  const int tiles_m2 = static_cast<int>((p.M + 2 * BM - 1) / (2 * BM));
+  const int n_tiles = tiles_m2 * p.tiles_n;
+  const int nk = p.K / BK;
+
+  if (warp == kWarpTma) {
+    if (lane == 0 && !s.abort) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = pair; ok && t < n_tiles; t += n_pairs) {
+        const int m0 = (t % tiles_m2) * 2 * BM + rank * BM, n0 = (t / tiles_m2) * BN + rank * BM;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const uint32_t st = it % ST2;
+          if (it >= ST2 && !mbar_wait(&s.empty[st], ((it / ST2) - 1) & 1, p.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (rank == 0) mbar_arrive_expect_tx(&s.full[st], 2 * (kStageA + kStageB2));
+          const uint32_t bar = map_to_rank(&s.full[st], 0);
+          tma_load_2d_pair(s.a[st], &tmap_a, bar, kb * BK, m0);
+          tma_load_2d_pair(s.b[st], &tmap_w, bar, kb * BK, n0);
+        }
+      }
+    }
+  } else if (warp == kWarpMma) {
+    if (lane == 0 && rank == 0 && !s.abort) {
+      constexpr uint32_t kIdesc = idesc_bf16_f32(2 * BM, BN, false, false);
+      uint32_t it = 0, tc = 0;
+      bool ok = true;
+      for (int t = pair; ok && t < n_tiles; t += n_pairs, ++tc) {
+        const uint32_t ab = tc & 1, use = tc >> 1;
+        if (use > 0 && !mbar_wait(&s.acc_empty[ab], (use - 1) & 1, p.err, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + ab * BN;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const uint32_t st = it % ST2;
+          if (!mbar_wait(&s.full[st], (it / ST2) & 1, p.err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t da = sw128_desc(smem_u32(s.a[st]), 16, 1024);
+          const uint64_t db = sw128_desc(smem_u32(s.b[st]), 16, 1024);
+          if (kb == 0)
+            umma_pair<false>(d, da, db, kIdesc);
+          else
+            umma_pair<true>(d, da, db, kIdesc);
+          umma_pair<true>(d, da + 2, db + 2, kIdesc);
+          umma_pair<true>(d, da + 4, db + 4, kIdesc);
+          umma_pair<true>(d, da + 6, db + 6, kIdesc);
+          umma_commit_pair(&s.empty[st]);
+        }
+        if (ok) umma_commit_pair(&s.acc_full[ab]);
+      }
+      asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                       smem_u32(&s.fin))
+                   : "memory");
+      mbar_wait(&s.fin, 0, p.err, nullptr);
+    }
+  } else {
+    const int q = warp & 3;
+    const int r = 32 * q + lane;
+    uint32_t tc = 0;
+    for (int t = pair; !s.abort && t < n_tiles; t += n_pairs, ++tc) {
+      const uint32_t ab = tc & 1, use = tc >> 1;
+      if (!warp_wait(&s.acc_full[ab], use & 1, p.err, abort_flag)) break;
+      tc_fence_after();
+      const int m0 = (t % tiles_m2) * 2 * BM + rank * BM, n0 = (t / tiles_m2) * BN;
+      const long long row = static_cast<long long>(m0) + r;
+      const bool row_ok = row < p.M;
+      const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
+      epilogue_row(p, row, row_ok, n0, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (rank == 0)
+          mbar_arrive(&s.acc_empty[ab]);
+        else
+          remote_arrive(map_to_rank(&s.acc_empty[ab], 0));
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // no CTA leaves while its peer may still signal it or read its operands
+  if (warp == kWarpMma) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols2) : "memory");
+  }
+}
+
 // cos/sin table of the rotary embedding: tab[p][d] = (cos, sin)(p * theta^(-2d/D)).
 __global__ void rope_table_kernel(float2* tab, int max_pos, int half, double theta) {
   pdl_launch_dependents();
@@ -461,6 +670,7 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   if (e != cudaSuccess) return cuda_fail(e);
   if (dev < 0 || dev >= 64) return DAVET_ERR_UNSUPPORTED;
   const size_t smem = sizeof(Smem) + 1024;
+  const size_t smem2 = sizeof(Smem2) + 1024;
   {
     std::lock_guard<std::mutex> g(g_mu);
     if (g_sms[dev] == 0) {
@@ -469,6 +679,8 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
     }
     if (!g_attr[dev]) {
       e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(gemm2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem2));
       if (e != cudaSuccess) return cuda_fail(e);
       g_attr[dev] = true;
     }
@@ -496,8 +708,35 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   p.err = err;
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // 256 x 256 tiles on CTA pairs whenever the odd CTA has rows to compute:
+  // the same work per SM as 128 x 256 tiles, half the operand bytes per SM
+  const int pairs = g_sms[dev] / 2;
+  const long long tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * p.tiles_n;
+  if (M > BM) {
+    CUtensorMap mw2;
+    if (!make_map(&mw2, W, N, K, BM)) return DAVET_ERR_INVALID_ARG;
+    const int grid2 = 2 * static_cast<int>(std::min<long long>(tiles2, pairs));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid2);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem2;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 2 : 1;
+    e = cudaLaunchKernelEx(&cfg, gemm2_kernel, ma, mw2, p);
+    if (e != cudaSuccess) return cuda_fail(e);
+    return check_launch();
+  }
   const int grid = static_cast<int>(std::min<long long>(tiles, g_sms[dev]));
-  e = launch(gemm_kernel, dim3(grid), dim3(kThreads), smem, static_cast<cudaStream_t>(stream), ma, mw, p);
+  e = launch(gemm_kernel, dim3(grid), dim3(kThreads), smem, st, ma, mw, p);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

@@ -217,3 +217,55 @@ def test_large_projection_sampled_rows(davet):
     rows = np.concatenate([rows, [0, 127, 128, M - 1]])
     ref = f64(A)[rows] @ f64(W).T
     check_close(out[torch.from_numpy(rows).cuda()], ref, "qkv 8B rows")
+
+
+# ------------------------------------------------------------- 2-SM tiles
+# Shapes with at least one wave of 256 x 256 tiles (76 CTA pairs) take the
+# CTA-pair kernel; M not a multiple of 256 leaves the odd CTA of the last row
+# block partly or wholly past the end.
+@pytest.mark.parametrize("M,K,N", [(512, 256, 256 * 76), (600, 512, 256 * 40), (300, 128, 256 * 80)])
+def test_pair_tiles_store(davet, M, K, N):
+    A = rand_bf16((M, K), 60 + M).cuda()
+    W = rand_bf16((N, K), 61 + K, K ** -0.5).cuda()
+    out = linear(davet, A, W)
+    rows = np.unique(np.concatenate([np.random.default_rng(M).choice(M, 64, replace=False), [0, 127, 128, 255, 256,
+                                                                                              M - 1]]))
+    check_close(out[torch.from_numpy(rows).cuda()], f64(A)[rows] @ f64(W).T, f"pair {M}x{K}x{N}")
+
+
+def test_pair_tiles_residual_and_gated_mlp(davet):
+    M, K = 520, 256
+    N = 256 * 38
+    A = rand_bf16((M, K), 70).cuda()
+    W = rand_bf16((N, K), 71, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 72).cuda()
+    x = R.clone()
+    davet.davet_linear(A, M, K, W, N, x, davet.EPI_RESIDUAL, x)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    check_close(x, f64(R) + f64(A) @ f64(W).T, "pair residual")
+    F = 128 * 80
+    Wg = rand_bf16((F, K), 73, K ** -0.5)
+    Wu = rand_bf16((F, K), 74, K ** -0.5)
+    Wgu = torch.stack([Wg.reshape(F // 128, 128, K), Wu.reshape(F // 128, 128, K)], 1).reshape(2 * F, K).cuda()
+    out = linear(davet, A, Wgu, davet.EPI_SWIGLU, out_cols=F)
+    a = f64(A)
+    check_close(out, L.silu(a @ f64(Wg).T) * (a @ f64(Wu).T), "pair swiglu")
+
+
+def test_pair_tiles_rotary(davet):
+    D, H, K = 128, 64, 256
+    HD = H * D
+    cu = [0, 300, 301, 700]
+    M = cu[-1]
+    A = rand_bf16((M, K), 80).cuda()
+    W = rand_bf16((3 * HD, K), 81, K ** -0.5).cuda()
+    tab = torch.empty((1024, D // 2, 2), dtype=torch.float32, device="cuda")
+    davet.davet_rope_table(1024, D, THETA, tab)
+    out = linear(davet, A, W, davet.EPI_ROPE, cu_seqlens=torch.tensor(cu, dtype=torch.int32, device="cuda"),
+                 batch=3, rope_cols=2 * HD, head_dim=D, rope_table=tab, max_pos=1024)
+    y = f64(A) @ f64(W).T
+    pos = L.positions(cu)
+    ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
+                          y[:, 2 * HD:]], axis=1)
+    check_close(out, ref, "pair rope")
