@@ -482,7 +482,21 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  *            (davet_rope_table, [max_pos][head_dim/2] float2), max_pos:
  *            epilogue 3 only (nullable otherwise); a position >= max_pos is
  *            clamped and flags DAVET_DEV_ARG
- * One persistent kernel on `stream`.
+ *   workspace, workspace_bytes   device scratch, nullable.  When the output
+ *            tiles would occupy less than half of the SMs (few rows, few
+ *            column blocks) and the workspace holds at least
+ *            davet_linear_workspace_bytes(M, K, N) bytes (16-byte aligned), K is
+ *            split into slices on separate SM pairs whose fp32 partials are
+ *            added in slice order (the result does not depend on timing)
+ *            before the epilogue; otherwise one pass over K per tile.  A
+ *            workspace must not be shared by calls that may run at the same
+ *            time.
+ * One persistent kernel on `stream` (with a split: a second kernel adds the
+ * slices and applies the epilogue).  M > 128 runs on CTA pairs (clusters of
+ * two CTAs on two SMs).
+ *
+ * davet_linear_workspace_bytes -- the workspace davet_linear can use for this
+ * shape on the current device (0: none).
  *
  * davet_rope_table -- table[p][d] = (cos, sin)(p * theta^(-2d/head_dim)),
  * fp32, for p < max_pos and d < head_dim/2 (computed in fp64 on the device).
@@ -501,7 +515,9 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  */
 davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                           const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols, int head_dim,
-                          const void* rope_table, int max_pos, void* stream);
+                          const void* rope_table, int max_pos, void* workspace, size_t workspace_bytes,
+                          void* stream);
+davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, size_t* bytes);
 davet_status davet_rope_table(int max_pos, int head_dim, double theta, void* table, void* stream);
 davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
                            const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, void* stream);

@@ -62,6 +62,11 @@ struct Params {
   int max_pos;
   const float2* rope;  // [max_pos][head_dim / 2] (cos, sin)
   unsigned* err;
+  // split of K (CTA-pair kernel): `split` slices of `kb_per` k-blocks (the last
+  // takes the rest) write fp32 partials [split][tiles_n][M rounded to 256][256]
+  int split;
+  int kb_per;
+  float* part;
 };
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1) {
@@ -417,16 +422,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   const int tiles_m2 = static_cast<int>((p.M + 2 * BM - 1) / (2 * BM));
-  const int n_tiles = tiles_m2 * p.tiles_n;
+  const int n_tiles = tiles_m2 * p.tiles_n * p.split;
   const int nk = p.K / BK;
+  // unit t: slice t % split of output tile t / split (m-block fastest)
+  auto k_range = [&](int t, int& kb0, int& kb1) {
+    const int sl = t % p.split;
+    kb0 = sl * p.kb_per;
+    kb1 = sl + 1 == p.split ? nk : kb0 + p.kb_per;
+  };
 
   if (warp == kWarpTma) {
     if (lane == 0 && !s.abort) {
       uint32_t it = 0;
       bool ok = true;
       for (int t = pair; ok && t < n_tiles; t += n_pairs) {
-        const int m0 = (t % tiles_m2) * 2 * BM + rank * BM, n0 = (t / tiles_m2) * BN + rank * BM;
-        for (int kb = 0; kb < nk; ++kb, ++it) {
+        const int bt = t / p.split;
+        const int m0 = (bt % tiles_m2) * 2 * BM + rank * BM, n0 = (bt / tiles_m2) * BN + rank * BM;
+        int kb0, kb1;
+        k_range(t, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const uint32_t st = it % ST2;
           if (it >= ST2 && !mbar_wait(&s.empty[st], ((it / ST2) - 1) & 1, p.err, abort_flag)) {
             ok = false;
@@ -449,7 +463,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (use > 0 && !mbar_wait(&s.acc_empty[ab], (use - 1) & 1, p.err, abort_flag)) break;
         tc_fence_after();
         const uint32_t d = tmem + ab * BN;
-        for (int kb = 0; kb < nk; ++kb, ++it) {
+        int kb0, kb1;
+        k_range(t, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const uint32_t st = it % ST2;
           if (!mbar_wait(&s.full[st], (it / ST2) & 1, p.err, abort_flag)) {
             ok = false;
@@ -458,7 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           const uint64_t da = sw128_desc(smem_u32(s.a[st]), 16, 1024);
           const uint64_t db = sw128_desc(smem_u32(s.b[st]), 16, 1024);
-          if (kb == 0)
+          if (kb == kb0)
             umma_pair<false>(d, da, db, kIdesc);
           else
             umma_pair<true>(d, da, db, kIdesc);
@@ -482,11 +498,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t ab = tc & 1, use = tc >> 1;
       if (!warp_wait(&s.acc_full[ab], use & 1, p.err, abort_flag)) break;
       tc_fence_after();
-      const int m0 = (t % tiles_m2) * 2 * BM + rank * BM, n0 = (t / tiles_m2) * BN;
+      const int bt = t / p.split;
+      const int m0 = (bt % tiles_m2) * 2 * BM + rank * BM, nb = bt / tiles_m2;
       const long long row = static_cast<long long>(m0) + r;
       const bool row_ok = row < p.M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
-      epilogue_row(p, row, row_ok, n0, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
+      if (p.split > 1) {
+        // fp32 partial products of this slice; the reduction kernel applies the epilogue
+        float4* dst = reinterpret_cast<float4*>(
+            p.part + ((static_cast<long long>(t % p.split) * p.tiles_n + nb) * (tiles_m2 * 2 * BM) + row) * BN);
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          load_acc32(acc + c, v);
+          if (row_ok) {
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              dst[c / 4 + u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+          }
+        }
+      } else {
+        epilogue_row(p, row, row_ok, nb * BN, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -504,6 +537,84 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kWarpMma) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols2) : "memory");
+  }
+}
+
+// Sum of the K slices' partials in slice order, then the epilogue: one warp
+// per (row, 256-column block), lane l holding columns [8l, 8l + 8) (coalesced
+// 1 KB per slice); the gated MLP pairs lane l with lane l + 16 (gate, up),
+// the rotary embedding lane l with lane l ^ (D/16) (columns d, d + D/2).
+__global__ void __launch_bounds__(256) split_reduce_kernel(Params p) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  const long long mp = ((p.M + 2 * BM - 1) / (2 * BM)) * 2 * BM;
+  for (long long u = w0; u < p.M * p.tiles_n; u += nw) {
+    const int nb = static_cast<int>(u / p.M);
+    const long long row = u % p.M;
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = 0.0f;
+    for (int sl = 0; sl < p.split; ++sl) {
+      const float4* src =
+          reinterpret_cast<const float4*>(p.part + ((static_cast<long long>(sl) * p.tiles_n + nb) * mp + row) * BN) +
+          2 * lane;
+      const float4 a = __ldcg(src), b = __ldcg(src + 1);
+      v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
+      v[4] += b.x; v[5] += b.y; v[6] += b.z; v[7] += b.w;
+    }
+    const int n0 = nb * BN;
+    uint4 o;
+    uint16_t* dst;
+    bool write = true;
+    if (p.epi == EPI_SWIGLU) {
+      float up[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) up[i] = __shfl_down_sync(0xffffffffu, v[i], 16);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = silu(v[i]) * up[i];
+      write = lane < 16;
+      dst = p.out + row * p.ldo + n0 / 2 + 8 * lane;
+    } else if (p.epi == EPI_ROPE && n0 < p.rope_cols) {
+      const int half = p.head_dim / 2;
+      float pv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) pv[i] = __shfl_xor_sync(0xffffffffu, v[i], half / 8);
+      int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (p.cu[mid] <= row) lo = mid; else hi = mid;
+      }
+      int pos = static_cast<int>(row - p.cu[lo]);
+      if (pos >= p.max_pos) {
+        if (lane == 0) raise_error(p.err, DEV_ERR_ARG);
+        pos = p.max_pos - 1;
+      }
+      const bool first = (8 * lane) % p.head_dim < half;  // columns in the first half of the head
+      const float2* tab = p.rope + static_cast<long long>(pos) * half + (8 * lane) % half;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float2 cs = tab[i];
+        v[i] = first ? v[i] * cs.x - pv[i] * cs.y : v[i] * cs.x + pv[i] * cs.y;
+      }
+      dst = p.out + row * p.ldo + n0 + 8 * lane;
+    } else {
+      dst = p.out + row * p.ldo + n0 + 8 * lane;
+      if (p.epi == EPI_RESIDUAL) {
+        const uint4 w = *reinterpret_cast<const uint4*>(p.residual + row * p.ldo + n0 + 8 * lane);
+        v[0] += bf16lo(w.x); v[1] += bf16hi(w.x);
+        v[2] += bf16lo(w.y); v[3] += bf16hi(w.y);
+        v[4] += bf16lo(w.z); v[5] += bf16hi(w.z);
+        v[6] += bf16lo(w.w); v[7] += bf16hi(w.w);
+      }
+    }
+    o.x = pack_bf16x2(v[0], v[1]);
+    o.y = pack_bf16x2(v[2], v[3]);
+    o.z = pack_bf16x2(v[4], v[5]);
+    o.w = pack_bf16x2(v[6], v[7]);
+    if (write) *reinterpret_cast<uint4*>(dst) = o;
   }
 }
 
@@ -650,11 +761,42 @@ std::mutex g_mu;
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+
+// K slices for the CTA-pair kernel when its tiles cover less than half of the
+// pairs (few rows and few column blocks): as many slices as fill the pairs,
+// each at least 8 k-blocks.  1 = no split.
+int pick_split(long long M, int tiles_n, int nk, int pairs) {
+  if (M <= BM) return 1;
+  const long long tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * tiles_n;
+  if (2 * tiles2 > pairs) return 1;
+  const int S = std::min(static_cast<int>(pairs / tiles2), nk / 8);
+  return S >= 2 ? S : 1;
+}
+
+size_t split_bytes(long long M, int tiles_n, int S) {
+  return static_cast<size_t>(S) * tiles_n * (((M + 2 * BM - 1) / (2 * BM)) * 2 * BM) * BN * 4;
+}
+
 }  // namespace
+
+extern "C" davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, size_t* bytes) {
+  if (!bytes || M < 0 || K < BK || K % BK != 0 || N < BN || N % BN != 0) return DAVET_ERR_INVALID_ARG;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= 64) return DAVET_ERR_UNSUPPORTED;
+  int sms = 0;
+  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  const int S = pick_split(M, N / BN, K / BK, sms / 2);
+  *bytes = S > 1 ? split_bytes(M, N / BN, S) : 0;
+  return DAVET_OK;
+}
 
 extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                                      const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols,
-                                     int head_dim, const void* rope_table, int max_pos, void* stream) {
+                                     int head_dim, const void* rope_table, int max_pos, void* workspace,
+                                     size_t workspace_bytes, void* stream) {
   if (M < 0 || M > 0x7fffffffLL || K < BK || K % BK != 0 || N < BN || N % BN != 0) return DAVET_ERR_INVALID_ARG;
   if (epilogue < EPI_STORE || epilogue > EPI_ROPE) return DAVET_ERR_INVALID_ARG;
   if (M == 0) return DAVET_OK;
@@ -706,6 +848,9 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   p.max_pos = max_pos;
   p.rope = static_cast<const float2*>(rope_table);
   p.err = err;
+  p.split = 1;
+  p.kb_per = K / BK;
+  p.part = nullptr;
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -714,9 +859,15 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   const int pairs = g_sms[dev] / 2;
   const long long tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * p.tiles_n;
   if (M > BM) {
+    const int S = pick_split(M, p.tiles_n, K / BK, pairs);
+    if (S > 1 && workspace && workspace_bytes >= split_bytes(M, p.tiles_n, S) && aligned16(workspace)) {
+      p.split = S;
+      p.kb_per = (K / BK) / S;
+      p.part = static_cast<float*>(workspace);
+    }
     CUtensorMap mw2;
     if (!make_map(&mw2, W, N, K, BM)) return DAVET_ERR_INVALID_ARG;
-    const int grid2 = 2 * static_cast<int>(std::min<long long>(tiles2, pairs));
+    const int grid2 = 2 * static_cast<int>(std::min<long long>(tiles2 * p.split, pairs));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid2);
     cfg.blockDim = dim3(kThreads);
@@ -733,6 +884,12 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
     cfg.numAttrs = pdl_enabled() ? 2 : 1;
     e = cudaLaunchKernelEx(&cfg, gemm2_kernel, ma, mw2, p);
     if (e != cudaSuccess) return cuda_fail(e);
+    if (p.split > 1) {
+      const long long warps = M * p.tiles_n;
+      const unsigned blocks = static_cast<unsigned>(std::min<long long>((warps + 7) / 8, 152LL * 16));
+      e = launch(split_reduce_kernel, dim3(blocks), dim3(256), 0, st, p);
+      if (e != cudaSuccess) return cuda_fail(e);
+    }
     return check_launch();
   }
   const int grid = static_cast<int>(std::min<long long>(tiles, g_sms[dev]));

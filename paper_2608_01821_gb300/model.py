@@ -104,6 +104,11 @@ class Backbone:
         self.stats = torch.zeros((w.T, w.batch, 2), dtype=torch.float32, device=dev)
         ws = self.lib.davet_unmask_topk_workspace(R, w.V, w.batch)
         self.workspace = torch.zeros(max(ws, 256), dtype=torch.uint8, device=dev)
+        # scratch of the projections' K split (steps with few rows)
+        shapes = [(C, 3 * self.HD), (self.HD, C), (C, 2 * F), (F, C), (C, w.V)]
+        rows = {self.rows(t) for t in range(w.T)} | {R}
+        gw = max(self.lib.davet_linear_workspace_bytes(m, k, n) for k, n in shapes for m in rows)
+        self.gemm_ws = torch.empty(max(gw, 256), dtype=torch.uint8, device=dev)
 
     # -------------------------------------------------------------- inputs
     def load_inputs(self, feats, prompts, non_blocking=False):
@@ -142,6 +147,7 @@ class Backbone:
         run = timed if timed is not None else (lambda kind, fn: fn())
         N = self.rows(t)
         C, HD, F = self.C, self.HD, self.F
+        ws = self.gemm_ws
         run("input", lambda: lib.davet_gather_view(self.pyr_ptrs, self.tiles, self.text, self.text_off, self.prompt,
                                                    self.resp, self.schedule[t], w.batch, w.grid, w.n_levels, 0, 0, C,
                                                    self.x, self.cu, self.max_rows, stream))
@@ -150,19 +156,21 @@ class Backbone:
         for p in self.layers:
             run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g1"], RMS_EPS, self.h, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wqkv"], 3 * HD, self.qkv, lib.EPI_ROPE, None,
-                                                 self.cu, w.batch, 2 * HD, w.D, self.rope, self.max_pos, stream))
+                                                 self.cu, w.batch, 2 * HD, w.D, self.rope, self.max_pos, ws,
+                                                 stream=stream))
             run("attention", lambda: lib.davet_step_attention(self.qkv, self.cu, w.batch, self.max_rows, w.H, w.D,
                                                               w.scale, self.att, stream))
             run("gemm", lambda: lib.davet_linear(self.att, N, HD, p["wo"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 stream=stream))
+                                                 workspace=ws, stream=stream))
             run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g2"], RMS_EPS, self.h, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wgu"], 2 * F, self.a, lib.EPI_SWIGLU,
-                                                 stream=stream))
+                                                 workspace=ws, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.a, N, F, p["wd"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 stream=stream))
+                                                 workspace=ws, stream=stream))
         run("norm", lambda: lib.davet_rmsnorm(self.x, self.R, C, self.gf, RMS_EPS, self.xa, self.cu, self.cu_resp,
                                               w.batch, stream))
-        run("gemm", lambda: lib.davet_linear(self.xa, self.R, C, self.wlm, w.V, self.logits, stream=stream))
+        run("gemm", lambda: lib.davet_linear(self.xa, self.R, C, self.wlm, w.V, self.logits, workspace=ws,
+                                             stream=stream))
 
     def step(self, t: int, stream=None, timed=None):
         w = self.w

@@ -269,3 +269,69 @@ def test_pair_tiles_rotary(davet):
     ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
                           y[:, 2 * HD:]], axis=1)
     check_close(out, ref, "pair rope")
+
+
+# ------------------------------------------------- K split on CTA pairs
+# Few rows and few column blocks (tiles on less than half of the SM pairs)
+# take the split path: K slices on separate pairs, fp32 partials added in
+# slice order by a second kernel that applies the epilogue.
+@pytest.mark.parametrize("M,K,N,epi", [(241, 4096, 4096, 1), (200, 12288, 4096, 1), (300, 2048, 2560, 0),
+                                       (241, 1024, 2048, 2)])
+def test_pair_split_k(davet, M, K, N, epi):
+    nbytes = davet.davet_linear_workspace_bytes(M, K, N)
+    assert nbytes > 0
+    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    A = rand_bf16((M, K), 90 + M).cuda()
+    W = rand_bf16((N, K), 91 + N, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 92).cuda() if epi == 1 else None
+    outs = []
+    for _ in range(2):
+        out = torch.full((M + 3, N // 2 if epi == 2 else N), float("nan"), dtype=torch.bfloat16, device="cuda")
+        if R is not None:
+            out[:M].copy_(R)
+        davet.davet_linear(A, M, K, W, N, out, epi, out if epi == 1 else None, workspace=ws)
+        torch.cuda.synchronize()
+        assert davet.davet_device_status() == (0, 0)
+        assert torch.isnan(out[M:].float()).all()
+        outs.append(out[:M].clone())
+    assert torch.equal(outs[0], outs[1])
+    y = f64(A) @ f64(W).T
+    if epi == 0:
+        ref = y
+    elif epi == 1:
+        ref = f64(R) + y
+    else:
+        F = N // 2
+        blocks = y.reshape(M, F // 128, 2, 128)
+        ref = (L.silu(blocks[:, :, 0]) * blocks[:, :, 1]).reshape(M, F)
+    check_close(outs[0], ref, f"split {M}x{K}x{N} epi {epi}")
+
+
+@pytest.mark.parametrize("D,H", [(128, 4), (64, 8)])
+def test_pair_split_k_rotary(davet, D, H):
+    K = 1024
+    HD = H * D
+    cu = [0, 37, 150, 201]
+    M = cu[-1]
+    A = rand_bf16((M, K), 95).cuda()
+    W = rand_bf16((3 * HD, K), 96, K ** -0.5).cuda()
+    tab = torch.empty((256, D // 2, 2), dtype=torch.float32, device="cuda")
+    davet.davet_rope_table(256, D, THETA, tab)
+    nbytes = davet.davet_linear_workspace_bytes(M, K, 3 * HD)
+    assert nbytes > 0
+    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    out = linear(davet, A, W, davet.EPI_ROPE, cu_seqlens=torch.tensor(cu, dtype=torch.int32, device="cuda"),
+                 batch=3, rope_cols=2 * HD, head_dim=D, rope_table=tab, max_pos=256, workspace=ws)
+    y = f64(A) @ f64(W).T
+    pos = L.positions(cu)
+    ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
+                          y[:, 2 * HD:]], axis=1)
+    check_close(out, ref, "split rope")
+
+
+def test_split_workspace_too_small_runs_one_pass(davet):
+    M, K, N = 241, 4096, 4096
+    A = rand_bf16((M, K), 97).cuda()
+    W = rand_bf16((N, K), 98, K ** -0.5).cuda()
+    out = linear(davet, A, W, workspace=torch.empty(256, dtype=torch.uint8, device="cuda"))
+    check_close(out, f64(A) @ f64(W).T, "fallback")
