@@ -441,7 +441,7 @@ def run_backbone(args, rank, world, local_rank):
             "flops_per_launch": gemm_flops / max(n_gemm, 1),
         },
         "clocks": clocks.summary(),
-        "gpu_launches": (w.batch + w.T * bb.launches_per_step()) * args.steps,
+        "gpu_launches": (sum(1 for x in w.tiles if x > 0) + sum(bb.launches(t) for t in range(w.T))) * args.steps,
         "e2e": e2e,
     }
 

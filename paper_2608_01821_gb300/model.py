@@ -189,9 +189,18 @@ class Backbone:
         per_layer = 2.0 * N * C * (3 * HD) + 2.0 * N * HD * C + 2.0 * N * C * (2 * F) + 2.0 * N * F * C
         return self.L * per_layer + 2.0 * self.R * C * self.w.V
 
-    def gemm_launches_per_step(self) -> int:
-        return 4 * self.L + 1
+    def gemm_launches(self, t: int) -> int:
+        """Kernels of step t's projections: one per GEMM, two where K is split."""
+        N = self.rows(t)
+        C, HD, F = self.C, self.HD, self.F
 
-    def launches_per_step(self) -> int:
-        # gather, embed, per layer 2 norms + 4 GEMMs + attention, final norm, LM head, 2 unmask kernels
-        return 2 + 7 * self.L + 2 + 2
+        def k(m, kk, n):
+            return 2 if self.lib.davet_linear_workspace_bytes(m, kk, n) > 0 else 1
+
+        per_layer = k(N, C, 3 * HD) + k(N, HD, C) + k(N, C, 2 * F) + k(N, F, C)
+        return self.L * per_layer + k(self.R, C, self.w.V)
+
+    def launches(self, t: int) -> int:
+        """Kernels of step t: gather, embedding, per layer two norms and the
+        attention, the projections, the final norm, two unmask kernels."""
+        return 2 + 3 * self.L + self.gemm_launches(t) + 1 + 2
