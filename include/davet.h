@@ -93,6 +93,14 @@ int davet_last_cuda_error(void);
  */
 davet_status davet_device_status(unsigned* flags, int clear);
 
+/*
+ * The same word read on `stream`: waits for the work queued on that stream
+ * only (not the whole device), copies the word to *flags (nullable) and
+ * returns DAVET_OK, DAVET_ERR_TIMEOUT or DAVET_ERR_DEVICE as above.  It does
+ * not clear the word.  Outside stream capture.
+ */
+davet_status davet_sync_status(void* stream, unsigned* flags);
+
 /* --------------------------------------------------------- evidence views */
 
 /*
@@ -209,6 +217,14 @@ davet_status davet_gather_view(const void* const* pyr_ptrs_dev, const int32_t* t
  */
 davet_status davet_step_attention(const void* qkv, const int32_t* cu_seqlens_dev, int batch,
                                   int64_t max_total_rows, int H, int D, float scale, void* out, void* stream);
+
+/*
+ * Scratch of davet_step_attention and davet_view_attention: *bytes = 0 (each
+ * CTA builds the request schedule in its shared memory), for callers that
+ * size a workspace per call.  DAVET_ERR_INVALID_ARG for a negative size or a
+ * null `bytes`, DAVET_ERR_UNSUPPORTED for D other than 64 or 128.
+ */
+davet_status davet_step_attention_workspace(int batch, int64_t max_total_rows, int H, int D, size_t* bytes);
 
 /*
  * View blocks (host-only helpers and the build).  In the view-block layout a

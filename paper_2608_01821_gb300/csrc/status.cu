@@ -83,3 +83,27 @@ extern "C" davet_status davet_device_status(unsigned* flags, int clear) {
   if (w) return DAVET_ERR_DEVICE;
   return DAVET_OK;
 }
+
+extern "C" davet_status davet_sync_status(void* stream, unsigned* flags) {
+  using namespace davet;
+  unsigned* word = device_error_word();
+  if (word == nullptr) return DAVET_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  unsigned w = 0;
+  cudaError_t e = cudaMemcpyAsync(&w, word, sizeof w, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (flags) *flags = w;
+  if (w & DEV_ERR_TIMEOUT) return DAVET_ERR_TIMEOUT;
+  if (w) return DAVET_ERR_DEVICE;
+  return DAVET_OK;
+}
+
+extern "C" davet_status davet_step_attention_workspace(int batch, int64_t max_total_rows, int H, int D,
+                                                       size_t* bytes) {
+  if (!bytes || batch < 0 || max_total_rows < 0 || H < 1) return DAVET_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return DAVET_ERR_UNSUPPORTED;
+  *bytes = 0;  // the attention kernel keeps its schedule in shared memory
+  return DAVET_OK;
+}

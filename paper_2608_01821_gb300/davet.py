@@ -63,6 +63,8 @@ def _declare(lib):
         "davet_status_string": (ctypes.c_char_p, [_int]),
         "davet_last_cuda_error": (_int, []),
         "davet_device_status": (_int, [ctypes.POINTER(ctypes.c_uint), _int]),
+        "davet_sync_status": (_int, [_vp, ctypes.POINTER(ctypes.c_uint)]),
+        "davet_step_attention_workspace": (_int, [_int, _i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_pyramid_layout": (_int, [_int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_i64)]),
         "davet_build_pyramid": (_int, [_vp, _vp, _int, _int, _int, _int, _vp, _vp]),
         "davet_mixed_view_rows": (_int, [_int, _int, _int, _int, ctypes.POINTER(_int)]),
@@ -122,6 +124,18 @@ class Davet:
         flags = ctypes.c_uint(0)
         st = self.lib.davet_device_status(ctypes.byref(flags), 1 if clear else 0)
         return int(st), int(flags.value)
+
+    def davet_sync_status(self, stream=None) -> tuple[int, int]:
+        """(status, flags) of the device error word after the work on `stream`."""
+        flags = ctypes.c_uint(0)
+        st = self.lib.davet_sync_status(_stream(stream), ctypes.byref(flags))
+        return int(st), int(flags.value)
+
+    def davet_step_attention_workspace(self, batch: int, max_total_rows: int, H: int, D: int) -> int:
+        n = _sz(0)
+        self._check("davet_step_attention_workspace",
+                    self.lib.davet_step_attention_workspace(batch, max_total_rows, H, D, ctypes.byref(n)))
+        return int(n.value)
 
     def davet_pyramid_layout(self, grid: int, n_levels: int, n_tiles: int):
         side = (_int * n_levels)()

@@ -116,6 +116,11 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, mw, 1024, null) == INV
     assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, null, ws10, null) == INV
     assert lib.davet_build_views_merged(null, null, null, 0, 27, 4, 0, 0, 0, 128, 0, 32, null, null, 0, null) == 0
+    # attention scratch query: none needed
+    assert lib.davet_step_attention_workspace(4, 1000, 32, 128, ctypes.byref(sz0 := ctypes.c_size_t(7))) == 0
+    assert sz0.value == 0
+    assert lib.davet_step_attention_workspace(4, 1000, 32, 96, ctypes.byref(sz0)) == UNS
+    assert lib.davet_step_attention_workspace(-1, 1000, 32, 128, ctypes.byref(sz0)) == INV
     # full-layer kernels: GEMM shapes, epilogue codes, rotary arguments, norms, embedding
     sz = ctypes.c_size_t(0)
     assert lib.davet_linear(p, 10, 100, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null) == INV

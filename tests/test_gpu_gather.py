@@ -161,3 +161,24 @@ def test_mixed_index_without_a_mixed_view_is_flagged(davet):
     st, flags = davet.davet_device_status(clear=True)
     assert flags & 0x4
     assert list(cu.cpu().numpy()) == [0, 20, 20 + 49 + 20]
+
+
+def test_sync_status_reads_the_word_after_a_stream(davet):
+    """davet_sync_status waits for one stream and reports the word without
+    clearing it; davet_device_status then clears it."""
+    grid, levels, C = 27, 4, 64
+    tiles, prompt, resp = [1, 1], [10, 10], [10, 10]
+    d = setup(davet, tiles, prompt, resp, grid, levels, C, 8)
+    davet.davet_device_status(clear=True)
+    s = torch.cuda.Stream()
+    packed = torch.empty((800, C), dtype=torch.bfloat16, device="cuda")
+    cu = torch.empty(3, dtype=torch.int32, device="cuda")
+    lv = torch.zeros(2, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    davet.davet_gather_view(d["pyr_ptrs"], d["tiles"], d["text"], d["text_off"], d["prompt"], d["resp"], lv, 2,
+                            grid, levels, 0, 0, C, packed, cu, 800, s)
+    st, flags = davet.davet_sync_status(s)
+    assert st == 5 and flags & 0x2  # DAVET_ERR_DEVICE: the capacity bit
+    assert davet.davet_sync_status(s)[1] & 0x2  # not cleared
+    davet.davet_device_status(clear=True)
+    assert davet.davet_sync_status(s) == (0, 0)
