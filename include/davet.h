@@ -101,6 +101,15 @@ davet_status davet_device_status(unsigned* flags, int clear);
  */
 davet_status davet_sync_status(void* stream, unsigned* flags);
 
+/*
+ * Diagnostic of the failure path: one thread waits, with the bounded wait
+ * every kernel of the library uses, on an mbarrier that nothing signals.
+ * After the wait budget (about a second of SM clocks) it gives up, raises
+ * DAVET_DEV_TIMEOUT in the device error word and writes 1 to *gave_up_dev
+ * (int32, device); the context stays usable.  Nothing else uses it.
+ */
+davet_status davet_selftest_wait_timeout(int* gave_up_dev, void* stream);
+
 /* --------------------------------------------------------- evidence views */
 
 /*

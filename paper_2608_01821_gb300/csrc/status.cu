@@ -107,3 +107,29 @@ extern "C" davet_status davet_step_attention_workspace(int batch, int64_t max_to
   *bytes = 0;  // the attention kernel keeps its schedule in shared memory
   return DAVET_OK;
 }
+
+namespace davet {
+namespace {
+// One thread waits, with the library's bounded wait, on an mbarrier that
+// nothing signals; the wait gives up after its budget and raises the timeout
+// bit, the same path every producer/consumer wait of the kernels takes.
+__global__ void selftest_wait_kernel(unsigned* err, int* gave_up) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    const bool ok = mbar_wait(&bar, 0, err, nullptr);
+    *gave_up = ok ? 0 : 1;
+  }
+}
+}  // namespace
+}  // namespace davet
+
+extern "C" davet_status davet_selftest_wait_timeout(int* gave_up_dev, void* stream) {
+  using namespace davet;
+  if (!gave_up_dev) return DAVET_ERR_INVALID_ARG;
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
+  selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(err, gave_up_dev);
+  return check_launch();
+}

@@ -64,6 +64,7 @@ def _declare(lib):
         "davet_last_cuda_error": (_int, []),
         "davet_device_status": (_int, [ctypes.POINTER(ctypes.c_uint), _int]),
         "davet_sync_status": (_int, [_vp, ctypes.POINTER(ctypes.c_uint)]),
+        "davet_selftest_wait_timeout": (_int, [_vp, _vp]),
         "davet_step_attention_workspace": (_int, [_int, _i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_pyramid_layout": (_int, [_int, _int, _int, ctypes.POINTER(_int), ctypes.POINTER(_i64)]),
         "davet_build_pyramid": (_int, [_vp, _vp, _int, _int, _int, _int, _vp, _vp]),
@@ -130,6 +131,10 @@ class Davet:
         flags = ctypes.c_uint(0)
         st = self.lib.davet_sync_status(_stream(stream), ctypes.byref(flags))
         return int(st), int(flags.value)
+
+    def davet_selftest_wait_timeout(self, gave_up, stream=None):
+        self._check("davet_selftest_wait_timeout",
+                    self.lib.davet_selftest_wait_timeout(_ptr(gave_up), _stream(stream)))
 
     def davet_step_attention_workspace(self, batch: int, max_total_rows: int, H: int, D: int) -> int:
         n = _sz(0)

@@ -175,11 +175,13 @@ class Backbone:
     def step(self, t: int, stream=None, timed=None):
         w = self.w
         run = timed if timed is not None else (lambda kind, fn: fn())
+        torch.cuda.nvtx.range_push(f"backbone step {t}")
         self.forward(t, stream, timed)
         run("unmask", lambda: self.lib.davet_unmask_topk(self.logits, w.V, self.cu_resp, w.batch, self.R, w.k,
                                                          self.masked, self.tokens, self.argmax, self.conf,
                                                          self.committed[t], self.stats[t], self.workspace,
                                                          stream=stream))
+        torch.cuda.nvtx.range_pop()
 
     # ---------------------------------------------------- accounting (host)
     def gemm_flops(self, t: int) -> float:

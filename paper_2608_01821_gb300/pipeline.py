@@ -170,9 +170,20 @@ class Pipeline:
                                    self.workspace, self.workspace.numel(), stream)
 
     def step(self, t: int, logits, stream=None):
+        """One denoising step; NVTX ranges name its parts for profilers
+        (host-side marks: they cost nothing on a replayed CUDA graph)."""
+        nvtx = torch.cuda.nvtx
+        nvtx.range_push(f"davet step {t}")
         if self.fused:
+            nvtx.range_push("view_attention")
             self.view_attention(t, stream)
+            nvtx.range_pop()
         else:
+            nvtx.range_push("gather + attention")
             self.gather(t, stream)
             self.attention(stream)
+            nvtx.range_pop()
+        nvtx.range_push("unmask")
         self.unmask(t, logits, stream)
+        nvtx.range_pop()
+        nvtx.range_pop()
