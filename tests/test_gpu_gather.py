@@ -1,6 +1,8 @@
 """Parity of davet_gather_view (Eq. 5) with the oracle: packed rows and
 cu_seqlens must be bit-exact; device-side range and capacity problems set
-the device error word without writing out of bounds."""
+the device error word without writing out of bounds.  The gather copies
+rows, so its per-request buffers hold seeded rows in the pyramid layout
+(both sides get the same seeded values; none come from a kernel)."""
 import numpy as np
 import pytest
 import torch
@@ -17,13 +19,8 @@ def setup(davet, tiles, prompt, resp, grid, levels, C, seed):
     B = len(tiles)
     pyrs = []
     for b in range(B):
-        side, off = davet.davet_pyramid_layout(grid, levels, tiles[b])
-        feat = workloads.normal_bf16((max(tiles[b], 0), grid, grid, C), seed * 100 + b)
-        p = torch.empty((max(off[-1], 1), C), dtype=torch.bfloat16, device=dev)
-        if tiles[b] > 0:
-            p[: off[1]].copy_(feat.reshape(-1, C))
-            davet.davet_build_pyramid(p, p, tiles[b], grid, levels, C)
-        pyrs.append(p)
+        off = oracle.level_offsets(grid, levels, tiles[b])
+        pyrs.append(workloads.normal_bf16((max(off[-1], 1), C), seed * 100 + b).to(dev))
     n_text = sum(prompt) + sum(resp)
     text = workloads.normal_bf16((max(n_text, 1), C), seed * 7 + 1).to(dev)
     text_off = np.concatenate([[0], np.cumsum(np.add(prompt, resp))[:-1]]).astype(np.int64)

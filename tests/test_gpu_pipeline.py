@@ -32,16 +32,27 @@ def oracle_pyramids(w, feats):
     return out
 
 
-def oracle_gather_inputs(w, gpu_pyr):
-    """Per-request buffers for the oracle gather: the pyramid, followed by
-    the oracle's materialized mixed view when the workload has one."""
+def oracle_gather_inputs(w, pyr):
+    """Per-request buffers for the oracle gather: the oracle's pyramid (fp64
+    means rounded to bf16), followed by the oracle's mixed view of it when
+    the workload has one."""
     if not w.mixed:
-        return gpu_pyr, 0
+        return pyr, 0
     out = []
-    for b, p in enumerate(gpu_pyr):
+    for b, p in enumerate(pyr):
         mv = oracle.mixed_view(p, w.tiles[b], w.grid, w.n_levels, *w.mixed, w.C)
         out.append(np.concatenate([bits(p), mv]))
     return out, w.view_rows_per_tile(w.n_levels)
+
+
+def check_packed(gpu_rows, ref_bits):
+    """Packed rows against the oracle's: text rows are copies (bit-exact); a
+    view row is the GPU's rounding of the same pooled value, so it may sit one
+    bf16 step from the oracle's round-to-nearest (|x| < 8 here)."""
+    got = gpu_rows.float().cpu().double().numpy()
+    ref = torch.from_numpy(ref_bits.view(np.int16)).view(torch.bfloat16).double().numpy()
+    assert np.abs(got - ref).max() <= 2.0 ** -5
+    assert (bits(gpu_rows) == ref_bits).mean() > 0.999
 
 
 @pytest.mark.parametrize("name,fused", [("tiny", False), ("tiny_mixed", False), ("tiny", True),
@@ -50,14 +61,12 @@ def test_tiny_workload_every_step(davet, name, fused):
     w = workloads.make(name)
     pl, feats, text = make_pipeline(davet, w, fused)
     pyr_ref = oracle_pyramids(w, feats)
-    # the GPU pyramid rounds the same values: compare it bitwise through the
-    # rounding rule, then feed the GPU's own pyramid to the oracle gather so
-    # the later steps compare like with like
+    # the GPU pyramid rounds the same values: at most one bf16 step away
     gpu_pyr = [pl.pyramid_cpu(b) for b in range(w.batch)]
     for b in range(w.batch):
         diff = (gpu_pyr[b].float() - pyr_ref[b].float()).abs()
         assert float(diff.max()) <= 2 ** -7  # at most one bf16 step on |x| < 2
-    oracle_pyr, mrows = oracle_gather_inputs(w, gpu_pyr)
+    oracle_pyr, mrows = oracle_gather_inputs(w, pyr_ref)
     masked = np.ones(w.total_resp, np.uint8)
     tokens = np.full(w.total_resp, -1, np.int32)
     argmax = np.full(w.total_resp, -1, np.int32)
@@ -72,7 +81,7 @@ def test_tiny_workload_every_step(davet, name, fused):
         N = int(cu_ref[-1])
         assert list(pl.cu.cpu().numpy()) == list(cu_ref)
         if not fused:
-            assert np.array_equal(bits(pl.packed[:N]), packed_ref)
+            check_packed(pl.packed[:N], packed_ref)
         att_ref = oracle.attention(packed_ref, cu_ref, w.H, w.D, w.scale)
         max_abs, rel = attn_errors(bf16_to_f64(pl.attn_out[:N]), att_ref)
         assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (t, max_abs, rel)
@@ -97,7 +106,7 @@ def test_workload_sampled_steps(davet, name):
     w = workloads.make(name)
     pl, feats, text = make_pipeline(davet, w)
     gpu_pyr = [pl.pyramid_cpu(b) for b in range(w.batch)]
-    oracle_pyr, mrows = oracle_gather_inputs(w, gpu_pyr)
+    oracle_pyr, mrows = oracle_gather_inputs(w, oracle_pyramids(w, feats))
     # pyramid: one request, first tile, all levels against the oracle
     side = w.level_sides()
     ref_off = oracle.level_offsets(w.grid, w.n_levels, 1)
@@ -131,7 +140,7 @@ def test_workload_sampled_steps(davet, name):
                                            w.schedule[t], w.grid, w.n_levels, w.C, mixed_rows_per_tile=mrows)
         N = int(cu_ref[-1])
         assert list(pl.cu.cpu().numpy()) == list(cu_ref)
-        assert np.array_equal(bits(pl.packed[:N]), packed_ref)
+        check_packed(pl.packed[:N], packed_ref)
         rows, heads = [], []
         for b in range(w.batch):
             rows += list(rng.integers(cu_ref[b], cu_ref[b + 1], size=16))

@@ -14,6 +14,7 @@ import pytest
 import torch
 
 import oracle
+from helpers import check_topk
 from paper_2608_01821_gb300 import workloads
 from paper_2608_01821_gb300.pipeline import Pipeline
 
@@ -111,8 +112,10 @@ def test_step_matches_oracle_risk_budget_and_view(davet):
 @pytest.mark.parametrize("name,view_level", [("tiny", [2, 1, 0]), ("tiny_mixed", [2, 3, 0])])
 def test_closed_loop_tiny_workload(davet, name, view_level):
     """The policy picks every step's view on the device from the previous
-    step's unmasking statistics; the oracle policy fed the same statistics
-    picks the same views, and the mean budget stays below B (Eq. 4).  With
+    step's unmasking statistics; the oracle's own closed loop (its unmasking
+    of the same logits, then its policy) picks the same views, budgets within
+    1e-5 (fp32 statistics on the device), and the mean budget stays below B
+    (Eq. 4).  With
     the mixed view the three views are those of Sec. 4.3: coarse (level 2),
     mixed (view index 3) and high (level 0)."""
     w = workloads.make(name)
@@ -132,13 +135,29 @@ def test_closed_loop_tiny_workload(davet, name, view_level):
         pl.step(t, workloads.logits(w, t).cuda())
     torch.cuda.synchronize()
     assert davet.davet_device_status() == (0, 0)
+    # the oracle's own closed loop: its unmasking of the same logits gives the
+    # statistics of every step (a near tie in the commits, where either set is
+    # correct, continues from the GPU's set once it is checked to be valid)
     p = oracle.policy_profile(w.T, "late")
     rlo, rup = oracle.policy_envelope(p, B, rho, d)
-    stats = pl.stats.cpu().numpy().astype(np.float64)
     bud = budget.cpu().numpy()[:, 0]
+    lev = level.cpu().numpy()[:, 0]
+    masked = np.ones(w.total_resp, np.uint8)
+    tokens = np.full(w.total_resp, -1, np.int32)
+    argmax = np.full(w.total_resp, -1, np.int32)
+    prev_st = (0.0, 0.0)
     for t in range(w.T):
-        r = oracle.policy_risk(t + 1, alpha, stats[t - 1, 0, 0] if t else 0.0, stats[t - 1, 0, 1] if t else 0.0)
+        r = oracle.policy_risk(t + 1, alpha, *prev_st)
         want = oracle.policy_budget(rlo[t], rup[t], r)
-        assert abs(bud[t] - want) < 1e-12
-        assert level.cpu().numpy()[t, 0] == view_level[oracle.policy_view(want)]
+        # fp32 statistics on the device against fp64 here
+        assert abs(bud[t] - want) < 1e-5
+        if min(abs(want - 1 / 3), abs(want - 2 / 3)) > 1e-5:
+            assert lev[t] == view_level[oracle.policy_view(want)]
+        before = masked.copy()
+        conf, _, st = oracle.unmask(workloads.logits(w, t), w.V, w.cu_resp(), w.k, masked, tokens, argmax)
+        picks = [int(x) for x in pl.committed[t, 0].cpu().numpy() if x >= 0]
+        if check_topk(picks, {int(i): conf[i] for i in np.nonzero(before)[0]}, w.k):
+            masked[:] = 1
+            masked[[i for i in range(w.total_resp) if not before[i]] + picks] = 0
+        prev_st = (float(st[0, 0]), float(st[0, 1]))
     assert bud.mean() <= B + 1e-12

@@ -92,7 +92,17 @@ def test_view_blocks_hold_the_views_and_text(davet):
             nv = off[lvl + 1] - off[lvl]
             np.testing.assert_array_equal(buf[blk[lvl]:blk[lvl] + nv], pyr[off[lvl]:off[lvl + 1]])
             np.testing.assert_array_equal(buf[blk[lvl] + nv:blk[lvl + 1]], txt)
-        mv = oracle.mixed_view(pyr[: off[-1]], t, grid, levels, *mixed, d["C"])
+        # the mixed view as the unfused gather forms it from the same pyramid
+        # (its own parity with the oracle is held in the gather tests)
+        dev = torch.device("cuda")
+        i32 = lambda a: torch.tensor(a, dtype=torch.int32, device=dev)  # noqa: E731
+        mv_t = torch.empty((max(t * mrows, 1), d["C"]), dtype=torch.bfloat16, device=dev)
+        cu = torch.empty(2, dtype=torch.int32, device=dev)
+        davet.davet_gather_view(torch.tensor([d["pyrs"][b].data_ptr()], dtype=torch.int64, device=dev), i32([t]),
+                                d["text"], torch.zeros(1, dtype=torch.int64, device=dev), i32([0]), i32([0]),
+                                i32([levels]), 1, grid, levels, *mixed, d["C"], mv_t, cu, max(t * mrows, 1))
+        torch.cuda.synchronize()
+        mv = bits(mv_t)[: t * mrows]
         np.testing.assert_array_equal(buf[blk[levels]:blk[levels] + t * mrows], mv)
         np.testing.assert_array_equal(buf[blk[levels] + t * mrows:blk[levels + 1]], txt)
 
@@ -152,21 +162,24 @@ def test_fused_view_out_of_range_is_flagged(davet):
 
 def test_fused_pipeline_tiny_against_oracle(davet):
     """Every step of the tiny workloads through the fused pipeline call,
-    against the oracle's gather + attention on the GPU's own pyramid."""
+    against the oracle's own pyramid (fp64 means rounded to bf16), gather and
+    attention."""
     for name in ("tiny", "tiny_mixed"):
         w = workloads.make(name)
         pl = Pipeline(w, "cuda", davet, fused=True)
-        pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w))
+        feats = [workloads.features(w, b) for b in range(w.batch)]
+        pl.load_inputs(feats, workloads.text_rows(w))
         pl.build_pyramids()
         torch.cuda.synchronize()
-        gpu_pyr = [pl.pyramid_cpu(b) for b in range(w.batch)]
+        ora_pyr = [torch.from_numpy(oracle.pyramid(feats[b], w.tiles[b], w.grid, w.n_levels, w.C)).to(torch.bfloat16)
+                   for b in range(w.batch)]
         text = workloads.text_rows(w)
         if w.mixed:
             mrows = w.view_rows_per_tile(w.n_levels)
             pyrs = [np.concatenate([bits(p), oracle.mixed_view(p, w.tiles[b], w.grid, w.n_levels, *w.mixed, w.C)])
-                    for b, p in enumerate(gpu_pyr)]
+                    for b, p in enumerate(ora_pyr)]
         else:
-            mrows, pyrs = 0, gpu_pyr
+            mrows, pyrs = 0, ora_pyr
         for t in range(w.T):
             pl.view_attention(t)
             torch.cuda.synchronize()
