@@ -335,3 +335,17 @@ def test_split_workspace_too_small_runs_one_pass(davet):
     W = rand_bf16((N, K), 98, K ** -0.5).cuda()
     out = linear(davet, A, W, workspace=torch.empty(256, dtype=torch.uint8, device="cuda"))
     check_close(out, f64(A) @ f64(W).T, "fallback")
+
+
+@pytest.mark.parametrize("M,N", [(129, 256 * 76), (129, 4096), (257, 4096)])
+def test_pair_tiles_single_valid_row_in_the_odd_cta(davet, M, N):
+    """M = 129: the odd CTA of the pair holds one valid row (row 128); with
+    N = 4096 the K split path too (its reduction sees one row of that CTA)."""
+    K = 4096 if N == 4096 else 256
+    A = rand_bf16((M, K), 100 + M).cuda()
+    W = rand_bf16((N, K), 101, K ** -0.5).cuda()
+    nbytes = davet.davet_linear_workspace_bytes(M, K, N)
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device="cuda")
+    out = linear(davet, A, W, workspace=ws)
+    rows = np.array(sorted({0, 1, 127, 128, M - 1}))
+    check_close(out[torch.from_numpy(rows).cuda()], f64(A)[rows] @ f64(W).T, f"edge {M}x{K}x{N}")
