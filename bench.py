@@ -137,6 +137,7 @@ class ClockSampler:
 
 # ------------------------------------------------------------- our arm
 def run_ours(args, rank, world, local_rank):
+    import numpy as np
     import torch
 
     from paper_2608_01821_gb300 import davet, workloads
@@ -167,10 +168,32 @@ def run_ours(args, rank, world, local_rank):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(device=dev)
 
+    # closed-loop policy (Eq. 6-9 on the device): each step's view comes from
+    # the previous step's unmasking statistics
+    policy = getattr(args, "policy", False)
+    if policy:
+        orient = 0 if args.orientation == "early" else 1
+        view_level = [min(2, w.n_levels - 1), w.n_levels if w.mixed else 1, 0]
+        lo = torch.empty((w.batch, w.T), dtype=torch.float64, device=dev)
+        up = torch.empty_like(lo)
+        demand = torch.tensor(workloads.request_demands(w), dtype=torch.float64, device=dev)
+        budget = torch.zeros((w.T, w.batch), dtype=torch.float64, device=dev)
+
+    def policy_pass():
+        lib.davet_policy_envelope(w.T, orient, args.budget, args.rho, demand, w.batch, lo, up)
+
+    def policy_step(t):
+        lib.davet_policy_step(t, w.T, lo, up, pl.stats[t - 1] if t else None, w.batch, args.alpha, view_level,
+                              pl.schedule[t], budget[t])
+
     def one_pass():
         pl.reset_state()
         pl.build_pyramids()
+        if policy:
+            policy_pass()
         for t in range(w.T):
+            if policy:
+                policy_step(t)
             pl.step(t, pool[t % P])
 
     # eager warm-up (first calls resolve device addresses), then graph capture
@@ -218,7 +241,9 @@ def run_ours(args, rank, world, local_rank):
     comp = kernel_times(pl, w, pool, P, stream)
 
     # ---------------------------------------------------------- e2e
-    e2e = None if args.no_e2e else run_e2e(args, pl, w, dev, stream, world)
+    e2e = None if args.no_e2e else run_e2e(args, pl, w, dev, stream, world,
+                                           policy_pass=policy_pass if policy else None,
+                                           policy_step=policy_step if policy else None)
 
     out = None
     if rank == 0:
@@ -228,6 +253,8 @@ def run_ours(args, rank, world, local_rank):
         # pyramid; per step the fused view attention (or gather and attention)
         # and the two unmask kernels
         launches_per_pass = build_launches(w, pl.realizer, pl.fused) + w.T * (3 if pl.fused else 4)
+        if policy:
+            launches_per_pass += 1 + w.T  # envelope, then one policy step per denoising step
         akey = "view_attention" if pl.fused else "attention"
         attn_flops_launch = comp[akey]["flops"] / comp[akey]["launches"]
         attn_ms = comp[akey]["ms"] / comp[akey]["launches"]
@@ -284,6 +311,14 @@ def run_ours(args, rank, world, local_rank):
             "e2e": e2e,
             "wall_s_timed": round(wall, 3),
         }
+        if policy:
+            lv = pl.schedule.cpu().numpy()
+            views, counts = np.unique(lv, return_counts=True)
+            out["config"]["schedule"] = "closed-loop policy (Eq. 6-9 on the device)"
+            out["policy"] = {"orientation": args.orientation, "B": args.budget, "rho": args.rho, "alpha": args.alpha,
+                             "view_levels": view_level, "demand": workloads.request_demands(w),
+                             "mean_budget": round(float(budget.mean().item()), 4),
+                             "steps_per_view": {int(v): int(c) for v, c in zip(views, counts)}}
     return out
 
 
@@ -573,7 +608,7 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
     return out
 
 
-def run_e2e(args, pl, w, dev, stream, world):
+def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None):
     """Same pass through the C ABI with pinned host inputs: features and text
     copied in, every step's logits read from pinned host memory, committed
     tokens copied out.
@@ -620,7 +655,11 @@ def run_e2e(args, pl, w, dev, stream, world):
         pl.reset_state()
         pl.load_inputs(feats, text, non_blocking=True, scores=scores)
         pl.build_pyramids()
+        if policy_pass:
+            policy_pass()
         for t in range(w.T):
+            if policy_step:
+                policy_step(t)
             pl.step(t, host_logits[t % P])
         tokens_host.copy_(pl.tokens, non_blocking=True)
 
@@ -632,9 +671,13 @@ def run_e2e(args, pl, w, dev, stream, world):
         pl.reset_state()
         pl.load_inputs(feats, text, non_blocking=True, scores=scores)
         pl.build_pyramids()
+        if policy_pass:
+            policy_pass()
         for t in range(w.T):
             slot = t % NB
             stream.wait_event(ready[slot])
+            if policy_step:
+                policy_step(t)
             pl.step(t, dev_logits[slot])
             free[slot].record(stream)
             if t + NB < w.T:
@@ -916,6 +959,12 @@ def main(argv=None):
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)
+    ap.add_argument("--policy", action="store_true",
+                    help="choose every step's view with the closed-loop allocation policy on the device")
+    ap.add_argument("--orientation", choices=["early", "late"], default="early")
+    ap.add_argument("--budget", type=float, default=0.75, help="average budget B")
+    ap.add_argument("--rho", type=float, default=0.20)
+    ap.add_argument("--alpha", type=float, default=1.0)
     ap.add_argument("--model", choices=["core", "full"], default="core",
                     help="core: the step-conditioning path (attention core); full: every step runs --layers "
                          "synthetic-weight backbone layers and the LM head")

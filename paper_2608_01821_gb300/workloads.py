@@ -281,6 +281,18 @@ def text_rows(w: Workload):
     return torch.cat(parts, 0)
 
 
+# Operation demand prior d(o) of the five operation categories (Table A:
+# lexical readout, numerical reasoning, entity grounding, binary decision,
+# general understanding).  The query parser that assigns a category is not
+# part of this path; requests take the categories in turn.
+DEMAND_PRIOR = (1.000, 0.941, 0.824, 0.647, 0.529)
+
+
+def request_demands(w: Workload) -> list[float]:
+    """d(o) of every request (categories assigned in turn, request b -> b mod 5)."""
+    return [DEMAND_PRIOR[b % len(DEMAND_PRIOR)] for b in range(w.batch)]
+
+
 def token_scores(w: Workload, b: int):
     """Importance score of every visual token of request b for the pruning
     realizer (the paper leaves the score open): fp32 [tiles, G*G] ~ N(0,1)."""
