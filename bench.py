@@ -147,6 +147,8 @@ def run_ours(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     lib = davet.load()
     w = workloads.make(args.config)
+    if args.schedule != "workload":
+        workloads.set_static_view(w, args.schedule)
     if rank > 0:
         w.seed = w.seed + 1000 * rank  # each replica gets its own batch
     realizer = getattr(args, "realizer", "pool")
@@ -173,7 +175,7 @@ def run_ours(args, rank, world, local_rank):
     policy = getattr(args, "policy", False)
     if policy:
         orient = 0 if args.orientation == "early" else 1
-        view_level = [min(2, w.n_levels - 1), w.n_levels if w.mixed else 1, 0]
+        view_level = workloads.policy_view_levels(w)
         lo = torch.empty((w.batch, w.T), dtype=torch.float64, device=dev)
         up = torch.empty_like(lo)
         demand = torch.tensor(workloads.request_demands(w), dtype=torch.float64, device=dev)
@@ -312,13 +314,10 @@ def run_ours(args, rank, world, local_rank):
             "wall_s_timed": round(wall, 3),
         }
         if policy:
-            lv = pl.schedule.cpu().numpy()
-            views, counts = np.unique(lv, return_counts=True)
             out["config"]["schedule"] = "closed-loop policy (Eq. 6-9 on the device)"
-            out["policy"] = {"orientation": args.orientation, "B": args.budget, "rho": args.rho, "alpha": args.alpha,
-                             "view_levels": view_level, "demand": workloads.request_demands(w),
-                             "mean_budget": round(float(budget.mean().item()), 4),
-                             "steps_per_view": {int(v): int(c) for v, c in zip(views, counts)}}
+            out["policy"] = policy_summary(args, w, pl.schedule.cpu().numpy(), budget)
+        elif args.schedule != "workload":
+            out["config"]["schedule"] = f"static {args.schedule} view"
     return out
 
 
@@ -335,9 +334,13 @@ def run_backbone(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     lib = davet.load()
     w = workloads.make(args.config)
+    if args.schedule != "workload":
+        workloads.set_static_view(w, args.schedule)
     if rank > 0:
         w.seed = w.seed + 1000 * rank
     bb = Backbone(w, args.layers, dev, lib)
+    if args.policy:
+        bb.use_policy(args.orientation, args.budget, args.rho, args.alpha)
     feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C),
                                    workloads.derive_seed(w.seed, workloads.KIND_FEAT, b)) for b in range(w.batch)]
     prompts = [workloads.normal_bf16((w.prompt[b], bb.C), workloads.derive_seed(w.seed, workloads.KIND_TEXT, b))
@@ -347,7 +350,7 @@ def run_backbone(args, rank, world, local_rank):
     stream = torch.cuda.Stream(device=dev)
 
     def one_pass(timed=None):
-        bb.reset_state()
+        bb.begin_pass()
         bb.build_pyramids()
         for t in range(w.T):
             bb.step(t, timed=timed)
@@ -404,7 +407,10 @@ def run_backbone(args, rank, world, local_rank):
     for kind, a, b in calls:
         kinds[kind] = kinds.get(kind, 0.0) + a.elapsed_time(b)
     n_gemm = sum(1 for k, _, _ in calls if k == "gemm")
-    gemm_flops = sum(bb.gemm_flops(t) for t in range(w.T))
+    # the views every step ran (the policy's choices are read back after the pass)
+    sched = bb.schedule.cpu().numpy()
+    step_rows = [bb.rows_of(sched[t]) for t in range(w.T)]
+    gemm_flops = sum(bb.gemm_flops(t, step_rows[t]) for t in range(w.T))
 
     # end to end: visual hidden states and prompt rows from pinned host memory,
     # committed tokens back to the host, every pass
@@ -461,6 +467,9 @@ def run_backbone(args, rank, world, local_rank):
             "parallelism": f"replicas x{world} (independent requests)",
             "timing": "CUDA events per pass on the launching stream; one CUDA graph per pass",
             "l2": f"{L2_FLUSH_BYTES >> 20} MiB write between timed passes (not timed); weights stream from HBM",
+            "schedule": ("closed-loop policy (Eq. 6-9 on the device)" if args.policy else
+                         "workload level schedule" if args.schedule == "workload" else f"static {args.schedule} view"),
+            "mean_rows_per_step": round(sum(step_rows) / w.T, 2),
         },
         "components": {k: {"ms_per_pass": round(v, 3), "share": round(v / sum(kinds.values()), 4)}
                        for k, v in kinds.items()},
@@ -476,9 +485,23 @@ def run_backbone(args, rank, world, local_rank):
             "flops_per_launch": gemm_flops / max(n_gemm, 1),
         },
         "clocks": clocks.summary(),
-        "gpu_launches": (sum(1 for x in w.tiles if x > 0) + sum(bb.launches(t) for t in range(w.T))) * args.steps,
+        "gpu_launches": (sum(1 for x in w.tiles if x > 0) + sum(bb.launches(t) for t in range(w.T))
+                         + (1 if args.policy else 0)) * args.steps,
         "e2e": e2e,
+        **({"policy": policy_summary(args, w, sched, bb.budget)} if args.policy else {}),
     }
+
+
+def policy_summary(args, w, sched, budget):
+    """The policy's settings and what it chose over one pass."""
+    import numpy as np
+
+    from paper_2608_01821_gb300 import workloads
+    views, counts = np.unique(sched, return_counts=True)
+    return {"orientation": args.orientation, "B": args.budget, "rho": args.rho, "alpha": args.alpha,
+            "view_levels": workloads.policy_view_levels(w), "demand": workloads.request_demands(w),
+            "mean_budget": round(float(budget.mean().item()), 4),
+            "steps_per_view": {int(v): int(c) for v, c in zip(views, counts)}}
 
 
 def merge_round_count(grid: int, n_levels: int) -> int:
@@ -961,6 +984,8 @@ def main(argv=None):
     ap.add_argument("--profile-step", type=int, default=0)
     ap.add_argument("--policy", action="store_true",
                     help="choose every step's view with the closed-loop allocation policy on the device")
+    ap.add_argument("--schedule", choices=["workload", "high", "mid", "low"], default="workload",
+                    help="the level schedule without --policy: the workload's own, or one static view for every step")
     ap.add_argument("--orientation", choices=["early", "late"], default="early")
     ap.add_argument("--budget", type=float, default=0.75, help="average budget B")
     ap.add_argument("--rho", type=float, default=0.20)

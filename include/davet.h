@@ -516,6 +516,13 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  *            before the epilogue; otherwise one pass over K per tile.  A
  *            workspace must not be shared by calls that may run at the same
  *            time.
+ *   rows_dev device int32, nullable: the row count to compute, read on the
+ *            device when the kernels start (after the previous work on
+ *            `stream`), clamped to [0, M]; rows from there on are neither read
+ *            for the epilogue nor written.  M is then the capacity: A, out
+ *            and the residual hold M rows, and the tiling and workspace are
+ *            chosen for M.  Lets a captured step run a row count that
+ *            earlier kernels decide (the allocation policy's views).
  * One persistent kernel on `stream` (with a split: a second kernel adds the
  * slices and applies the epilogue).  M > 128 runs on CTA pairs (clusters of
  * two CTAs on two SMs).
@@ -530,7 +537,9 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  * sums, bf16 out); x, out bf16 [M][C], gamma bf16 [C], C % 8 == 0.  With
  * cu_resp (int32 [batch+1], the answer-row boundaries) the M = total answer
  * rows are the last cu_resp[b+1] - cu_resp[b] rows of each request's rows
- * (cu_seqlens) and are written packed, in request order.
+ * (cu_seqlens) and are written packed, in request order.  rows_dev
+ * (device int32, nullable): the row count, read on the device and clamped to
+ * [0, M], as in davet_linear.
  *
  * davet_embed_answers -- writes the answer rows of the packed step input from
  * an embedding table: row cu_seqlens[b+1] - n_b + i (n_b answer rows of
@@ -541,11 +550,12 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
 davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                           const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols, int head_dim,
                           const void* rope_table, int max_pos, void* workspace, size_t workspace_bytes,
-                          void* stream);
+                          const int32_t* rows_dev, void* stream);
 davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, size_t* bytes);
 davet_status davet_rope_table(int max_pos, int head_dim, double theta, void* table, void* stream);
 davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
-                           const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, void* stream);
+                           const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, const int32_t* rows_dev,
+                           void* stream);
 davet_status davet_embed_answers(const void* table, int V, int C, const int32_t* tokens, int mask_id,
                                  const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, int64_t total_resp,
                                  void* x, void* stream);

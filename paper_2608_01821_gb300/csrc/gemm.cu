@@ -67,7 +67,19 @@ struct Params {
   int split;
   int kb_per;
   float* part;
+  // nullable: the row count on the device (at most M), read after the
+  // previous kernel finished; rows from there on are neither computed nor stored
+  const int32_t* rows_dev;
 };
+
+// The launch's row count: M, or the smaller count on the device.
+__device__ __forceinline__ void device_rows(Params& p) {
+  if (p.rows_dev) {
+    const long long m = *p.rows_dev;
+    p.M = m < 0 ? 0 : (m < p.M ? m : p.M);
+    p.tiles_m = static_cast<int>((p.M + BM - 1) / BM);
+  }
+}
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1) {
   asm volatile(
@@ -187,8 +199,9 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p) {
+    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p0) {
   extern __shared__ uint8_t smem_raw[];
+  Params p = p0;
   Smem& s = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   volatile int* abort_flag = &s.abort;
@@ -216,6 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_launch_dependents();
   pdl_wait();  // A (and the residual) come from the previous kernel
+  device_rows(p);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -374,8 +388,9 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm2_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p) {
+    gemm2_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p0) {
   extern __shared__ uint8_t smem_raw[];
+  Params p = p0;
   Smem2& s = *reinterpret_cast<Smem2*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   volatile int* abort_flag = &s.abort;
@@ -407,6 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_launch_dependents();
   pdl_wait();
+  device_rows(p);  // both CTAs of the pair read the same count
   tc_fence_before();
   cluster_sync_all();  // barriers initialized and TMEM allocated in both CTAs
   tc_fence_after();
@@ -544,9 +560,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 // per (row, 256-column block), lane l holding columns [8l, 8l + 8) (coalesced
 // 1 KB per slice); the gated MLP pairs lane l with lane l + 16 (gate, up),
 // the rotary embedding lane l with lane l ^ (D/16) (columns d, d + D/2).
-__global__ void __launch_bounds__(256) split_reduce_kernel(Params p) {
+__global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
   pdl_launch_dependents();
   pdl_wait();
+  Params p = p0;
+  device_rows(p);
   const int lane = threadIdx.x & 31;
   const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
@@ -638,9 +656,14 @@ template <bool ANSWERS>
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const uint16_t* __restrict__ x, long long M, int C,
                                                       const uint16_t* __restrict__ gamma, float eps,
                                                       uint16_t* __restrict__ out, const int32_t* cu,
-                                                      const int32_t* cu_resp, int batch) {
+                                                      const int32_t* cu_resp, int batch,
+                                                      const int32_t* __restrict__ rows_dev) {
   pdl_launch_dependents();
   pdl_wait();
+  if (rows_dev) {
+    const long long m = *rows_dev;
+    M = m < 0 ? 0 : (m < M ? m : M);
+  }
   const int lane = threadIdx.x & 31;
   const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
@@ -796,7 +819,7 @@ extern "C" davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, si
 extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                                      const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols,
                                      int head_dim, const void* rope_table, int max_pos, void* workspace,
-                                     size_t workspace_bytes, void* stream) {
+                                     size_t workspace_bytes, const int32_t* rows_dev, void* stream) {
   if (M < 0 || M > 0x7fffffffLL || K < BK || K % BK != 0 || N < BN || N % BN != 0) return DAVET_ERR_INVALID_ARG;
   if (epilogue < EPI_STORE || epilogue > EPI_ROPE) return DAVET_ERR_INVALID_ARG;
   if (M == 0) return DAVET_OK;
@@ -851,6 +874,7 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   p.split = 1;
   p.kb_per = K / BK;
   p.part = nullptr;
+  p.rows_dev = rows_dev;
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -909,7 +933,8 @@ extern "C" davet_status davet_rope_table(int max_pos, int head_dim, double theta
 }
 
 extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
-                                      const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, void* stream) {
+                                      const int32_t* cu_seqlens, const int32_t* cu_resp, int batch,
+                                      const int32_t* rows_dev, void* stream) {
   if (M < 0 || C < 8 || C % 8 != 0 || !(eps >= 0.0f)) return DAVET_ERR_INVALID_ARG;
   if (M == 0) return DAVET_OK;
   if (!x || !gamma || !out || !aligned16(x) || !aligned16(gamma) || !aligned16(out)) return DAVET_ERR_INVALID_ARG;
@@ -922,9 +947,9 @@ extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const voi
   uint16_t* os = static_cast<uint16_t*>(out);
   const cudaError_t e =
       answers ? launch(rmsnorm_kernel<true>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs, eps,
-                       os, cu_seqlens, cu_resp, batch)
+                       os, cu_seqlens, cu_resp, batch, rows_dev)
               : launch(rmsnorm_kernel<false>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs,
-                       eps, os, cu_seqlens, cu_resp, batch);
+                       eps, os, cu_seqlens, cu_resp, batch, rows_dev);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

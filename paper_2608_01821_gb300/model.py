@@ -10,6 +10,14 @@ epilogues, davet_step_attention), the final normalization of the answer rows
 and the LM head give the logits that davet_unmask_topk commits from.  The
 rows carry hidden states of width C = H * D; the MLP width is 3C.
 
+Each step's view comes either from the workload's schedule (known on the
+host, so every launch is sized to the step's rows) or, after use_policy(),
+from the allocation policy (Eq. 6-9) on the device, fed by the previous
+step's unmasking statistics.  Then the row count exists only on the device
+(cu_seqlens[batch] after the gather): the norms and projections are launched
+for the largest view and read the count when they start, so a captured pass
+runs whatever views the policy picks without a host round trip.
+
 Weights are random (no checkpoint is available): each matrix ~ N(0, 1/fan_in),
 normalization gains ~ 1 + N(0, 0.1^2), drawn on the device from torch
 generators seeded per tensor.  This module performs no arithmetic of its own.
@@ -19,7 +27,7 @@ from __future__ import annotations
 import torch
 
 from . import davet as _davet
-from .workloads import Workload, derive_seed
+from .workloads import Workload, derive_seed, policy_view_levels, request_demands
 
 KIND_WEIGHT = 16
 ROPE_THETA = 500000.0
@@ -106,9 +114,23 @@ class Backbone:
         self.workspace = torch.zeros(max(ws, 256), dtype=torch.uint8, device=dev)
         # scratch of the projections' K split (steps with few rows)
         shapes = [(C, 3 * self.HD), (self.HD, C), (C, 2 * F), (F, C), (C, w.V)]
-        rows = {self.rows(t) for t in range(w.T)} | {R}
+        rows = {self.rows(t) for t in range(w.T)} | {R, self.max_rows}
         gw = max(self.lib.davet_linear_workspace_bytes(m, k, n) for k, n in shapes for m in rows)
         self.gemm_ws = torch.empty(max(gw, 256), dtype=torch.uint8, device=dev)
+        self.policy = None
+
+    def use_policy(self, orientation: str = "early", B: float = 0.75, rho: float = 0.2, alpha: float = 1.0):
+        """Choose every step's view with the closed-loop allocation policy:
+        the budget envelope (Eq. 6-7) at the start of each pass, the view of
+        step t from step t-1's unmasking statistics (Eq. 8-9)."""
+        if orientation not in ("early", "late"):
+            raise ValueError("orientation is 'early' or 'late'")
+        w, dev = self.w, self.dev
+        self.policy = dict(orientation=orientation, B=B, rho=rho, alpha=alpha, view_levels=policy_view_levels(w))
+        self.lo = torch.empty((w.batch, w.T), dtype=torch.float64, device=dev)
+        self.up = torch.empty_like(self.lo)
+        self.demand = torch.tensor(request_demands(w), dtype=torch.float64, device=dev)
+        self.budget = torch.zeros((w.T, w.batch), dtype=torch.float64, device=dev)
 
     # -------------------------------------------------------------- inputs
     def load_inputs(self, feats, prompts, non_blocking=False):
@@ -128,6 +150,14 @@ class Backbone:
         self.tokens.fill_(-1)
         self.argmax.fill_(-1)
 
+    def begin_pass(self, stream=None):
+        """Fresh answer state; with the policy, the pass's budget envelope."""
+        self.reset_state()
+        if self.policy:
+            pol = self.policy
+            self.lib.davet_policy_envelope(self.w.T, 0 if pol["orientation"] == "early" else 1, pol["B"], pol["rho"],
+                                           self.demand, self.w.batch, self.lo, self.up, stream)
+
     def build_pyramids(self, stream=None):
         w = self.w
         for b in range(w.batch):
@@ -136,8 +166,12 @@ class Backbone:
 
     # ---------------------------------------------------------------- path
     def rows(self, t: int) -> int:
-        """Rows of step t's packed sequence (the schedule is known on the host)."""
+        """Rows of step t's packed sequence under the workload's schedule."""
         return int(sum(self.w.step_lengths(t)))
+
+    def rows_of(self, levels) -> int:
+        """Rows of a step whose requests take the views `levels`."""
+        return int(sum(self.w.seq_len(b, int(v)) for b, v in enumerate(levels)))
 
     def forward(self, t: int, stream=None, timed=None):
         """Step t's input rows and every layer; leaves the answer logits.
@@ -145,28 +179,31 @@ class Backbone:
         timing); kind is "input", "norm", "gemm" or "attention"."""
         w, lib = self.w, self.lib
         run = timed if timed is not None else (lambda kind, fn: fn())
-        N = self.rows(t)
+        if self.policy:
+            N, nd = self.max_rows, self.cu[w.batch:]  # the count the gather writes
+        else:
+            N, nd = self.rows(t), None
         C, HD, F = self.C, self.HD, self.F
         ws = self.gemm_ws
         run("input", lambda: lib.davet_gather_view(self.pyr_ptrs, self.tiles, self.text, self.text_off, self.prompt,
-                                                   self.resp, self.schedule[t], w.batch, w.grid, w.n_levels, 0, 0, C,
-                                                   self.x, self.cu, self.max_rows, stream))
+                                                   self.resp, self.schedule[t], w.batch, w.grid, w.n_levels,
+                                                   *w.mixed_args, C, self.x, self.cu, self.max_rows, stream))
         run("input", lambda: lib.davet_embed_answers(self.emb, w.V, C, self.tokens, self.mask_id, self.cu,
                                                      self.cu_resp, w.batch, self.R, self.x, stream))
         for p in self.layers:
-            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g1"], RMS_EPS, self.h, stream=stream))
+            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g1"], RMS_EPS, self.h, rows_dev=nd, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wqkv"], 3 * HD, self.qkv, lib.EPI_ROPE, None,
                                                  self.cu, w.batch, 2 * HD, w.D, self.rope, self.max_pos, ws,
-                                                 stream=stream))
+                                                 rows_dev=nd, stream=stream))
             run("attention", lambda: lib.davet_step_attention(self.qkv, self.cu, w.batch, self.max_rows, w.H, w.D,
                                                               w.scale, self.att, stream))
             run("gemm", lambda: lib.davet_linear(self.att, N, HD, p["wo"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 workspace=ws, stream=stream))
-            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g2"], RMS_EPS, self.h, stream=stream))
+                                                 workspace=ws, rows_dev=nd, stream=stream))
+            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g2"], RMS_EPS, self.h, rows_dev=nd, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wgu"], 2 * F, self.a, lib.EPI_SWIGLU,
-                                                 workspace=ws, stream=stream))
+                                                 workspace=ws, rows_dev=nd, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.a, N, F, p["wd"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 workspace=ws, stream=stream))
+                                                 workspace=ws, rows_dev=nd, stream=stream))
         run("norm", lambda: lib.davet_rmsnorm(self.x, self.R, C, self.gf, RMS_EPS, self.xa, self.cu, self.cu_resp,
                                               w.batch, stream))
         run("gemm", lambda: lib.davet_linear(self.xa, self.R, C, self.wlm, w.V, self.logits, workspace=ws,
@@ -176,6 +213,12 @@ class Backbone:
         w = self.w
         run = timed if timed is not None else (lambda kind, fn: fn())
         torch.cuda.nvtx.range_push(f"backbone step {t}")
+        if self.policy:
+            pol = self.policy
+            run("policy", lambda: self.lib.davet_policy_step(t, w.T, self.lo, self.up,
+                                                             self.stats[t - 1] if t else None, w.batch, pol["alpha"],
+                                                             pol["view_levels"], self.schedule[t], self.budget[t],
+                                                             stream))
         self.forward(t, stream, timed)
         run("unmask", lambda: self.lib.davet_unmask_topk(self.logits, w.V, self.cu_resp, w.batch, self.R, w.k,
                                                          self.masked, self.tokens, self.argmax, self.conf,
@@ -184,16 +227,17 @@ class Backbone:
         torch.cuda.nvtx.range_pop()
 
     # ---------------------------------------------------- accounting (host)
-    def gemm_flops(self, t: int) -> float:
-        """Tensor-core FLOPs of step t's projections and LM head."""
-        N = self.rows(t)
+    def gemm_flops(self, t: int, N: int | None = None) -> float:
+        """Tensor-core FLOPs of step t's projections and LM head (N rows;
+        default: the workload's schedule)."""
+        N = self.rows(t) if N is None else N
         C, HD, F = self.C, self.HD, self.F
         per_layer = 2.0 * N * C * (3 * HD) + 2.0 * N * HD * C + 2.0 * N * C * (2 * F) + 2.0 * N * F * C
         return self.L * per_layer + 2.0 * self.R * C * self.w.V
 
     def gemm_launches(self, t: int) -> int:
         """Kernels of step t's projections: one per GEMM, two where K is split."""
-        N = self.rows(t)
+        N = self.max_rows if self.policy else self.rows(t)
         C, HD, F = self.C, self.HD, self.F
 
         def k(m, kk, n):
@@ -204,5 +248,6 @@ class Backbone:
 
     def launches(self, t: int) -> int:
         """Kernels of step t: gather, embedding, per layer two norms and the
-        attention, the projections, the final norm, two unmask kernels."""
-        return 2 + 3 * self.L + self.gemm_launches(t) + 1 + 2
+        attention, the projections, the final norm, two unmask kernels; with
+        the policy, its step kernel."""
+        return 2 + 3 * self.L + self.gemm_launches(t) + 1 + 2 + (1 if self.policy else 0)

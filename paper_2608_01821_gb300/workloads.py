@@ -293,6 +293,20 @@ def request_demands(w: Workload) -> list[float]:
     return [DEMAND_PRIOR[b % len(DEMAND_PRIOR)] for b in range(w.batch)]
 
 
+def set_static_view(w: Workload, which: str) -> None:
+    """Replace the level schedule by one view for every step and request:
+    'high' (level 0), 'mid' or 'low' (the policy's other two views)."""
+    lv = dict(zip(("low", "mid", "high"), policy_view_levels(w)))[which]
+    w.schedule = np.full_like(w.schedule, lv)
+
+
+def policy_view_levels(w: Workload) -> list[int]:
+    """The views the allocation policy picks among, as the gather numbers
+    them: [low, mid, high] = [pyramid level 2 (or the coarsest), the mixed
+    view (or level 1), level 0]."""
+    return [min(2, w.n_levels - 1), w.n_levels if w.mixed else 1, 0]
+
+
 def token_scores(w: Workload, b: int):
     """Importance score of every visual token of request b for the pruning
     realizer (the paper leaves the score open): fp32 [tiles, G*G] ~ N(0,1)."""

@@ -115,7 +115,7 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_build_views_merged(p, p, null, 1, 27, 4, 0, 0, 0, 128, 4, 32, null, mw, ws10, null) == INV
     assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, mw, 1024, null) == INV
     assert lib.davet_build_views_merged(p, p, null, 10, 27, 4, 0, 0, 0, 128, 0, 32, null, null, ws10, null) == INV
-    assert lib.davet_build_views_merged(null, null, null, 0, 27, 4, 0, 0, 0, 128, 0, 32, null, null, 0, null) == 0
+    assert lib.davet_build_views_merged(null, null, null, 0, 27, 4, 0, 0, 0, 128, 0, 32, null, null, 0, null, null) == 0
     # attention scratch query: none needed
     assert lib.davet_step_attention_workspace(4, 1000, 32, 128, ctypes.byref(sz0 := ctypes.c_size_t(7))) == 0
     assert sz0.value == 0
@@ -123,19 +123,19 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_step_attention_workspace(-1, 1000, 32, 128, ctypes.byref(sz0)) == INV
     # full-layer kernels: GEMM shapes, epilogue codes, rotary arguments, norms, embedding
     sz = ctypes.c_size_t(0)
-    assert lib.davet_linear(p, 10, 100, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 100, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 256, p, 7, null, null, 0, 0, 128, null, 0, null, 0, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 256, p, 1, null, null, 0, 0, 128, null, 0, null, 0, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 512, 96, p, 16, null, 0, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 300, 128, p, 16, null, 0, null) == INV
-    assert lib.davet_linear(p, -1, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null) == INV
-    assert lib.davet_linear(null, 0, 128, null, 256, null, 0, null, null, 0, 0, 128, null, 0, null, 0, null) == 0
+    assert lib.davet_linear(p, 10, 100, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 100, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 7, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 1, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 512, 96, p, 16, null, 0, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 300, 128, p, 16, null, 0, null, null) == INV
+    assert lib.davet_linear(p, -1, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
+    assert lib.davet_linear(null, 0, 128, null, 256, null, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == 0
     assert lib.davet_linear_workspace_bytes(10, 100, 256, ctypes.byref(sz)) == INV
     assert lib.davet_rope_table(16, 96, ctypes.c_double(1e4), p, null) == INV
     assert lib.davet_rope_table(16, 128, ctypes.c_double(1.0), p, null) == INV
-    assert lib.davet_rmsnorm(p, 10, 12, p, ctypes.c_float(1e-5), p, null, null, 0, null) == INV
-    assert lib.davet_rmsnorm(p, 10, 16, p, ctypes.c_float(1e-5), p, null, p, 0, null) == INV
+    assert lib.davet_rmsnorm(p, 10, 12, p, ctypes.c_float(1e-5), p, null, null, 0, null, null) == INV
+    assert lib.davet_rmsnorm(p, 10, 16, p, ctypes.c_float(1e-5), p, null, p, 0, null, null) == INV
     assert lib.davet_embed_answers(p, 100, 16, p, 100, p, p, 1, 5, p, null) == INV
     assert lib.davet_embed_answers(p, 100, 16, p, 3, p, p, 1, 0, p, null) == 0
     # gather: bad levels count, batch too large

@@ -49,10 +49,16 @@ def layer_weights(p, F):
                 wg=gu[:, 0].reshape(F, C), wu=gu[:, 1].reshape(F, C), wd=f64(p["wd"]))
 
 
-@pytest.mark.parametrize("t", [0, 2, 5])
-def test_tiny_two_layer_step_logits(davet, t):
+@pytest.mark.parametrize("t,device_rows", [(0, False), (2, False), (5, False), (2, True), (5, True)])
+def test_tiny_two_layer_step_logits(davet, t, device_rows):
+    """device_rows: the policy's launch mode, every kernel launched for the
+    largest view and reading the step's row count on the device (the step's
+    view still comes from the workload's schedule here)."""
     w = workloads.make("tiny")
     bb = Backbone(w, 2, lib=davet)
+    if device_rows:
+        bb.use_policy()
+        assert bb.rows(t) < bb.max_rows
     feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C), 100 + b) for b in range(w.batch)]
     prompts = [workloads.normal_bf16((w.prompt[b], bb.C), 200 + b) for b in range(w.batch)]
     bb.load_inputs(feats, prompts)
@@ -97,3 +103,30 @@ def test_closed_loop_commits_every_position(davet):
     assert int(bb.masked.sum()) == w.total_resp - w.T * w.k
     tok = bb.tokens.cpu().numpy()
     assert ((tok[flat] >= 0) & (tok[flat] < w.V)).all()
+
+
+def test_policy_closed_loop(davet):
+    """The allocation policy picks every step's view on the device from the
+    previous step's statistics; the steps run the rows of the views it picked
+    (cu_seqlens of the last step) and the loop commits every position."""
+    w = workloads.make("tiny")
+    bb = Backbone(w, 1, lib=davet)
+    bb.use_policy("early", 0.75, 0.2, 1.0)
+    feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C), 500 + b) for b in range(w.batch)]
+    prompts = [workloads.normal_bf16((w.prompt[b], bb.C), 600 + b) for b in range(w.batch)]
+    bb.load_inputs(feats, prompts)
+    bb.begin_pass()
+    bb.build_pyramids()
+    for t in range(w.T):
+        bb.step(t)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    sched = bb.schedule.cpu().numpy()
+    assert set(np.unique(sched).tolist()) <= set(workloads.policy_view_levels(w))
+    cu = bb.cu.cpu().numpy()
+    assert int(cu[-1]) == bb.rows_of(sched[-1])
+    assert [int(cu[b + 1] - cu[b]) for b in range(w.batch)] == [w.seq_len(b, int(v)) for b, v in enumerate(sched[-1])]
+    committed = bb.committed.cpu().numpy().reshape(-1)
+    assert len(set(committed.tolist())) == len(committed) == w.T * w.k
+    budget = bb.budget.cpu().numpy()
+    assert ((budget >= 0) & (budget <= 1)).all()

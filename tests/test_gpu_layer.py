@@ -349,3 +349,88 @@ def test_pair_tiles_single_valid_row_in_the_odd_cta(davet, M, N):
     out = linear(davet, A, W, workspace=ws)
     rows = np.array(sorted({0, 1, 127, 128, M - 1}))
     check_close(out[torch.from_numpy(rows).cuda()], f64(A)[rows] @ f64(W).T, f"edge {M}x{K}x{N}")
+
+
+# ------------------------------------------- row count read on the device
+# rows_dev: the kernels are launched for a capacity of M rows and read the
+# row count m from device memory when they start; rows from m on keep their
+# contents, rows below m match the oracle (and the launch without rows_dev).
+@pytest.mark.parametrize("M,m,K,N,epi", [(100, 37, 256, 512, 0),      # one-CTA tiles
+                                         (700, 300, 512, 1024, 1),    # CTA pairs, residual
+                                         (700, 129, 512, 1024, 2),    # pairs, one valid row in the odd CTA
+                                         (700, 0, 256, 512, 0),       # nothing to compute
+                                         (241, 97, 4096, 4096, 1),    # pairs with the K split
+                                         (241, 241, 1024, 2048, 2),   # K split, every row
+                                         (500, 900, 256, 256, 0)])    # a count above M is clamped to M
+def test_linear_device_row_count(davet, M, m, K, N, epi):
+    A = rand_bf16((M, K), 110 + M).cuda()
+    W = rand_bf16((N, K), 111 + N, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 112).cuda() if epi == 1 else None
+    nbytes = davet.davet_linear_workspace_bytes(M, K, N)
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device="cuda")
+    cols = N // 2 if epi == 2 else N
+    outs = []
+    for rows_dev in (None, torch.tensor([m], dtype=torch.int32, device="cuda")):
+        out = torch.full((M, cols), -7.0, dtype=torch.bfloat16, device="cuda")
+        if R is not None:
+            out.copy_(R)
+        davet.davet_linear(A, M, K, W, N, out, epi, out if epi == 1 else None, workspace=ws, rows_dev=rows_dev)
+        torch.cuda.synchronize()
+        assert davet.davet_device_status() == (0, 0)
+        outs.append(out)
+    full, dyn = outs
+    n = min(m, M)
+    untouched = R if epi == 1 else torch.full((M, cols), -7.0, dtype=torch.bfloat16, device="cuda")
+    assert torch.equal(dyn[n:], untouched[n:])
+    # the same tiling and K slices as the launch for all M rows: bit-identical rows
+    assert torch.equal(dyn[:n], full[:n])
+    if n:
+        y = f64(A[:n]) @ f64(W).T
+        if epi == 0:
+            ref = y
+        elif epi == 1:
+            ref = f64(R[:n]) + y
+        else:
+            blocks = y.reshape(n, N // 256, 2, 128)
+            ref = (L.silu(blocks[:, :, 0]) * blocks[:, :, 1]).reshape(n, N // 2)
+        check_close(dyn[:n], ref, f"rows_dev {m} of {M}")
+
+
+def test_rotary_device_row_count(davet):
+    """The rotary epilogue with the packed sequence shorter than the launch:
+    cu_seqlens ends at the device count (as the gather leaves it)."""
+    D, H, K = 128, 2, 256
+    HD = H * D
+    cu = [0, 150, 151, 333]
+    M = 600
+    A = rand_bf16((M, K), 113).cuda()
+    W = rand_bf16((3 * HD, K), 114, K ** -0.5).cuda()
+    tab = torch.empty((1024, D // 2, 2), dtype=torch.float32, device="cuda")
+    davet.davet_rope_table(1024, D, THETA, tab)
+    cu_d = torch.tensor(cu, dtype=torch.int32, device="cuda")
+    out = torch.full((M, 3 * HD), -7.0, dtype=torch.bfloat16, device="cuda")
+    davet.davet_linear(A, M, K, W, 3 * HD, out, davet.EPI_ROPE, None, cu_d, 3, 2 * HD, D, tab, 1024,
+                       rows_dev=cu_d[3:])
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    n = cu[-1]
+    assert (out[n:].float() == -7.0).all()
+    y = f64(A[:n]) @ f64(W).T
+    pos = L.positions(cu)
+    ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
+                          y[:, 2 * HD:]], axis=1)
+    check_close(out[:n], ref, "rope rows_dev")
+
+
+@pytest.mark.parametrize("m", [0, 1, 77, 200])
+def test_rmsnorm_device_row_count(davet, m):
+    M, C = 160, 512
+    x = rand_bf16((M, C), 115).cuda()
+    g = (1 + 0.1 * rand_bf16((C,), 116).float()).to(torch.bfloat16).cuda()
+    out = torch.full((M, C), -7.0, dtype=torch.bfloat16, device="cuda")
+    davet.davet_rmsnorm(x, M, C, g, 1e-5, out, rows_dev=torch.tensor([m], dtype=torch.int32, device="cuda"))
+    torch.cuda.synchronize()
+    n = min(m, M)
+    assert (out[n:].float() == -7.0).all()
+    if n:
+        check_close(out[:n], L.rmsnorm(f64(x[:n]), f64(g), 1e-5), "rmsnorm rows_dev")
