@@ -504,9 +504,10 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  *            the angle of the row's position in its request, row - cu[b] for
  *            cu_seqlens[b] <= row < cu_seqlens[b+1]), the rest stored as is
  *   cu_seqlens, batch, rope_cols, head_dim (64 or 128), rope_table
- *            (davet_rope_table, [max_pos][head_dim/2] float2), max_pos:
- *            epilogue 3 only (nullable otherwise); a position >= max_pos is
- *            clamped and flags DAVET_DEV_ARG
+ *            (davet_rope_table, [head_dim/2][max_pos] float2), max_pos (the
+ *            table's, also its row stride): epilogue 3 only (nullable
+ *            otherwise); a position >= max_pos is clamped and flags
+ *            DAVET_DEV_ARG
  *   workspace, workspace_bytes   device scratch, nullable.  When the output
  *            tiles would occupy less than half of the SMs (few rows, few
  *            column blocks) and the workspace holds at least
@@ -530,8 +531,10 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  * davet_linear_workspace_bytes -- the workspace davet_linear can use for this
  * shape on the current device (0: none).
  *
- * davet_rope_table -- table[p][d] = (cos, sin)(p * theta^(-2d/head_dim)),
- * fp32, for p < max_pos and d < head_dim/2 (computed in fp64 on the device).
+ * davet_rope_table -- table[d][p] = (cos, sin)(p * theta^(-2d/head_dim)),
+ * fp32, for d < head_dim/2 and p < max_pos (frequency-major, so that rows
+ * at consecutive positions read consecutive entries; computed in fp64 on
+ * the device).
  *
  * davet_rmsnorm -- out = x / sqrt(mean(x^2) + eps) * gamma per row (fp32
  * sums, bf16 out); x, out bf16 [M][C], gamma bf16 [C], C % 8 == 0.  With

@@ -9,8 +9,13 @@
 //   warp 1     owns TMEM (512 columns: two 128 x 256 fp32 accumulators) and
 //              issues the MMAs (one thread, M = 128, N = 256, K = 16 each);
 //   warps 2-5  epilogue: thread r of the four warps owns accumulator row r,
-//              reads it from TMEM 32 columns at a time and writes bf16 rows;
-//              it runs on one accumulator while the MMAs fill the other.
+//              reads it from TMEM 32 columns at a time, applies the epilogue
+//              and writes bf16 into the warp's two 32 x 64 shared-memory
+//              slabs (128-byte swizzle), which the warp's lane 0 stores with
+//              TMA (full 128-byte lines; the threads do not wait for the
+//              writes); it runs on one accumulator while the MMAs fill the
+//              other.  A warp whose 32 rows are not all below M stores its
+//              valid rows directly instead.
 // Output tiles are visited m-fastest, so the CTAs working at the same time
 // share one 256-row block of W through L2.
 // Epilogues: plain store; residual add (out = residual + product, in place
@@ -18,7 +23,9 @@
 // 128: columns [0,128) of each tile are the gate, [128,256) the up
 // projection; out = silu(gate) * up, half as many columns); rotary position
 // embedding on the query and key columns (pairs (d, d + D/2) of each head,
-// angle from a cos/sin table indexed by the row's position in its request).
+// angle from a cos/sin table indexed by the row's position in its request;
+// the table is frequency-major, so the lanes of a warp, rows at consecutive
+// positions, read consecutive entries).
 #include <algorithm>
 #include <mutex>
 
@@ -36,9 +43,12 @@ constexpr uint32_t kStageB = BN * BK * 2;  // 32 KB
 
 enum : int { EPI_STORE = 0, EPI_RESIDUAL = 1, EPI_SWIGLU = 2, EPI_ROPE = 3 };
 
+constexpr uint32_t kSlab = 32 * 128;  // an epilogue warp's 32 rows x 64 bf16 columns: 4 KB
+
 struct Smem {
   alignas(1024) uint8_t a[STAGES][kStageA];
   alignas(1024) uint8_t b[STAGES][kStageB];
+  alignas(1024) uint8_t epi[4][2][kSlab];  // [epilogue warp][slab]
   uint64_t full[STAGES], empty[STAGES];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t fin;
@@ -60,7 +70,7 @@ struct Params {
   int rope_cols;  // columns [0, rope_cols) are query and key heads
   int head_dim;
   int max_pos;
-  const float2* rope;  // [max_pos][head_dim / 2] (cos, sin)
+  const float2* rope;  // [head_dim / 2][max_pos] (cos, sin), frequency-major
   unsigned* err;
   // split of K (CTA-pair kernel): `split` slices of `kb_per` k-blocks (the last
   // takes the rest) write fp32 partials [split][tiles_n][M rounded to 256][256]
@@ -151,7 +161,7 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
       }
     }
     const int half = p.head_dim / 2;
-    const float2* tab = p.rope + static_cast<long long>(pos) * half;
+    const float2* tab = p.rope + pos;  // frequency d at tab[d * max_pos]
     uint16_t* dst = p.out + row * p.ldo + n0;
 #pragma unroll 1
     for (int hb = 0; hb < BN; hb += p.head_dim) {
@@ -163,7 +173,7 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
         if (row_ok) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float2 cs = tab[c + i];
+            const float2 cs = tab[static_cast<long long>(c + i) * p.max_pos];
             const float a = x[i], b = y[i];
             x[i] = a * cs.x - b * cs.y;
             y[i] = b * cs.x + a * cs.y;
@@ -198,8 +208,134 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
   }
 }
 
+__device__ __forceinline__ void tma_store_2d(const void* tmap, const void* src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// the shared-memory sources of this thread's bulk stores have been read
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// ... and their writes are done
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// 32 values of this lane's row into a 32 x 64 slab, columns [col, col + 32)
+// (col 0 or 32), in the 128-byte swizzle the output map uses: 16-byte chunk
+// j of row r sits at r * 128 + (j ^ (r % 8)) * 16 (conflict-free per warp).
+__device__ __forceinline__ void stage32(uint8_t* slab, int lane, int col, const float (&v)[32]) {
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    uint4 w;
+    w.x = pack_bf16x2(v[8 * u + 0], v[8 * u + 1]);
+    w.y = pack_bf16x2(v[8 * u + 2], v[8 * u + 3]);
+    w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
+    w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
+    const int j = (col >> 3) + u;
+    *reinterpret_cast<uint4*>(slab + lane * 128 + ((j ^ (lane & 7)) << 4)) = w;
+  }
+}
+
+// 32 fp32 values of this lane's row into a 32 x 32 fp32 slab, same swizzle.
+__device__ __forceinline__ void stage32_f32(uint8_t* slab, int lane, const float (&v)[32]) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    *reinterpret_cast<float4*>(slab + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+        make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+}
+
+// The epilogue of one warp's 32 rows [row0, row0 + 32), all below M, of a
+// 256-column tile at column n0, in groups of 128 output columns: the group
+// goes through the warp's two slabs and out with two TMA stores of 32 x 64.
+// `get` is the TMEM read of epilogue_row.
+template <class Get>
+__device__ __forceinline__ void epilogue_warp_staged(const Params& p, const void* tmap_out, uint8_t* slab0,
+                                                     uint8_t* slab1, int lane, long long row0, int n0, Get&& get) {
+  const long long row = row0 + lane;
+  const bool swiglu = p.epi == EPI_SWIGLU, rope = p.epi == EPI_ROPE && n0 < p.rope_cols;
+  const int out0 = swiglu ? n0 / 2 : n0;
+  int pos = 0;
+  if (rope) {
+    int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (p.cu[mid] <= row) lo = mid; else hi = mid;
+    }
+    pos = static_cast<int>(row - p.cu[lo]);
+    if (pos >= p.max_pos) {
+      raise_error(p.err, DEV_ERR_ARG);
+      pos = p.max_pos - 1;
+    }
+  }
+#pragma unroll 1
+  for (int g = 0; g < (swiglu ? 1 : 2); ++g) {
+    if (lane == 0) bulk_wait_read();  // the previous group's stores have left the slabs
+    __syncwarp();
+    if (swiglu) {
+#pragma unroll 1
+      for (int c = 0; c < 128; c += 32) {
+        float a[32], u[32];
+        get(c, a);
+        get(128 + c, u);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) a[i] = silu(a[i]) * u[i];
+        stage32(c < 64 ? slab0 : slab1, lane, c & 63, a);
+      }
+    } else if (rope) {
+      const int half = p.head_dim / 2;
+#pragma unroll 1
+      for (int hb = 128 * g; hb < 128 * g + 128; hb += p.head_dim) {
+#pragma unroll 1
+        for (int c = 0; c < half; c += 32) {
+          float x[32], y[32];
+          get(hb + c, x);
+          get(hb + half + c, y);
+          const float2* tab = p.rope + static_cast<long long>(c) * p.max_pos + pos;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float2 cs = tab[static_cast<long long>(i) * p.max_pos];
+            const float a = x[i], b = y[i];
+            x[i] = a * cs.x - b * cs.y;
+            y[i] = b * cs.x + a * cs.y;
+          }
+          const int cx = hb + c - 128 * g, cy = cx + half;
+          stage32(cx < 64 ? slab0 : slab1, lane, cx & 63, x);
+          stage32(cy < 64 ? slab0 : slab1, lane, cy & 63, y);
+        }
+      }
+    } else {
+      const uint16_t* res = p.epi == EPI_RESIDUAL ? p.residual + row * p.ldo + n0 + 128 * g : nullptr;
+#pragma unroll 1
+      for (int c = 0; c < 128; c += 32) {
+        float v[32];
+        get(128 * g + c, v);
+        if (res) {
+          const uint4* r4 = reinterpret_cast<const uint4*>(res + c);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const uint4 w = r4[u];
+            v[8 * u + 0] += bf16lo(w.x); v[8 * u + 1] += bf16hi(w.x);
+            v[8 * u + 2] += bf16lo(w.y); v[8 * u + 3] += bf16hi(w.y);
+            v[8 * u + 4] += bf16lo(w.z); v[8 * u + 5] += bf16hi(w.z);
+            v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
+          }
+        }
+        stage32(c < 64 ? slab0 : slab1, lane, c & 63, v);
+      }
+    }
+    fence_proxy_async_smem();  // the slabs' generic writes, visible to the TMA unit
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tmap_out, slab0, out0 + 128 * g, static_cast<int>(row0));
+      tma_store_2d(tmap_out, slab1, out0 + 128 * g + 64, static_cast<int>(row0));
+      bulk_commit();
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p0) {
+    gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w,
+                const __grid_constant__ CUtensorMap tmap_out, Params p0) {
   extern __shared__ uint8_t smem_raw[];
   Params p = p0;
   Smem& s = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -226,6 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kWarpTma && lane == 0) {
     tma_prefetch_desc(&tmap_a);
     tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_out);
   }
   pdl_launch_dependents();
   pdl_wait();  // A (and the residual) come from the previous kernel
@@ -303,11 +440,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const long long row = static_cast<long long>(m0) + r;
       const bool row_ok = row < p.M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
-      epilogue_row(p, row, row_ok, n0, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
+      auto get = [&](int c, float (&v)[32]) { load_acc32(acc + c, v); };
+      const long long row0 = static_cast<long long>(m0) + 32 * q;
+      if (row0 + 32 <= p.M)
+        epilogue_warp_staged(p, &tmap_out, s.epi[q][0], s.epi[q][1], lane, row0, n0, get);
+      else
+        epilogue_row(p, row, row_ok, n0, get);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.acc_empty[ab]);
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -336,6 +479,7 @@ constexpr uint32_t kTmemCols2 = 512;        // two 128 x 256 accumulators per CT
 struct Smem2 {
   alignas(1024) uint8_t a[ST2][kStageA];
   alignas(1024) uint8_t b[ST2][kStageB2];
+  alignas(1024) uint8_t epi[4][2][kSlab];  // [epilogue warp][slab]
   uint64_t full[ST2], empty[ST2];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t fin;
@@ -388,7 +532,9 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm2_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w, Params p0) {
+    gemm2_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w,
+                 const __grid_constant__ CUtensorMap tmap_out, const __grid_constant__ CUtensorMap tmap_part,
+                 Params p0) {
   extern __shared__ uint8_t smem_raw[];
   Params p = p0;
   Smem2& s = *reinterpret_cast<Smem2*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -419,6 +565,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kWarpTma && lane == 0) {
     tma_prefetch_desc(&tmap_a);
     tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_out);
+    if (p.split > 1) tma_prefetch_desc(&tmap_part);
   }
   pdl_launch_dependents();
   pdl_wait();
@@ -520,21 +668,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool row_ok = row < p.M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
       if (p.split > 1) {
-        // fp32 partial products of this slice; the reduction kernel applies the epilogue
-        float4* dst = reinterpret_cast<float4*>(
-            p.part + ((static_cast<long long>(t % p.split) * p.tiles_n + nb) * (tiles_m2 * 2 * BM) + row) * BN);
+        // fp32 partial products of this slice (all 32 rows of the warp; rows
+        // past M are never read): 32 x 32 blocks through the slabs, TMA
+        // stores; the reduction kernel applies the epilogue
+        const int prow = static_cast<int>((static_cast<long long>(t % p.split) * p.tiles_n + nb) * (tiles_m2 * 2 * BM) +
+                                          m0 + 32 * q);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 0; c < BN; c += 64) {
+          if (lane == 0) bulk_wait_read();
+          __syncwarp();
           float v[32];
           load_acc32(acc + c, v);
-          if (row_ok) {
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-              dst[c / 4 + u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+          stage32_f32(s.epi[q][0], lane, v);
+          load_acc32(acc + c + 32, v);
+          stage32_f32(s.epi[q][1], lane, v);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmap_part, s.epi[q][0], c, prow);
+            tma_store_2d(&tmap_part, s.epi[q][1], c + 32, prow);
+            bulk_commit();
           }
         }
       } else {
-        epilogue_row(p, row, row_ok, nb * BN, [&](int c, float (&v)[32]) { load_acc32(acc + c, v); });
+        auto get = [&](int c, float (&v)[32]) { load_acc32(acc + c, v); };
+        const long long row0 = static_cast<long long>(m0) + 32 * q;
+        if (row0 + 32 <= p.M)
+          epilogue_warp_staged(p, &tmap_out, s.epi[q][0], s.epi[q][1], lane, row0, nb * BN, get);
+        else
+          epilogue_row(p, row, row_ok, nb * BN, get);
       }
       tc_fence_before();
       __syncwarp();
@@ -545,6 +707,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           remote_arrive(map_to_rank(&s.acc_empty[ab], 0));
       }
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   tc_fence_before();
@@ -611,10 +774,10 @@ __global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
         pos = p.max_pos - 1;
       }
       const bool first = (8 * lane) % p.head_dim < half;  // columns in the first half of the head
-      const float2* tab = p.rope + static_cast<long long>(pos) * half + (8 * lane) % half;
+      const float2* tab = p.rope + static_cast<long long>((8 * lane) % half) * p.max_pos + pos;
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const float2 cs = tab[i];
+        const float2 cs = tab[static_cast<long long>(i) * p.max_pos];
         v[i] = first ? v[i] * cs.x - pv[i] * cs.y : v[i] * cs.x + pv[i] * cs.y;
       }
       dst = p.out + row * p.ldo + n0 + 8 * lane;
@@ -636,14 +799,15 @@ __global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
   }
 }
 
-// cos/sin table of the rotary embedding: tab[p][d] = (cos, sin)(p * theta^(-2d/D)).
+// cos/sin table of the rotary embedding, frequency-major:
+// tab[d][p] = (cos, sin)(p * theta^(-2d/D)).
 __global__ void rope_table_kernel(float2* tab, int max_pos, int half, double theta) {
   pdl_launch_dependents();
   pdl_wait();
   const long long total = static_cast<long long>(max_pos) * half;
   for (long long q = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; q < total;
        q += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int pos = static_cast<int>(q / half), d = static_cast<int>(q % half);
+    const int d = static_cast<int>(q / max_pos), pos = static_cast<int>(q % max_pos);
     const double ang = pos * pow(theta, -static_cast<double>(d) / half);
     tab[q] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
   }
@@ -796,8 +960,23 @@ int pick_split(long long M, int tiles_n, int nk, int pairs) {
   return S >= 2 ? S : 1;
 }
 
-size_t split_bytes(long long M, int tiles_n, int S) {
-  return static_cast<size_t>(S) * tiles_n * (((M + 2 * BM - 1) / (2 * BM)) * 2 * BM) * BN * 4;
+// fp32 partial rows: [S][tiles_n][M rounded up to 256][256]
+long long split_rows(long long M, int tiles_n, int S) {
+  return static_cast<long long>(S) * tiles_n * (((M + 2 * BM - 1) / (2 * BM)) * 2 * BM);
+}
+size_t split_bytes(long long M, int tiles_n, int S) { return static_cast<size_t>(split_rows(M, tiles_n, S)) * BN * 4; }
+
+// 2-D map over the fp32 partial rows [rows][256], boxes of 32 x 32.
+bool make_part_map(CUtensorMap* m, void* base, long long rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(BN), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(BN) * 4};
+  const cuuint32_t box[2] = {32, 32};
+  const cuuint32_t estride[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -853,7 +1032,11 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   unsigned* err = device_error_word();
   if (!err) return DAVET_ERR_CUDA;
   CUtensorMap ma, mw;
-  if (!make_map(&ma, A, M, K, BM) || !make_map(&mw, W, N, K, BN)) return DAVET_ERR_INVALID_ARG;
+  // the output map: boxes of 32 rows x 64 columns (one epilogue warp's slab)
+  CUtensorMap mo;
+  if (!make_map(&ma, A, M, K, BM) || !make_map(&mw, W, N, K, BN) ||
+      !make_map(&mo, out, M, epilogue == EPI_SWIGLU ? N / 2 : N, 32))
+    return DAVET_ERR_INVALID_ARG;
   Params p;
   p.M = M;
   p.N = N;
@@ -883,14 +1066,16 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   const int pairs = g_sms[dev] / 2;
   const long long tiles2 = ((M + 2 * BM - 1) / (2 * BM)) * p.tiles_n;
   if (M > BM) {
+    CUtensorMap mw2, mp;
+    if (!make_map(&mw2, W, N, K, BM)) return DAVET_ERR_INVALID_ARG;
+    mp = mo;  // the partial map is read only with a split
     const int S = pick_split(M, p.tiles_n, K / BK, pairs);
     if (S > 1 && workspace && workspace_bytes >= split_bytes(M, p.tiles_n, S) && aligned16(workspace)) {
+      if (!make_part_map(&mp, workspace, split_rows(M, p.tiles_n, S))) return DAVET_ERR_INVALID_ARG;
       p.split = S;
       p.kb_per = (K / BK) / S;
       p.part = static_cast<float*>(workspace);
     }
-    CUtensorMap mw2;
-    if (!make_map(&mw2, W, N, K, BM)) return DAVET_ERR_INVALID_ARG;
     const int grid2 = 2 * static_cast<int>(std::min<long long>(tiles2 * p.split, pairs));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid2);
@@ -906,7 +1091,7 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl_enabled() ? 2 : 1;
-    e = cudaLaunchKernelEx(&cfg, gemm2_kernel, ma, mw2, p);
+    e = cudaLaunchKernelEx(&cfg, gemm2_kernel, ma, mw2, mo, mp, p);
     if (e != cudaSuccess) return cuda_fail(e);
     if (p.split > 1) {
       const long long warps = M * p.tiles_n;
@@ -917,7 +1102,7 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
     return check_launch();
   }
   const int grid = static_cast<int>(std::min<long long>(tiles, g_sms[dev]));
-  e = launch(gemm_kernel, dim3(grid), dim3(kThreads), smem, st, ma, mw, p);
+  e = launch(gemm_kernel, dim3(grid), dim3(kThreads), smem, st, ma, mw, mo, p);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

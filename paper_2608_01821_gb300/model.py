@@ -102,7 +102,7 @@ class Backbone:
         self.xa = torch.empty((max(R, 1), C), dtype=torch.bfloat16, device=dev)
         self.logits = torch.empty((max(R, 1), w.V), dtype=torch.bfloat16, device=dev)
         self.max_pos = max(max(w.seq_len(b, v) for v in range(w.n_views())) for b in range(w.batch))
-        self.rope = torch.empty((self.max_pos, D // 2, 2), dtype=torch.float32, device=dev)
+        self.rope = torch.empty((D // 2, self.max_pos, 2), dtype=torch.float32, device=dev)
         self.lib.davet_rope_table(self.max_pos, D, ROPE_THETA, self.rope)
         self.masked = torch.ones(R, dtype=torch.uint8, device=dev)
         self.tokens = torch.full((R,), -1, dtype=torch.int32, device=dev)

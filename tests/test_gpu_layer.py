@@ -93,7 +93,7 @@ def test_linear_rotary_qkv(davet, D, H):
     A = rand_bf16((M, K), 8).cuda()
     W = rand_bf16((3 * HD, K), 9, K ** -0.5).cuda()
     max_pos = 512
-    tab = torch.empty((max_pos, D // 2, 2), dtype=torch.float32, device="cuda")
+    tab = torch.empty((D // 2, max_pos, 2), dtype=torch.float32, device="cuda")
     davet.davet_rope_table(max_pos, D, THETA, tab)
     cu_d = torch.tensor(cu, dtype=torch.int32, device="cuda")
     out = linear(davet, A, W, davet.EPI_ROPE, cu_seqlens=cu_d, batch=len(cu) - 1, rope_cols=2 * HD, head_dim=D,
@@ -103,8 +103,8 @@ def test_linear_rotary_qkv(davet, D, H):
     ref = np.concatenate([L.rope(y[:, :HD], pos, H, D, THETA), L.rope(y[:, HD:2 * HD], pos, H, D, THETA),
                           y[:, 2 * HD:]], axis=1)
     check_close(out, ref, "rope")
-    # the table itself: fp32 rounding of the fp64 angles' cos and sin
-    ang = L.rope_angles(np.arange(max_pos), D, THETA)
+    # the table itself (frequency-major): fp32 rounding of the fp64 angles' cos and sin
+    ang = L.rope_angles(np.arange(max_pos), D, THETA).T
     t = tab.cpu().double().numpy()
     assert np.abs(t[..., 0] - np.cos(ang)).max() < 1e-6 and np.abs(t[..., 1] - np.sin(ang)).max() < 1e-6
 
@@ -112,7 +112,7 @@ def test_linear_rotary_qkv(davet, D, H):
 def test_rope_position_past_the_table_is_flagged(davet):
     D, H, K = 64, 4, 64
     cu = torch.tensor([0, 40], dtype=torch.int32, device="cuda")
-    tab = torch.empty((16, D // 2, 2), dtype=torch.float32, device="cuda")
+    tab = torch.empty((D // 2, 16, 2), dtype=torch.float32, device="cuda")
     davet.davet_rope_table(16, D, THETA, tab)
     A = rand_bf16((40, K), 10).cuda()
     W = rand_bf16((3 * H * D, K), 11, K ** -0.5).cuda()
@@ -187,7 +187,7 @@ def test_one_layer_against_the_oracle(davet):
     wqkv = torch.cat([wq, wk, wv]).to(dev)
     wgu = torch.stack([wg.reshape(F // 128, 128, C), wu.reshape(F // 128, 128, C)], 1).reshape(2 * F, C).to(dev)
     cu_d = torch.tensor(cu, dtype=torch.int32, device=dev)
-    tab = torch.empty((512, D // 2, 2), dtype=torch.float32, device=dev)
+    tab = torch.empty((D // 2, 512, 2), dtype=torch.float32, device=dev)
     davet.davet_rope_table(512, D, THETA, tab)
     h = torch.empty((N, C), dtype=torch.bfloat16, device=dev)
     qkv = torch.empty((N, 3 * HD), dtype=torch.bfloat16, device=dev)
@@ -260,7 +260,7 @@ def test_pair_tiles_rotary(davet):
     M = cu[-1]
     A = rand_bf16((M, K), 80).cuda()
     W = rand_bf16((3 * HD, K), 81, K ** -0.5).cuda()
-    tab = torch.empty((1024, D // 2, 2), dtype=torch.float32, device="cuda")
+    tab = torch.empty((D // 2, 1024, 2), dtype=torch.float32, device="cuda")
     davet.davet_rope_table(1024, D, THETA, tab)
     out = linear(davet, A, W, davet.EPI_ROPE, cu_seqlens=torch.tensor(cu, dtype=torch.int32, device="cuda"),
                  batch=3, rope_cols=2 * HD, head_dim=D, rope_table=tab, max_pos=1024)
@@ -315,7 +315,7 @@ def test_pair_split_k_rotary(davet, D, H):
     M = cu[-1]
     A = rand_bf16((M, K), 95).cuda()
     W = rand_bf16((3 * HD, K), 96, K ** -0.5).cuda()
-    tab = torch.empty((256, D // 2, 2), dtype=torch.float32, device="cuda")
+    tab = torch.empty((D // 2, 256, 2), dtype=torch.float32, device="cuda")
     davet.davet_rope_table(256, D, THETA, tab)
     nbytes = davet.davet_linear_workspace_bytes(M, K, 3 * HD)
     assert nbytes > 0
@@ -354,7 +354,8 @@ def test_pair_tiles_single_valid_row_in_the_odd_cta(davet, M, N):
 # ------------------------------------------- row count read on the device
 # rows_dev: the kernels are launched for a capacity of M rows and read the
 # row count m from device memory when they start; rows from m on keep their
-# contents, rows below m match the oracle (and the launch without rows_dev).
+# contents, rows below m match the oracle (and, bit for bit, the launch
+# without rows_dev: the tiling and the K slices are chosen for M).
 @pytest.mark.parametrize("M,m,K,N,epi", [(100, 37, 256, 512, 0),      # one-CTA tiles
                                          (700, 300, 512, 1024, 1),    # CTA pairs, residual
                                          (700, 129, 512, 1024, 2),    # pairs, one valid row in the odd CTA
@@ -382,7 +383,6 @@ def test_linear_device_row_count(davet, M, m, K, N, epi):
     n = min(m, M)
     untouched = R if epi == 1 else torch.full((M, cols), -7.0, dtype=torch.bfloat16, device="cuda")
     assert torch.equal(dyn[n:], untouched[n:])
-    # the same tiling and K slices as the launch for all M rows: bit-identical rows
     assert torch.equal(dyn[:n], full[:n])
     if n:
         y = f64(A[:n]) @ f64(W).T
@@ -405,7 +405,7 @@ def test_rotary_device_row_count(davet):
     M = 600
     A = rand_bf16((M, K), 113).cuda()
     W = rand_bf16((3 * HD, K), 114, K ** -0.5).cuda()
-    tab = torch.empty((1024, D // 2, 2), dtype=torch.float32, device="cuda")
+    tab = torch.empty((D // 2, 1024, 2), dtype=torch.float32, device="cuda")
     davet.davet_rope_table(1024, D, THETA, tab)
     cu_d = torch.tensor(cu, dtype=torch.int32, device="cuda")
     out = torch.full((M, 3 * HD), -7.0, dtype=torch.bfloat16, device="cuda")
