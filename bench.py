@@ -636,12 +636,16 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
     copied in, every step's logits read from pinned host memory, committed
     tokens copied out.
 
-    Mode "mapped" (default): the unmasking kernel reads each step's logits
-    straight from pinned host memory (device-addressable), so only the rows
-    still masked cross the host link.  Mode "copy": every step's full logits
-    are copied on a second stream into a ring of three device buffers, the
-    copy for step t+1 overlapping the kernels of step t (ordered with events);
-    the timed region spans both streams."""
+    Mode "staged" (default): on a second stream, davet_stage_masked_rows
+    copies the rows of step t's logits that were still masked after step t-2
+    (a superset of the rows step t reads) from pinned host memory into a ring
+    of three device buffers, overlapping the kernels of step t-1; step t's
+    unmasking reads the staged rows.  Mode "mapped": the unmasking kernel
+    reads each step's logits straight from pinned host memory (only rows still
+    masked cross the host link), in line with the step's other kernels.  Mode
+    "copy": every step's full logits are copied on the second stream, the copy
+    for step t+1 overlapping the kernels of step t.  The timed region spans
+    both streams; events order them."""
     import torch
 
     from paper_2608_01821_gb300 import workloads
@@ -652,11 +656,17 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
     P = 4
     host_logits = [workloads.logits(w, t).pin_memory() for t in range(P)]
     NB = 3
-    mapped = getattr(args, "e2e_mode", "mapped") == "mapped"
+    mode = getattr(args, "e2e_mode", "staged")
+    mapped = mode == "mapped"
     dev_logits = [] if mapped else [torch.empty((w.total_resp, w.V), dtype=torch.bfloat16, device=dev)
                                     for _ in range(NB)]
     tokens_host = torch.empty(w.total_resp, dtype=torch.int32).pin_memory()
-    logit_rows = sum(w.masked_rows(t) for t in range(w.T)) if mapped else w.T * w.total_resp
+    if mode == "mapped":
+        logit_rows = sum(w.masked_rows(t) for t in range(w.T))
+    elif mode == "staged":
+        logit_rows = sum(w.masked_rows(max(t - 1, 0)) for t in range(w.T))
+    else:
+        logit_rows = w.T * w.total_resp
     h2d = sum(f.numel() * 2 for f in feats) + text.numel() * 2 + logit_rows * w.V * 2
     if scores is not None:
         h2d += sum(x.numel() * 4 for x in scores)
@@ -707,7 +717,41 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
                 issue_copy(t + NB)
         tokens_host.copy_(pl.tokens, non_blocking=True)
 
-    one = one_mapped if mapped else one_copy
+    lib = pl.lib
+    reset_done = torch.cuda.Event()
+    step_done = [torch.cuda.Event() for _ in range(NB)]
+
+    def issue_stage(t):
+        # rows masked now (after step t-2's commits, or all at the start of the pass)
+        with torch.cuda.stream(copy_stream):
+            lib.davet_stage_masked_rows(host_logits[t % P], w.V, pl.masked, w.total_resp, dev_logits[t % NB],
+                                        copy_stream)
+            ready[t % NB].record(copy_stream)
+
+    def one_staged():
+        pl.reset_state()
+        reset_done.record(stream)
+        copy_stream.wait_event(reset_done)
+        for t in range(min(2, w.T)):
+            issue_stage(t)
+        pl.load_inputs(feats, text, non_blocking=True, scores=scores)
+        pl.build_pyramids()
+        if policy_pass:
+            policy_pass()
+        for t in range(w.T):
+            slot = t % NB
+            stream.wait_event(ready[slot])
+            if policy_step:
+                policy_step(t)
+            pl.step(t, dev_logits[slot])
+            step_done[slot].record(stream)
+            if t + 2 < w.T:
+                # step t's commits are done and step t-1 no longer reads slot (t+2) % 3
+                copy_stream.wait_event(step_done[slot])
+                issue_stage(t + 2)
+        tokens_host.copy_(pl.tokens, non_blocking=True)
+
+    one = {"mapped": one_mapped, "copy": one_copy, "staged": one_staged}[mode]
     with torch.cuda.stream(stream):
         one()
     torch.cuda.synchronize()
@@ -722,7 +766,7 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
     torch.cuda.synchronize()
     t = allreduce_max(s.elapsed_time(e) / 1e3, world, dev)
     return {"value": round(w.T * n * world / t, 3), "unit": "denoising steps/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "passes": n, "mode": "mapped" if mapped else "copy",
+            "d2h_bytes_per_step": int(d2h), "passes": n, "mode": mode,
             "h2d_GBps": round(h2d * n / t / 1e9, 1)}
 
 
@@ -975,8 +1019,9 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--logit-pool", type=int, default=0, help="cap on distinct device logit buffers")
-    ap.add_argument("--e2e-mode", choices=["mapped", "copy"], default="mapped",
-                    help="e2e logits: read from pinned host memory by the kernel, or copied to the device")
+    ap.add_argument("--e2e-mode", choices=["staged", "mapped", "copy"], default="staged",
+                    help="e2e logits: masked rows staged on a second stream one step ahead, read from pinned host "
+                         "memory by the unmasking kernel, or full logits copied to the device")
     ap.add_argument("--unfused", action="store_true",
                     help="pack each step with davet_gather_view, then davet_step_attention (instead of the fused call)")
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,

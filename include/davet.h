@@ -445,6 +445,26 @@ davet_status davet_policy_step(int t, int T, const double* lower_dev, const doub
                                const float* stats_prev_dev, int batch, double alpha, const int32_t* view_level,
                                int32_t* level_out_dev, double* budget_out_dev, void* stream);
 
+/*
+ * davet_stage_masked_rows -- copies row i (V bf16) of src to row i of dst for
+ * every i < total_rows with masked_dev[i] != 0; other rows of dst are left
+ * as they are.  The paper has no counterpart: it is input staging for the
+ * unmasking (Eq. 2 reads only the still-masked positions' distributions).
+ * A caller whose step logits live in pinned host memory can stage step t's
+ * rows on a second stream while the GPU runs step t-1, using the mask after
+ * step t-2 (a superset of the rows step t reads: commits only clear it), and
+ * then call davet_unmask_topk on dst.
+ *   src   bf16 [total_rows][V], device-addressable (device memory or pinned
+ *         host memory), 16-byte aligned; dst bf16 [total_rows][V] device
+ *         memory, 16-byte aligned; V % 8 == 0
+ *   masked_dev  uint8 [total_rows]; may change during the call only from
+ *         nonzero to zero (a row then copied or not, either is correct for
+ *         a later call that reads only rows still masked)
+ * One kernel on `stream`.
+ */
+davet_status davet_stage_masked_rows(const void* src, int V, const uint8_t* masked_dev, int64_t total_rows,
+                                     void* dst, void* stream);
+
 /* Size of the scratch array that davet_unmask_topk_noalloc uses (per device). */
 #define DAVET_NOALLOC_SCRATCH_BYTES (1u << 20)
 

@@ -480,6 +480,64 @@ extern "C" davet_status davet_unmask_topk(const void* logits, int V, const int32
 }
 
 // ---------------------------------------------------------------------------
+// Staging of the rows the unmasking will read: row i of `src` (device
+// addressable: device memory or pinned host memory) is copied to row i of
+// `dst` wherever masked[i] != 0.  One warp per (row, 8 KB chunk), the
+// chunk's 16-byte loads all issued before the first store.
+namespace davet {
+namespace unm {
+
+__global__ void __launch_bounds__(kRowThreads) stage_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst,
+                                                            int V8, int nchunk, int chunk, long long total_rows,
+                                                            const uint8_t* __restrict__ masked) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const long long unit = (static_cast<long long>(blockIdx.x) * kRowThreads + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (unit >= total_rows * nchunk) return;
+  const long long row = unit / nchunk;
+  if (!masked[row]) return;
+  const int ch = static_cast<int>(unit - row * nchunk);
+  const int lo = ch * chunk, hi = min(V8, lo + chunk);
+  const uint4* s = src + row * static_cast<long long>(V8);
+  uint4* d = dst + row * static_cast<long long>(V8);
+  for (int v = lo + lane; v < hi; v += 32 * kLoads) {
+    uint4 u[kLoads];
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k)
+      if (v + 32 * k < hi) u[k] = ld_stream(s + v + 32 * k);
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k)
+      if (v + 32 * k < hi) d[v + 32 * k] = u[k];
+  }
+}
+
+}  // namespace unm
+}  // namespace davet
+
+extern "C" davet_status davet_stage_masked_rows(const void* src, int V, const uint8_t* masked_dev, int64_t total_rows,
+                                                void* dst, void* stream) {
+  using namespace davet;
+  using namespace davet::unm;
+  if (V < 8 || V % 8 != 0 || total_rows < 0) return DAVET_ERR_INVALID_ARG;
+  if (total_rows == 0) return DAVET_OK;
+  if (!src || !dst || !masked_dev) return DAVET_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) return DAVET_ERR_INVALID_ARG;
+  if (total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
+  const int V8 = V / 8;
+  const int nchunk = std::max(1, std::min(kMaxChunks, (V8 + 511) / 512));
+  const int chunk = (V8 + nchunk - 1) / nchunk;
+  const long long warps = total_rows * nchunk;
+  const long long blocks = (warps + kRowThreads / 32 - 1) / (kRowThreads / 32);
+  const cudaError_t e = launch(stage_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kRowThreads), 0,
+                               static_cast<cudaStream_t>(stream), static_cast<const uint4*>(src),
+                               static_cast<uint4*>(dst), V8, nchunk, chunk, static_cast<long long>(total_rows),
+                               masked_dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
+// ---------------------------------------------------------------------------
 // Allocation-free variant of davet_unmask_topk.
 //
 // Its scratch lives in a fixed device array owned by the library, so the

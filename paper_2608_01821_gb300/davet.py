@@ -91,6 +91,7 @@ def _declare(lib):
                                 _sz, _vp, _vp]),
         "davet_linear_workspace_bytes": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_rope_table": (_int, [_int, _int, ctypes.c_double, _vp, _vp]),
+        "davet_stage_masked_rows": (_int, [_vp, _int, _vp, _i64, _vp, _vp]),
         "davet_rmsnorm": (_int, [_vp, _i64, _int, _vp, _f32, _vp, _vp, _vp, _int, _vp, _vp]),
         "davet_embed_answers": (_int, [_vp, _int, _int, _vp, _int, _vp, _vp, _int, _i64, _vp, _vp]),
         "davet_unmask_topk_noalloc": (_int, [_vp, _int, _vp, _int, _i64, _int, _vp, _vp, _vp, _vp, _vp, _vp,
@@ -287,6 +288,11 @@ class Davet:
         self._check("davet_policy_step",
                     self.lib.davet_policy_step(t, T, _ptr(lower), _ptr(upper), _ptr(stats_prev), batch, float(alpha),
                                                vl, _ptr(level_out), _ptr(budget_out), _stream(stream)))
+
+    def davet_stage_masked_rows(self, src, V: int, masked, total_rows: int, dst, stream=None):
+        self._check("davet_stage_masked_rows",
+                    self.lib.davet_stage_masked_rows(_ptr(src), V, _ptr(masked), total_rows, _ptr(dst),
+                                                     _stream(stream)))
 
     def davet_unmask_topk_noalloc(self, logits, V: int, cu_resp, batch: int, total_rows: int, k: int, masked,
                                   tokens, argmax=None, conf=None, committed=None, stats=None, stream=None):

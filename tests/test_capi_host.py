@@ -138,6 +138,11 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_rmsnorm(p, 10, 16, p, ctypes.c_float(1e-5), p, null, p, 0, null, null) == INV
     assert lib.davet_embed_answers(p, 100, 16, p, 100, p, p, 1, 5, p, null) == INV
     assert lib.davet_embed_answers(p, 100, 16, p, 3, p, p, 1, 0, p, null) == 0
+    # masked-row staging: V, null buffers, alignment; nothing to copy is fine
+    assert lib.davet_stage_masked_rows(p, 12, p, 4, p, null) == INV
+    assert lib.davet_stage_masked_rows(null, 16, p, 4, p, null) == INV
+    assert lib.davet_stage_masked_rows(ctypes.c_void_p((1 << 20) + 2), 16, p, 4, p, null) == INV
+    assert lib.davet_stage_masked_rows(null, 16, null, 0, null, null) == 0
     # gather: bad levels count, batch too large
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 1, 27, 0, 0, 0, 16, p, p, 100, null) == INV
     assert lib.davet_gather_view(p, p, p, p, p, p, p, 5000, 27, 4, 0, 0, 16, p, p, 100, null) == UNS

@@ -161,3 +161,28 @@ def test_host_mapped_logits_match_device_logits(davet):
         assert davet.davet_device_status() == (0, 0)
         for key in ("masked", "tokens", "argmax", "conf", "committed", "stats"):
             assert torch.equal(a.d[key], b.d[key]), (t, key)
+
+
+@pytest.mark.parametrize("V,src_host", [(workloads.VOCAB_8B, True), (workloads.VOCAB_8B, False), (1024, True),
+                                        (4104, False)])
+def test_stage_masked_rows_copies_exactly_the_masked_rows(davet, V, src_host):
+    """davet_stage_masked_rows: every masked row bit for bit (from pinned host
+    or device memory, a vocabulary that is not a multiple of the chunk), every
+    other row of the destination untouched, nothing for an all-clear mask."""
+    R = 37
+    lg = workloads.normal_bf16((R, V), 950 + V, 2 ** 0.5)
+    src = lg.pin_memory() if src_host else lg.cuda()
+    g = torch.Generator().manual_seed(V)
+    masked = (torch.rand(R, generator=g) < 0.6).to(torch.uint8)
+    masked[0], masked[-1] = 1, 0
+    dst = torch.full((R, V), -3.0, dtype=torch.bfloat16, device="cuda")
+    davet.davet_stage_masked_rows(src, V, masked.cuda(), R, dst)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    m = masked.bool()
+    out = dst.cpu()
+    assert torch.equal(out[m].view(torch.int16), lg[m].view(torch.int16))
+    assert (out[~m].float() == -3.0).all()
+    davet.davet_stage_masked_rows(src, V, torch.zeros(R, dtype=torch.uint8, device="cuda"), R, dst)
+    torch.cuda.synchronize()
+    assert torch.equal(dst.cpu().view(torch.int16), out.view(torch.int16))
