@@ -544,6 +544,18 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  *            and the residual hold M rows, and the tiling and workspace are
  *            chosen for M.  Lets a captured step run a row count that
  *            earlier kernels decide (the allocation policy's views).
+ *   row_ss, row_ss_parts, row_ss_eps   nullable: RMS normalization of A's
+ *            rows folded into the product.  Row r of A . W^T is multiplied by
+ *            1 / sqrt(sum_{j < parts} row_ss[r * parts + j] / K + eps)
+ *            before the epilogue (fp32), so that with the normalization gain
+ *            folded into W (W[n][k] * gamma[k]) the call computes
+ *            rmsnorm(A) . W^T without a normalized copy of A.  row_ss: fp32
+ *            [M][parts], partial sums of squares of A's rows (ss_out of the
+ *            call that produced A, or davet_row_sumsq).
+ *   ss_out   nullable, epilogues 0 and 1 only: fp32 [M][N/256];
+ *            ss_out[r * (N/256) + j] = sum of squares of the bf16 values
+ *            stored in row r, columns [256j, 256j + 256) (for the next
+ *            call's row_ss with parts = N/256).
  * One persistent kernel on `stream` (with a split: a second kernel adds the
  * slices and applies the epilogue).  M > 128 runs on CTA pairs (clusters of
  * two CTAs on two SMs).
@@ -564,6 +576,10 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  * (device int32, nullable): the row count, read on the device and clamped to
  * [0, M], as in davet_linear.
  *
+ * davet_row_sumsq -- ss_out[r] = sum over c of x[r][c]^2 (fp32 sums of the
+ * bf16 values) for r < M (rows_dev as in davet_linear): row_ss with one part
+ * for the first projection of a step.  x bf16 [M][C], C % 8 == 0.
+ *
  * davet_embed_answers -- writes the answer rows of the packed step input from
  * an embedding table: row cu_seqlens[b+1] - n_b + i (n_b answer rows of
  * request b) becomes table[tokens[cu_resp[b] + i]], or table[mask_id] while
@@ -573,12 +589,14 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
 davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                           const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols, int head_dim,
                           const void* rope_table, int max_pos, void* workspace, size_t workspace_bytes,
+                          const float* row_ss, int row_ss_parts, float row_ss_eps, float* ss_out,
                           const int32_t* rows_dev, void* stream);
 davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, size_t* bytes);
 davet_status davet_rope_table(int max_pos, int head_dim, double theta, void* table, void* stream);
 davet_status davet_rmsnorm(const void* x, int64_t M, int C, const void* gamma, float eps, void* out,
                            const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, const int32_t* rows_dev,
                            void* stream);
+davet_status davet_row_sumsq(const void* x, int64_t M, int C, float* ss_out, const int32_t* rows_dev, void* stream);
 davet_status davet_embed_answers(const void* table, int V, int C, const int32_t* tokens, int mask_id,
                                  const int32_t* cu_seqlens, const int32_t* cu_resp, int batch, int64_t total_resp,
                                  void* x, void* stream);

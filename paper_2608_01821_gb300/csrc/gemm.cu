@@ -80,15 +80,34 @@ struct Params {
   // nullable: the row count on the device (at most M), read after the
   // previous kernel finished; rows from there on are neither computed nor stored
   const int32_t* rows_dev;
+  // normalization folded into the product (nullable): row r of the product
+  // is scaled by 1 / sqrt(sum_j rss[r * rss_parts + j] / K + rss_eps) before
+  // the epilogue, i.e. A's rows are RMS-normalized (the gain is in W)
+  const float* rss;
+  int rss_parts;
+  float rss_eps;
+  // nullable (store and residual epilogues): ss_out[r * tiles_n + n-block] =
+  // sum of squares of the row's 256 stored bf16 values, for the next
+  // product's normalization
+  float* ss_out;
 };
 
-// The launch's row count: M, or the smaller count on the device.
-__device__ __forceinline__ void device_rows(Params& p) {
-  if (p.rows_dev) {
-    const long long m = *p.rows_dev;
-    p.M = m < 0 ? 0 : (m < p.M ? m : p.M);
-    p.tiles_m = static_cast<int>((p.M + BM - 1) / BM);
-  }
+// 1 / rms of A's row from its partial sums of squares (1 without them).
+__device__ __forceinline__ float row_scale(const Params& p, long long row, bool row_ok) {
+  if (!p.rss || !row_ok) return 1.0f;
+  const float* s = p.rss + row * p.rss_parts;
+  float t = 0.0f;
+  for (int j = 0; j < p.rss_parts; ++j) t += s[j];
+  return rsqrtf(t / static_cast<float>(p.K) + p.rss_eps);
+}
+
+// The launch's row count: M, or the smaller count on the device.  Kernels
+// keep it in a scalar of their own rather than in their copy of the
+// parameters.
+__device__ __forceinline__ long long rows_now(const Params& p) {
+  if (!p.rows_dev) return p.M;
+  const long long m = *p.rows_dev;
+  return m < 0 ? 0 : (m < p.M ? m : p.M);
 }
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1) {
@@ -107,8 +126,20 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
 // silu(g) = g * sigmoid(g); the fast division is exact enough for a bf16 output
 __device__ __forceinline__ float silu(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
-__device__ __forceinline__ void store32(uint16_t* dst, const float (&v)[32]) {
+// sum of squares of the 8 bf16 values of a 16-byte word
+__device__ __forceinline__ float sumsq8(uint4 w) {
+  float s = 0.0f;
+  s = fmaf(bf16lo(w.x), bf16lo(w.x), s); s = fmaf(bf16hi(w.x), bf16hi(w.x), s);
+  s = fmaf(bf16lo(w.y), bf16lo(w.y), s); s = fmaf(bf16hi(w.y), bf16hi(w.y), s);
+  s = fmaf(bf16lo(w.z), bf16lo(w.z), s); s = fmaf(bf16hi(w.z), bf16hi(w.z), s);
+  s = fmaf(bf16lo(w.w), bf16lo(w.w), s); s = fmaf(bf16hi(w.w), bf16hi(w.w), s);
+  return s;
+}
+
+// Stores 32 values as bf16; returns the sum of squares of the stored values.
+__device__ __forceinline__ float store32(uint16_t* dst, const float (&v)[32]) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
+  float ss = 0.0f;
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     uint4 w;
@@ -117,7 +148,9 @@ __device__ __forceinline__ void store32(uint16_t* dst, const float (&v)[32]) {
     w.z = pack_bf16x2(v[8 * u + 4], v[8 * u + 5]);
     w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
     d4[u] = w;
+    ss += sumsq8(w);
   }
+  return ss;
 }
 
 __device__ __forceinline__ void load_acc32(uint32_t taddr, float (&v)[32]) {
@@ -186,6 +219,7 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
   } else {
     uint16_t* dst = p.out + row * p.ldo + n0;
     const uint16_t* res = p.epi == EPI_RESIDUAL ? p.residual + row * p.ldo + n0 : nullptr;
+    float ss = 0.0f;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
       float v[32];
@@ -202,9 +236,10 @@ __device__ __forceinline__ void epilogue_row(const Params& p, long long row, boo
             v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
           }
         }
-        store32(dst + c, v);
+        ss += store32(dst + c, v);
       }
     }
+    if (p.ss_out && row_ok) p.ss_out[row * p.tiles_n + n0 / BN] = ss;
   }
 }
 
@@ -223,7 +258,9 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 // 32 values of this lane's row into a 32 x 64 slab, columns [col, col + 32)
 // (col 0 or 32), in the 128-byte swizzle the output map uses: 16-byte chunk
 // j of row r sits at r * 128 + (j ^ (r % 8)) * 16 (conflict-free per warp).
-__device__ __forceinline__ void stage32(uint8_t* slab, int lane, int col, const float (&v)[32]) {
+// Returns the sum of squares of the staged bf16 values.
+__device__ __forceinline__ float stage32(uint8_t* slab, int lane, int col, const float (&v)[32]) {
+  float ss = 0.0f;
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     uint4 w;
@@ -233,7 +270,9 @@ __device__ __forceinline__ void stage32(uint8_t* slab, int lane, int col, const 
     w.w = pack_bf16x2(v[8 * u + 6], v[8 * u + 7]);
     const int j = (col >> 3) + u;
     *reinterpret_cast<uint4*>(slab + lane * 128 + ((j ^ (lane & 7)) << 4)) = w;
+    ss += sumsq8(w);
   }
+  return ss;
 }
 
 // 32 fp32 values of this lane's row into a 32 x 32 fp32 slab, same swizzle.
@@ -254,6 +293,7 @@ __device__ __forceinline__ void epilogue_warp_staged(const Params& p, const void
   const long long row = row0 + lane;
   const bool swiglu = p.epi == EPI_SWIGLU, rope = p.epi == EPI_ROPE && n0 < p.rope_cols;
   const int out0 = swiglu ? n0 / 2 : n0;
+  float ss = 0.0f;  // of the stored values (store and residual epilogues)
   int pos = 0;
   if (rope) {
     int lo = 0, hi = p.batch;  // largest b with cu[b] <= row
@@ -320,7 +360,7 @@ __device__ __forceinline__ void epilogue_warp_staged(const Params& p, const void
             v[8 * u + 6] += bf16lo(w.w); v[8 * u + 7] += bf16hi(w.w);
           }
         }
-        stage32(c < 64 ? slab0 : slab1, lane, c & 63, v);
+        ss += stage32(c < 64 ? slab0 : slab1, lane, c & 63, v);
       }
     }
     fence_proxy_async_smem();  // the slabs' generic writes, visible to the TMA unit
@@ -331,13 +371,14 @@ __device__ __forceinline__ void epilogue_warp_staged(const Params& p, const void
       bulk_commit();
     }
   }
+  if (p.ss_out && !swiglu && !rope) p.ss_out[row * p.tiles_n + n0 / BN] = ss;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_w,
                 const __grid_constant__ CUtensorMap tmap_out, Params p0) {
   extern __shared__ uint8_t smem_raw[];
-  Params p = p0;
+  const Params& p = p0;
   Smem& s = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   volatile int* abort_flag = &s.abort;
@@ -366,19 +407,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_launch_dependents();
   pdl_wait();  // A (and the residual) come from the previous kernel
-  device_rows(p);
+  const long long M = rows_now(p);
+  const int tiles_m = static_cast<int>((M + BM - 1) / BM);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s.tmem;
-  const int n_tiles = p.tiles_m * p.tiles_n;
+  const int n_tiles = tiles_m * p.tiles_n;
   const int nk = p.K / BK;
 
   if (warp == kWarpTma) {
     if (lane == 0) {
       uint32_t it = 0;
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
-        const int m0 = (t % p.tiles_m) * BM, n0 = (t / p.tiles_m) * BN;
+        const int m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * BN;
         bool ok = true;
         for (int kb = 0; kb < nk; ++kb, ++it) {
           const uint32_t st = it % STAGES;
@@ -436,13 +478,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t ab = tc & 1, use = tc >> 1;
       if (!warp_wait(&s.acc_full[ab], use & 1, p.err, abort_flag)) break;
       tc_fence_after();
-      const int m0 = (t % p.tiles_m) * BM, n0 = (t / p.tiles_m) * BN;
+      const int m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * BN;
       const long long row = static_cast<long long>(m0) + r;
-      const bool row_ok = row < p.M;
+      const bool row_ok = row < M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
-      auto get = [&](int c, float (&v)[32]) { load_acc32(acc + c, v); };
+      const float rs = row_scale(p, row, row_ok);
+      auto get = [&](int c, float (&v)[32]) {
+        load_acc32(acc + c, v);
+        if (p.rss) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] *= rs;
+        }
+      };
       const long long row0 = static_cast<long long>(m0) + 32 * q;
-      if (row0 + 32 <= p.M)
+      if (row0 + 32 <= M)
         epilogue_warp_staged(p, &tmap_out, s.epi[q][0], s.epi[q][1], lane, row0, n0, get);
       else
         epilogue_row(p, row, row_ok, n0, get);
@@ -536,7 +585,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                  const __grid_constant__ CUtensorMap tmap_out, const __grid_constant__ CUtensorMap tmap_part,
                  Params p0) {
   extern __shared__ uint8_t smem_raw[];
-  Params p = p0;
+  const Params& p = p0;
   Smem2& s = *reinterpret_cast<Smem2*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   volatile int* abort_flag = &s.abort;
@@ -570,7 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_launch_dependents();
   pdl_wait();
-  device_rows(p);  // both CTAs of the pair read the same count
+  const long long M = rows_now(p);  // both CTAs of the pair read the same count
   tc_fence_before();
   cluster_sync_all();  // barriers initialized and TMEM allocated in both CTAs
   tc_fence_after();
@@ -585,7 +634,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __syncthreads();
-  const int tiles_m2 = static_cast<int>((p.M + 2 * BM - 1) / (2 * BM));
+  const int tiles_m2 = static_cast<int>((M + 2 * BM - 1) / (2 * BM));
   const int n_tiles = tiles_m2 * p.tiles_n * p.split;
   const int nk = p.K / BK;
   // unit t: slice t % split of output tile t / split (m-block fastest)
@@ -665,7 +714,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int bt = t / p.split;
       const int m0 = (bt % tiles_m2) * 2 * BM + rank * BM, nb = bt / tiles_m2;
       const long long row = static_cast<long long>(m0) + r;
-      const bool row_ok = row < p.M;
+      const bool row_ok = row < M;
       const uint32_t acc = tmem + (static_cast<uint32_t>(32 * q) << 16) + ab * BN;
       if (p.split > 1) {
         // fp32 partial products of this slice (all 32 rows of the warp; rows
@@ -691,9 +740,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       } else {
-        auto get = [&](int c, float (&v)[32]) { load_acc32(acc + c, v); };
+        const float rs = row_scale(p, row, row_ok);
+        auto get = [&](int c, float (&v)[32]) {
+          load_acc32(acc + c, v);
+          if (p.rss) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= rs;
+          }
+        };
         const long long row0 = static_cast<long long>(m0) + 32 * q;
-        if (row0 + 32 <= p.M)
+        if (row0 + 32 <= M)
           epilogue_warp_staged(p, &tmap_out, s.epi[q][0], s.epi[q][1], lane, row0, nb * BN, get);
         else
           epilogue_row(p, row, row_ok, nb * BN, get);
@@ -726,15 +782,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
   pdl_launch_dependents();
   pdl_wait();
-  Params p = p0;
-  device_rows(p);
+  const Params& p = p0;
+  const long long M = rows_now(p);
   const int lane = threadIdx.x & 31;
   const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
-  const long long mp = ((p.M + 2 * BM - 1) / (2 * BM)) * 2 * BM;
-  for (long long u = w0; u < p.M * p.tiles_n; u += nw) {
-    const int nb = static_cast<int>(u / p.M);
-    const long long row = u % p.M;
+  const long long mp = ((M + 2 * BM - 1) / (2 * BM)) * 2 * BM;
+  for (long long u = w0; u < M * p.tiles_n; u += nw) {
+    const int nb = static_cast<int>(u / M);
+    const long long row = u % M;
     float v[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) v[i] = 0.0f;
@@ -745,6 +801,11 @@ __global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
       const float4 a = __ldcg(src), b = __ldcg(src + 1);
       v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
       v[4] += b.x; v[5] += b.y; v[6] += b.z; v[7] += b.w;
+    }
+    if (p.rss) {
+      const float rs = row_scale(p, row, true);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] *= rs;
     }
     const int n0 = nb * BN;
     uint4 o;
@@ -796,6 +857,12 @@ __global__ void __launch_bounds__(256) split_reduce_kernel(Params p0) {
     o.z = pack_bf16x2(v[4], v[5]);
     o.w = pack_bf16x2(v[6], v[7]);
     if (write) *reinterpret_cast<uint4*>(dst) = o;
+    if (p.ss_out && (p.epi == EPI_STORE || p.epi == EPI_RESIDUAL)) {
+      float ss = sumsq8(o);  // lanes in order by a shuffle tree: a fixed order
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+      if (lane == 0) p.ss_out[row * p.tiles_n + nb] = ss;
+    }
   }
 }
 
@@ -866,6 +933,30 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const uint16_t* __restrict
       w.w = pack_bf16x2(bf16lo(v.w) * inv * bf16lo(g.w), bf16hi(v.w) * inv * bf16hi(g.w));
       orow[c] = w;
     }
+  }
+}
+
+// Sum of squares of each row's bf16 values (fp32, one warp per row, lanes in
+// a shuffle tree): the normalization input of the first projection.
+__global__ void __launch_bounds__(256) row_sumsq_kernel(const uint16_t* __restrict__ x, long long M, int C,
+                                                        float* __restrict__ ss, const int32_t* __restrict__ rows_dev) {
+  pdl_launch_dependents();
+  pdl_wait();
+  if (rows_dev) {
+    const long long m = *rows_dev;
+    M = m < 0 ? 0 : (m < M ? m : M);
+  }
+  const int lane = threadIdx.x & 31;
+  const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  const int C8 = C / 8;
+  for (long long r = w0; r < M; r += nw) {
+    const uint4* xr = reinterpret_cast<const uint4*>(x + r * C);
+    float s = 0.0f;
+    for (int c = lane; c < C8; c += 32) s += sumsq8(xr[c]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) ss[r] = s;
   }
 }
 
@@ -998,9 +1089,12 @@ extern "C" davet_status davet_linear_workspace_bytes(int64_t M, int K, int N, si
 extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void* W, int N, void* out, int epilogue,
                                      const void* residual, const int32_t* cu_seqlens, int batch, int rope_cols,
                                      int head_dim, const void* rope_table, int max_pos, void* workspace,
-                                     size_t workspace_bytes, const int32_t* rows_dev, void* stream) {
+                                     size_t workspace_bytes, const float* row_ss, int row_ss_parts, float row_ss_eps,
+                                     float* ss_out, const int32_t* rows_dev, void* stream) {
   if (M < 0 || M > 0x7fffffffLL || K < BK || K % BK != 0 || N < BN || N % BN != 0) return DAVET_ERR_INVALID_ARG;
   if (epilogue < EPI_STORE || epilogue > EPI_ROPE) return DAVET_ERR_INVALID_ARG;
+  if (row_ss && (row_ss_parts < 1 || !(row_ss_eps >= 0.0f))) return DAVET_ERR_INVALID_ARG;
+  if (ss_out && epilogue != EPI_STORE && epilogue != EPI_RESIDUAL) return DAVET_ERR_INVALID_ARG;
   if (M == 0) return DAVET_OK;
   if (!A || !W || !out || !aligned16(A) || !aligned16(W) || !aligned16(out)) return DAVET_ERR_INVALID_ARG;
   if (epilogue == EPI_RESIDUAL && (!residual || !aligned16(residual))) return DAVET_ERR_INVALID_ARG;
@@ -1058,6 +1152,10 @@ extern "C" davet_status davet_linear(const void* A, int64_t M, int K, const void
   p.kb_per = K / BK;
   p.part = nullptr;
   p.rows_dev = rows_dev;
+  p.rss = row_ss;
+  p.rss_parts = row_ss ? row_ss_parts : 0;
+  p.rss_eps = row_ss_eps;
+  p.ss_out = ss_out;
   const long long tiles = static_cast<long long>(p.tiles_m) * p.tiles_n;
   if (tiles > 0x7fffffffLL) return DAVET_ERR_UNSUPPORTED;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1135,6 +1233,18 @@ extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const voi
                        os, cu_seqlens, cu_resp, batch, rows_dev)
               : launch(rmsnorm_kernel<false>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs,
                        eps, os, cu_seqlens, cu_resp, batch, rows_dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return check_launch();
+}
+
+extern "C" davet_status davet_row_sumsq(const void* x, int64_t M, int C, float* ss_out, const int32_t* rows_dev,
+                                         void* stream) {
+  if (M < 0 || C < 8 || C % 8 != 0) return DAVET_ERR_INVALID_ARG;
+  if (M == 0) return DAVET_OK;
+  if (!x || !ss_out || !aligned16(x)) return DAVET_ERR_INVALID_ARG;
+  const int blocks = static_cast<int>(std::min<long long>((M + 7) / 8, 152LL * 16));
+  const cudaError_t e = launch(row_sumsq_kernel, dim3(blocks), dim3(256), 0, static_cast<cudaStream_t>(stream),
+                               static_cast<const uint16_t*>(x), static_cast<long long>(M), C, ss_out, rows_dev);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

@@ -88,7 +88,8 @@ def _declare(lib):
         "davet_policy_step": (_int, [_int, _int, _vp, _vp, _vp, _int, ctypes.c_double, ctypes.POINTER(_i32), _vp,
                                      _vp, _vp]),
         "davet_linear": (_int, [_vp, _i64, _int, _vp, _int, _vp, _int, _vp, _vp, _int, _int, _int, _vp, _int, _vp,
-                                _sz, _vp, _vp]),
+                                _sz, _vp, _int, _f32, _vp, _vp, _vp]),
+        "davet_row_sumsq": (_int, [_vp, _i64, _int, _vp, _vp, _vp]),
         "davet_linear_workspace_bytes": (_int, [_i64, _int, _int, ctypes.POINTER(_sz)]),
         "davet_rope_table": (_int, [_int, _int, ctypes.c_double, _vp, _vp]),
         "davet_stage_masked_rows": (_int, [_vp, _int, _vp, _i64, _vp, _vp]),
@@ -247,13 +248,15 @@ class Davet:
 
     def davet_linear(self, A, M: int, K: int, W, N: int, out, epilogue: int = 0, residual=None, cu_seqlens=None,
                      batch: int = 0, rope_cols: int = 0, head_dim: int = 128, rope_table=None, max_pos: int = 0,
-                     workspace=None, workspace_bytes: int = 0, rows_dev=None, stream=None):
+                     workspace=None, workspace_bytes: int = 0, row_ss=None, row_ss_parts: int = 0,
+                     row_ss_eps: float = 0.0, ss_out=None, rows_dev=None, stream=None):
         if workspace is not None and not isinstance(workspace, int) and workspace_bytes == 0:
             workspace_bytes = workspace.numel() * workspace.element_size()
         self._check("davet_linear",
                     self.lib.davet_linear(_ptr(A), M, K, _ptr(W), N, _ptr(out), epilogue, _ptr(residual),
                                           _ptr(cu_seqlens), batch, rope_cols, head_dim, _ptr(rope_table), max_pos,
-                                          _ptr(workspace), workspace_bytes, _ptr(rows_dev), _stream(stream)))
+                                          _ptr(workspace), workspace_bytes, _ptr(row_ss), row_ss_parts,
+                                          float(row_ss_eps), _ptr(ss_out), _ptr(rows_dev), _stream(stream)))
 
     def davet_linear_workspace_bytes(self, M: int, K: int, N: int) -> int:
         n = _sz(0)
@@ -269,6 +272,10 @@ class Davet:
         self._check("davet_rmsnorm",
                     self.lib.davet_rmsnorm(_ptr(x), M, C, _ptr(gamma), float(eps), _ptr(out), _ptr(cu_seqlens),
                                            _ptr(cu_resp), batch, _ptr(rows_dev), _stream(stream)))
+
+    def davet_row_sumsq(self, x, M: int, C: int, ss_out, rows_dev=None, stream=None):
+        self._check("davet_row_sumsq",
+                    self.lib.davet_row_sumsq(_ptr(x), M, C, _ptr(ss_out), _ptr(rows_dev), _stream(stream)))
 
     def davet_embed_answers(self, table, V: int, C: int, tokens, mask_id: int, cu_seqlens, cu_resp, batch: int,
                             total_resp: int, x, stream=None):

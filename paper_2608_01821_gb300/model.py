@@ -5,10 +5,18 @@ step sequence [v_t || q || y^(t-1)]: the step's view rows and prompt rows
 come from the evidence pyramid and the text store (davet_gather_view), the
 answer rows are the embeddings of the current answer state (committed token
 or the mask token; davet_embed_answers); then `n_layers` pre-normalization
-layers (davet_rmsnorm, davet_linear with the rotary / residual / gated-MLP
-epilogues, davet_step_attention), the final normalization of the answer rows
-and the LM head give the logits that davet_unmask_topk commits from.  The
-rows carry hidden states of width C = H * D; the MLP width is 3C.
+layers (davet_linear with the rotary / residual / gated-MLP epilogues,
+davet_step_attention), the final normalization of the answer rows
+(davet_rmsnorm) and the LM head give the logits that davet_unmask_topk
+commits from.  The rows carry hidden states of width C = H * D; the MLP
+width is 3C.
+
+The two normalizations of a layer are folded into the projections that
+read them: the gains are multiplied into the QKV and gate/up weights once,
+the residual projections (output, down) also emit each row's partial sums of
+squares, and the next projection scales its product rows by 1 / rms (for the
+first layer the sums come from davet_row_sumsq).  rmsnorm(x) W^T =
+(x (W diag g)^T) / rms(x), so no normalized copy of x is written or read.
 
 Each step's view comes either from the workload's schedule (known on the
 host, so every launch is sized to the step's rows) or, after use_policy(),
@@ -59,19 +67,24 @@ class Backbone:
         def gain(k):
             return (1.0 + rnd((C,), k, 0.1).float()).to(torch.bfloat16)
 
+        def fold(wt, g):  # W diag(g), rounded to bf16 once
+            return (wt.float() * g.float()[None, :]).to(torch.bfloat16)
+
         self.layers = []
         for l in range(n_layers):
             base = 16 * (l + 1)
             wg = rnd((F, C), base + 4, C ** -0.5)
             wu = rnd((F, C), base + 5, C ** -0.5)
+            g1, g2 = gain(base + 0), gain(base + 3)
             self.layers.append(dict(
-                g1=gain(base + 0),
-                wqkv=rnd((3 * self.HD, C), base + 1, C ** -0.5),
+                g1=g1,
+                g2=g2,
+                # the normalization gains folded in: wqkv = Wqkv diag(g1), wgu = Wgu diag(g2)
+                wqkv=fold(rnd((3 * self.HD, C), base + 1, C ** -0.5), g1),
                 wo=rnd((C, self.HD), base + 2, self.HD ** -0.5),
-                g2=gain(base + 3),
                 # gate and up rows interleaved in blocks of 128 (the gated-MLP epilogue's layout)
-                wgu=torch.stack([wg.reshape(F // 128, 128, C), wu.reshape(F // 128, 128, C)], 1)
-                .reshape(2 * F, C).contiguous(),
+                wgu=fold(torch.stack([wg.reshape(F // 128, 128, C), wu.reshape(F // 128, 128, C)], 1)
+                         .reshape(2 * F, C), g2).contiguous(),
                 wd=rnd((C, F), base + 6, F ** -0.5),
             ))
             del wg, wu
@@ -95,7 +108,11 @@ class Backbone:
         self.cu = torch.zeros(w.batch + 1, dtype=torch.int32, device=dev)
         self.cu_resp = torch.from_numpy(w.cu_resp()).to(dev)
         self.x = torch.empty((self.max_rows, C), dtype=torch.bfloat16, device=dev)
-        self.h = torch.empty((self.max_rows, C), dtype=torch.bfloat16, device=dev)
+        # partial sums of squares of x's rows: from the input (one part) and
+        # from the residual projections (one part per 256 columns)
+        self.ss_in = torch.empty((self.max_rows, 1), dtype=torch.float32, device=dev)
+        self.ss_parts = C // 256
+        self.ss = [torch.empty((self.max_rows, self.ss_parts), dtype=torch.float32, device=dev) for _ in range(2)]
         self.qkv = torch.empty((self.max_rows, 3 * self.HD), dtype=torch.bfloat16, device=dev)
         self.att = torch.empty((self.max_rows, self.HD), dtype=torch.bfloat16, device=dev)
         self.a = torch.empty((self.max_rows, F), dtype=torch.bfloat16, device=dev)
@@ -190,20 +207,23 @@ class Backbone:
                                                    *w.mixed_args, C, self.x, self.cu, self.max_rows, stream))
         run("input", lambda: lib.davet_embed_answers(self.emb, w.V, C, self.tokens, self.mask_id, self.cu,
                                                      self.cu_resp, w.batch, self.R, self.x, stream))
-        for p in self.layers:
-            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g1"], RMS_EPS, self.h, rows_dev=nd, stream=stream))
-            run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wqkv"], 3 * HD, self.qkv, lib.EPI_ROPE, None,
+        run("norm", lambda: lib.davet_row_sumsq(self.x, N, C, self.ss_in, rows_dev=nd, stream=stream))
+        sa, sb, parts = self.ss[0], self.ss[1], self.ss_parts
+        for i, p in enumerate(self.layers):
+            ss, sp = (self.ss_in, 1) if i == 0 else (sb, parts)
+            run("gemm", lambda: lib.davet_linear(self.x, N, C, p["wqkv"], 3 * HD, self.qkv, lib.EPI_ROPE, None,
                                                  self.cu, w.batch, 2 * HD, w.D, self.rope, self.max_pos, ws,
-                                                 rows_dev=nd, stream=stream))
+                                                 row_ss=ss, row_ss_parts=sp, row_ss_eps=RMS_EPS, rows_dev=nd,
+                                                 stream=stream))
             run("attention", lambda: lib.davet_step_attention(self.qkv, self.cu, w.batch, self.max_rows, w.H, w.D,
                                                               w.scale, self.att, stream))
             run("gemm", lambda: lib.davet_linear(self.att, N, HD, p["wo"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 workspace=ws, rows_dev=nd, stream=stream))
-            run("norm", lambda: lib.davet_rmsnorm(self.x, N, C, p["g2"], RMS_EPS, self.h, rows_dev=nd, stream=stream))
-            run("gemm", lambda: lib.davet_linear(self.h, N, C, p["wgu"], 2 * F, self.a, lib.EPI_SWIGLU,
-                                                 workspace=ws, rows_dev=nd, stream=stream))
+                                                 workspace=ws, ss_out=sa, rows_dev=nd, stream=stream))
+            run("gemm", lambda: lib.davet_linear(self.x, N, C, p["wgu"], 2 * F, self.a, lib.EPI_SWIGLU,
+                                                 workspace=ws, row_ss=sa, row_ss_parts=parts, row_ss_eps=RMS_EPS,
+                                                 rows_dev=nd, stream=stream))
             run("gemm", lambda: lib.davet_linear(self.a, N, F, p["wd"], C, self.x, lib.EPI_RESIDUAL, self.x,
-                                                 workspace=ws, rows_dev=nd, stream=stream))
+                                                 workspace=ws, ss_out=sb, rows_dev=nd, stream=stream))
         run("norm", lambda: lib.davet_rmsnorm(self.x, self.R, C, self.gf, RMS_EPS, self.xa, self.cu, self.cu_resp,
                                               w.batch, stream))
         run("gemm", lambda: lib.davet_linear(self.xa, self.R, C, self.wlm, w.V, self.logits, workspace=ws,
@@ -247,7 +267,7 @@ class Backbone:
         return self.L * per_layer + k(self.R, C, self.w.V)
 
     def launches(self, t: int) -> int:
-        """Kernels of step t: gather, embedding, per layer two norms and the
-        attention, the projections, the final norm, two unmask kernels; with
-        the policy, its step kernel."""
-        return 2 + 3 * self.L + self.gemm_launches(t) + 1 + 2 + (1 if self.policy else 0)
+        """Kernels of step t: gather, embedding, the input's sums of squares,
+        per layer the attention, the projections, the final norm, two unmask
+        kernels; with the policy, its step kernel."""
+        return 3 + self.L + self.gemm_launches(t) + 1 + 2 + (1 if self.policy else 0)

@@ -123,14 +123,25 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_step_attention_workspace(-1, 1000, 32, 128, ctypes.byref(sz0)) == INV
     # full-layer kernels: GEMM shapes, epilogue codes, rotary arguments, norms, embedding
     sz = ctypes.c_size_t(0)
-    assert lib.davet_linear(p, 10, 100, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 100, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 256, p, 7, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 256, p, 1, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 512, 96, p, 16, null, 0, null, null) == INV
-    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 300, 128, p, 16, null, 0, null, null) == INV
-    assert lib.davet_linear(p, -1, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == INV
-    assert lib.davet_linear(null, 0, 128, null, 256, null, 0, null, null, 0, 0, 128, null, 0, null, 0, null, null) == 0
+    no_norm = (null, 0, ctypes.c_float(0), null, null, null)  # row_ss, parts, eps, ss_out, rows_dev, stream
+    assert lib.davet_linear(p, 10, 100, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, 10, 128, p, 100, p, 0, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 7, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 1, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 512, 96, p, 16, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, 10, 128, p, 768, p, 3, null, p, 1, 300, 128, p, 16, null, 0, *no_norm) == INV
+    assert lib.davet_linear(p, -1, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == INV
+    assert lib.davet_linear(null, 0, 128, null, 256, null, 0, null, null, 0, 0, 128, null, 0, null, 0, *no_norm) == 0
+    # folded normalization: parts >= 1, eps >= 0; sums of squares only from store / residual epilogues
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, p, 0,
+                            ctypes.c_float(1e-5), null, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 256, p, 0, null, null, 0, 0, 128, null, 0, null, 0, p, 16,
+                            ctypes.c_float(-1.0), null, null, null) == INV
+    assert lib.davet_linear(p, 10, 128, p, 512, p, 2, null, null, 0, 0, 128, null, 0, null, 0, null, 0,
+                            ctypes.c_float(0), p, null, null) == INV
+    assert lib.davet_row_sumsq(p, 10, 12, p, null, null) == INV
+    assert lib.davet_row_sumsq(p, 10, 16, null, null, null) == INV
+    assert lib.davet_row_sumsq(null, 0, 16, null, null, null) == 0
     assert lib.davet_linear_workspace_bytes(10, 100, 256, ctypes.byref(sz)) == INV
     assert lib.davet_rope_table(16, 96, ctypes.c_double(1e4), p, null) == INV
     assert lib.davet_rope_table(16, 128, ctypes.c_double(1.0), p, null) == INV

@@ -41,11 +41,15 @@ def oracle_inputs(bb, feats, prompts, t):
 
 
 def layer_weights(p, F):
+    """The oracle's layer weights from the model's: the normalization gains
+    are folded into the QKV and gate/up weights the model holds
+    (rmsnorm(x, g) W^T = rmsnorm(x, 1) (W diag g)^T), so the oracle takes
+    those bf16 weights with unit gains."""
     C = p["g1"].numel()
     wqkv = f64(p["wqkv"])
     HD = wqkv.shape[0] // 3
     gu = f64(p["wgu"]).reshape(F // 128, 2, 128, C)
-    return dict(g1=f64(p["g1"]), wq=wqkv[:HD], wk=wqkv[HD:2 * HD], wv=wqkv[2 * HD:], wo=f64(p["wo"]), g2=f64(p["g2"]),
+    return dict(g1=np.ones(C), wq=wqkv[:HD], wk=wqkv[HD:2 * HD], wv=wqkv[2 * HD:], wo=f64(p["wo"]), g2=np.ones(C),
                 wg=gu[:, 0].reshape(F, C), wu=gu[:, 1].reshape(F, C), wd=f64(p["wd"]))
 
 

@@ -434,3 +434,57 @@ def test_rmsnorm_device_row_count(davet, m):
     assert (out[n:].float() == -7.0).all()
     if n:
         check_close(out[:n], L.rmsnorm(f64(x[:n]), f64(g), 1e-5), "rmsnorm rows_dev")
+
+
+# ------------------------------------------- normalization folded into the product
+# rmsnorm(A, g) W^T = rmsnorm(A, 1) (W diag g)^T: the call scales product row r
+# by 1 / sqrt(sum of row_ss parts / K + eps); with W' = bf16(W diag g) as its
+# weights the oracle is rmsnorm(A, 1) W'^T on the same bf16 operands.
+@pytest.mark.parametrize("M,K,N,epi,split", [(300, 512, 768, 2, False), (100, 256, 512, 0, False),
+                                             (241, 4096, 4096, 0, True), (200, 1024, 2048, 2, True)])
+def test_linear_folded_rmsnorm(davet, M, K, N, epi, split):
+    A = rand_bf16((M, K), 120 + M, 3.0).cuda()
+    g = (1 + 0.1 * rand_bf16((K,), 121).float())
+    W = rand_bf16((N, K), 122 + N, K ** -0.5)
+    Wf = (W.float() * g[None, :]).to(torch.bfloat16).cuda()
+    ss = torch.empty((M, 1), dtype=torch.float32, device="cuda")
+    davet.davet_row_sumsq(A, M, K, ss)
+    nbytes = davet.davet_linear_workspace_bytes(M, K, N)
+    assert (nbytes > 0) == split
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device="cuda")
+    out = linear(davet, A, Wf, epi, out_cols=N // 2 if epi == 2 else N, workspace=ws, row_ss=ss, row_ss_parts=1,
+                 row_ss_eps=1e-5)
+    y = L.rmsnorm(f64(A), np.ones(K), 1e-5) @ f64(Wf).T
+    if epi == 2:
+        blocks = y.reshape(M, N // 256, 2, 128)
+        y = (L.silu(blocks[:, :, 0]) * blocks[:, :, 1]).reshape(M, N // 2)
+    check_close(out, y, f"folded norm {M}x{K}x{N} epi {epi}")
+    # the sums of squares themselves, against the fp64 sums of the bf16 rows
+    assert np.allclose(ss.cpu().numpy()[:, 0], (f64(A) ** 2).sum(1), rtol=1e-5)
+
+
+@pytest.mark.parametrize("M,K,N,parts_from_split", [(333, 512, 768, False), (241, 4096, 4096, True)])
+def test_linear_sums_of_squares_out_feed_the_next_product(davet, M, K, N, parts_from_split):
+    """A residual projection emits each row's sums of squares per 256 columns
+    (ss_out); they are the sums of the stored bf16 values, and as row_ss of
+    the next product they normalize its rows like rmsnorm would."""
+    A = rand_bf16((M, K), 130).cuda()
+    W = rand_bf16((N, K), 131, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 132).cuda()
+    nbytes = davet.davet_linear_workspace_bytes(M, K, N)
+    assert (nbytes > 0) == parts_from_split
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device="cuda")
+    x = R.clone()
+    parts = N // 256
+    ss = torch.full((M, parts), float("nan"), dtype=torch.float32, device="cuda")
+    davet.davet_linear(A, M, K, W, N, x, davet.EPI_RESIDUAL, x, workspace=ws, ss_out=ss)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    check_close(x, f64(R) + f64(A) @ f64(W).T, "residual with ss_out")
+    xs = f64(x).reshape(M, parts, 256)
+    assert np.allclose(ss.cpu().numpy(), (xs ** 2).sum(2), rtol=1e-5, atol=0)
+    # the next product normalizes x's rows from those sums
+    N2 = 512
+    W2 = rand_bf16((N2, N), 133, N ** -0.5).cuda()
+    out = linear(davet, x, W2, row_ss=ss, row_ss_parts=parts, row_ss_eps=1e-5)
+    check_close(out, L.rmsnorm(f64(x), np.ones(N), 1e-5) @ f64(W2).T, "normalized by ss_out")
