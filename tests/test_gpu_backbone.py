@@ -28,9 +28,14 @@ def oracle_inputs(bb, feats, prompts, t):
         lvl = int(w.schedule[t, b])
         parts = []
         if w.tiles[b]:
-            pyr = oracle.pyramid(feats[b], w.tiles[b], w.grid, w.n_levels, C)
-            off = oracle.level_offsets(w.grid, w.n_levels, w.tiles[b])
-            view = torch.from_numpy(pyr[off[lvl]:off[lvl + 1]]).to(torch.bfloat16)
+            pyr = torch.from_numpy(oracle.pyramid(feats[b], w.tiles[b], w.grid, w.n_levels, C)).to(torch.bfloat16)
+            if lvl < w.n_levels:
+                off = oracle.level_offsets(w.grid, w.n_levels, w.tiles[b])
+                view = pyr[off[lvl]:off[lvl + 1]]
+            else:  # the mixed view, from the oracle's own bf16 pyramid
+                bits = oracle.mixed_view(pyr.view(torch.int16).numpy().view(np.uint16), w.tiles[b], w.grid,
+                                         w.n_levels, *w.mixed, C)
+                view = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16)
             parts.append(f64(view))
         parts.append(f64(prompts[b]))
         parts.append(np.repeat(f64(bb.emb[bb.mask_id:bb.mask_id + 1]), w.resp[b], axis=0))
@@ -53,12 +58,15 @@ def layer_weights(p, F):
                 wg=gu[:, 0].reshape(F, C), wu=gu[:, 1].reshape(F, C), wd=f64(p["wd"]))
 
 
-@pytest.mark.parametrize("t,device_rows", [(0, False), (2, False), (5, False), (2, True), (5, True)])
-def test_tiny_two_layer_step_logits(davet, t, device_rows):
+@pytest.mark.parametrize("name,t,device_rows", [("tiny", 0, False), ("tiny", 2, False), ("tiny", 5, False),
+                                                ("tiny", 2, True), ("tiny", 5, True), ("tiny_mixed", 2, False),
+                                                ("tiny_mixed", 3, True)])
+def test_tiny_two_layer_step_logits(davet, name, t, device_rows):
     """device_rows: the policy's launch mode, every kernel launched for the
     largest view and reading the step's row count on the device (the step's
-    view still comes from the workload's schedule here)."""
-    w = workloads.make("tiny")
+    view still comes from the workload's schedule here).  tiny_mixed steps 2
+    and 3 take the mixed view (coarse rows plus the level-0 lattice)."""
+    w = workloads.make(name)
     bb = Backbone(w, 2, lib=davet)
     if device_rows:
         bb.use_policy()

@@ -463,7 +463,8 @@ def test_linear_folded_rmsnorm(davet, M, K, N, epi, split):
     assert np.allclose(ss.cpu().numpy()[:, 0], (f64(A) ** 2).sum(1), rtol=1e-5)
 
 
-@pytest.mark.parametrize("M,K,N,parts_from_split", [(333, 512, 768, False), (241, 4096, 4096, True)])
+@pytest.mark.parametrize("M,K,N,parts_from_split", [(100, 256, 512, False), (333, 512, 768, False),
+                                                    (241, 4096, 4096, True)])
 def test_linear_sums_of_squares_out_feed_the_next_product(davet, M, K, N, parts_from_split):
     """A residual projection emits each row's sums of squares per 256 columns
     (ss_out); they are the sums of the stored bf16 values, and as row_ss of
