@@ -178,7 +178,8 @@ def run_ours(args, rank, world, local_rank):
         view_level = workloads.policy_view_levels(w)
         lo = torch.empty((w.batch, w.T), dtype=torch.float64, device=dev)
         up = torch.empty_like(lo)
-        demand = torch.tensor(workloads.request_demands(w), dtype=torch.float64, device=dev)
+        demand = (None if args.uniform_demand else
+                  torch.tensor(workloads.request_demands(w), dtype=torch.float64, device=dev))
         budget = torch.zeros((w.T, w.batch), dtype=torch.float64, device=dev)
 
     def policy_pass():
@@ -340,7 +341,7 @@ def run_backbone(args, rank, world, local_rank):
         w.seed = w.seed + 1000 * rank
     bb = Backbone(w, args.layers, dev, lib)
     if args.policy:
-        bb.use_policy(args.orientation, args.budget, args.rho, args.alpha)
+        bb.use_policy(args.orientation, args.budget, args.rho, args.alpha, args.uniform_demand)
     feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C),
                                    workloads.derive_seed(w.seed, workloads.KIND_FEAT, b)) for b in range(w.batch)]
     prompts = [workloads.normal_bf16((w.prompt[b], bb.C), workloads.derive_seed(w.seed, workloads.KIND_TEXT, b))
@@ -499,7 +500,8 @@ def policy_summary(args, w, sched, budget):
     from paper_2608_01821_gb300 import workloads
     views, counts = np.unique(sched, return_counts=True)
     return {"orientation": args.orientation, "B": args.budget, "rho": args.rho, "alpha": args.alpha,
-            "view_levels": workloads.policy_view_levels(w), "demand": workloads.request_demands(w),
+            "view_levels": workloads.policy_view_levels(w),
+            "demand": [1.0] * w.batch if args.uniform_demand else workloads.request_demands(w),
             "mean_budget": round(float(budget.mean().item()), 4),
             "steps_per_view": {int(v): int(c) for v, c in zip(views, counts)}}
 
@@ -1035,6 +1037,8 @@ def main(argv=None):
     ap.add_argument("--budget", type=float, default=0.75, help="average budget B")
     ap.add_argument("--rho", type=float, default=0.20)
     ap.add_argument("--alpha", type=float, default=1.0)
+    ap.add_argument("--uniform-demand", action="store_true",
+                    help="with --policy: d(o) = 1 for every request instead of the Table A prior")
     ap.add_argument("--model", choices=["core", "full"], default="core",
                     help="core: the step-conditioning path (attention core); full: every step runs --layers "
                          "synthetic-weight backbone layers and the LM head")

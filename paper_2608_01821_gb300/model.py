@@ -136,17 +136,20 @@ class Backbone:
         self.gemm_ws = torch.empty(max(gw, 256), dtype=torch.uint8, device=dev)
         self.policy = None
 
-    def use_policy(self, orientation: str = "early", B: float = 0.75, rho: float = 0.2, alpha: float = 1.0):
+    def use_policy(self, orientation: str = "early", B: float = 0.75, rho: float = 0.2, alpha: float = 1.0,
+                   uniform_demand: bool = False):
         """Choose every step's view with the closed-loop allocation policy:
         the budget envelope (Eq. 6-7) at the start of each pass, the view of
-        step t from step t-1's unmasking statistics (Eq. 8-9)."""
+        step t from step t-1's unmasking statistics (Eq. 8-9).  The demand
+        prior d(o) comes from Table A by request, or is 1 for every request
+        (uniform_demand, the paper's ablation of the prior)."""
         if orientation not in ("early", "late"):
             raise ValueError("orientation is 'early' or 'late'")
         w, dev = self.w, self.dev
         self.policy = dict(orientation=orientation, B=B, rho=rho, alpha=alpha, view_levels=policy_view_levels(w))
         self.lo = torch.empty((w.batch, w.T), dtype=torch.float64, device=dev)
         self.up = torch.empty_like(self.lo)
-        self.demand = torch.tensor(request_demands(w), dtype=torch.float64, device=dev)
+        self.demand = None if uniform_demand else torch.tensor(request_demands(w), dtype=torch.float64, device=dev)
         self.budget = torch.zeros((w.T, w.batch), dtype=torch.float64, device=dev)
 
     # -------------------------------------------------------------- inputs
