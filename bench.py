@@ -612,7 +612,10 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
         out = {
             "timing_mode": mode,
             "pyramid": {"launches": nb, "ms": ms["pyramid"], "bytes": pbytes,
-                        "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9},
+                        "GBps": pbytes / (ms["pyramid"] * 1e-3) / 1e9,
+                        # with the view blocks' text copies (and mixed rows) the fill adds
+                        "bytes_with_fill": pbytes + w.view_fill_bytes(),
+                        "GBps_with_fill": (pbytes + w.view_fill_bytes()) / (ms["pyramid"] * 1e-3) / 1e9},
         }
     else:
         out = {

@@ -190,6 +190,16 @@ class Workload:
         rows_out = sum(self.tiles) * sum(g * g for g in sides[1:])
         return float((rows_in + rows_out) * self.C * 2)
 
+    def view_fill_bytes(self) -> float:
+        """Bytes the view-block fill moves (read + write, bf16): every view
+        block's copy of the request's text rows, and the mixed view's rows."""
+        rows = 0
+        for b in range(self.batch):
+            rows += self.n_views() * (self.prompt[b] + self.resp[b])
+            if self.mixed:
+                rows += self.tiles[b] * self.view_rows_per_tile(self.n_levels)
+        return float(rows * self.C * 2 * 2)
+
     def masked_rows(self, t: int) -> int:
         """|M_t| summed over requests when k positions are committed per step."""
         return sum(max(r - self.k * t, 0) for r in self.resp)
