@@ -117,13 +117,16 @@ def test_closed_loop_commits_every_position(davet):
     assert ((tok[flat] >= 0) & (tok[flat] < w.V)).all()
 
 
-def test_policy_closed_loop(davet):
+@pytest.mark.parametrize("orientation,B,rho,alpha,uniform", [("early", 0.75, 0.2, 1.0, False),
+                                                             ("late", 0.45, 0.2, 0.5, True)])
+def test_policy_closed_loop(davet, orientation, B, rho, alpha, uniform):
     """The allocation policy picks every step's view on the device from the
     previous step's statistics; the steps run the rows of the views it picked
-    (cu_seqlens of the last step) and the loop commits every position."""
+    (cu_seqlens of the last step) and the loop commits every position.  The
+    budgets stay inside the envelope's bounds (Eq. 8 interpolates them)."""
     w = workloads.make("tiny")
     bb = Backbone(w, 1, lib=davet)
-    bb.use_policy("early", 0.75, 0.2, 1.0)
+    bb.use_policy(orientation, B, rho, alpha, uniform_demand=uniform)
     feats = [workloads.normal_bf16((w.tiles[b], w.grid, w.grid, bb.C), 500 + b) for b in range(w.batch)]
     prompts = [workloads.normal_bf16((w.prompt[b], bb.C), 600 + b) for b in range(w.batch)]
     bb.load_inputs(feats, prompts)
@@ -140,5 +143,7 @@ def test_policy_closed_loop(davet):
     assert [int(cu[b + 1] - cu[b]) for b in range(w.batch)] == [w.seq_len(b, int(v)) for b, v in enumerate(sched[-1])]
     committed = bb.committed.cpu().numpy().reshape(-1)
     assert len(set(committed.tolist())) == len(committed) == w.T * w.k
-    budget = bb.budget.cpu().numpy()
+    budget = bb.budget.cpu().numpy()  # [T][batch]
+    lo, up = bb.lo.cpu().numpy().T, bb.up.cpu().numpy().T  # [T][batch]
+    assert ((budget >= lo - 1e-12) & (budget <= up + 1e-12)).all()
     assert ((budget >= 0) & (budget <= 1)).all()
