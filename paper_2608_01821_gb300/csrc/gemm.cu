@@ -26,6 +26,14 @@
 // angle from a cos/sin table indexed by the row's position in its request;
 // the table is frequency-major, so the lanes of a warp, rows at consecutive
 // positions, read consecutive entries).
+// Around every epilogue: an optional row scale 1/rms from partial sums of
+// squares (an RMS normalization of A folded into the product, its gain in W)
+// and, for the store and residual epilogues, the sums of squares of the
+// stored rows per 256 columns (the next product's normalization input).
+// M > 128 runs on CTA pairs (gemm2_kernel below), with a K split into fp32
+// partials and a reduction kernel when the tiles leave most pairs idle.
+// A row count on the device (rows_dev) limits every kernel to the rows the
+// step has; each kernel keeps it in a scalar of its own.
 #include <algorithm>
 #include <mutex>
 
