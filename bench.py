@@ -137,7 +137,6 @@ class ClockSampler:
 
 # ------------------------------------------------------------- our arm
 def run_ours(args, rank, world, local_rank):
-    import numpy as np
     import torch
 
     from paper_2608_01821_gb300 import davet, workloads
