@@ -328,7 +328,7 @@ namespace pyr {
 davet_status enqueue(const void* feat, void* pyr, int n_tiles, int grid, int n_levels, int C, float* pyr_f32,
                      const int64_t* off, int64_t extent, cudaStream_t st) {
   Geom g;
-  int side[kMaxLevels];
+  int side[kMaxLevels] = {};
   davet_pyramid_layout(grid, n_levels, n_tiles, side, nullptr);
   for (int l = 0; l < kMaxLevels; ++l) g.side[l] = l < n_levels ? side[l] : 1;
   for (int l = 0; l <= kMaxLevels; ++l) g.off[l] = l < n_levels ? off[l] : extent;
