@@ -489,3 +489,43 @@ def test_linear_sums_of_squares_out_feed_the_next_product(davet, M, K, N, parts_
     W2 = rand_bf16((N2, N), 133, N ** -0.5).cuda()
     out = linear(davet, x, W2, row_ss=ss, row_ss_parts=parts, row_ss_eps=1e-5)
     check_close(out, L.rmsnorm(f64(x), np.ones(N), 1e-5) @ f64(W2).T, "normalized by ss_out")
+
+
+@pytest.mark.parametrize("M,m,K,N", [(100, 37, 256, 512), (300, 150, 512, 768), (241, 97, 4096, 4096)])
+def test_norm_fold_with_device_row_count(davet, M, m, K, N):
+    """Sums of squares out and the folded normalization in, with the row count
+    read on the device: rows from m on keep their contents and their sums."""
+    A = rand_bf16((M, K), 140 + M).cuda()
+    W = rand_bf16((N, K), 141, K ** -0.5).cuda()
+    R = rand_bf16((M, N), 142).cuda()
+    rows_dev = torch.tensor([m], dtype=torch.int32, device="cuda")
+    ws = torch.empty(max(davet.davet_linear_workspace_bytes(M, K, N), 256), dtype=torch.uint8, device="cuda")
+    parts = N // 256
+    x = R.clone()
+    ss = torch.full((M, parts), float("nan"), dtype=torch.float32, device="cuda")
+    davet.davet_linear(A, M, K, W, N, x, davet.EPI_RESIDUAL, x, workspace=ws, ss_out=ss, rows_dev=rows_dev)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    assert torch.equal(x[m:], R[m:]) and torch.isnan(ss[m:]).all()
+    check_close(x[:m], f64(R[:m]) + f64(A[:m]) @ f64(W).T, "residual rows_dev")
+    assert np.allclose(ss[:m].cpu().numpy(), (f64(x[:m]).reshape(m, parts, 256) ** 2).sum(2), rtol=1e-5, atol=0)
+    # the next product over the same rows, normalized from those sums
+    W2 = rand_bf16((512, N), 143, N ** -0.5).cuda()
+    out = torch.full((M, 512), -7.0, dtype=torch.bfloat16, device="cuda")
+    ws2 = torch.empty(max(davet.davet_linear_workspace_bytes(M, N, 512), 256), dtype=torch.uint8, device="cuda")
+    davet.davet_linear(x, M, N, W2, 512, out, workspace=ws2, row_ss=ss, row_ss_parts=parts, row_ss_eps=1e-5,
+                       rows_dev=rows_dev)
+    torch.cuda.synchronize()
+    assert davet.davet_device_status() == (0, 0)
+    assert (out[m:].float() == -7.0).all()
+    check_close(out[:m], L.rmsnorm(f64(x[:m]), np.ones(N), 1e-5) @ f64(W2).T, "normalized rows_dev")
+
+
+def test_row_sumsq_device_row_count(davet):
+    M, C, m = 90, 4096, 33
+    x = rand_bf16((M, C), 144, 2.0).cuda()
+    ss = torch.full((M, 1), float("nan"), dtype=torch.float32, device="cuda")
+    davet.davet_row_sumsq(x, M, C, ss, rows_dev=torch.tensor([m], dtype=torch.int32, device="cuda"))
+    torch.cuda.synchronize()
+    assert torch.isnan(ss[m:]).all()
+    assert np.allclose(ss[:m, 0].cpu().numpy(), (f64(x[:m]) ** 2).sum(1), rtol=1e-5)
