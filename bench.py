@@ -32,7 +32,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "step attention TFLOP/s (% bf16 peak); pyramid/unmask HBM GB/s; steps/s"
-DEFAULT_CONFIG = "single"
+DEFAULT_CONFIG = "highres"
 L2_FLUSH_BYTES = 512 << 20
 
 
@@ -240,7 +240,10 @@ def run_ours(args, rank, world, local_rank):
         raise RuntimeError(f"device error word {flags:#x} after the timed region")
 
     # ------------------------------------ per-kernel times (eager, events)
-    comp = kernel_times(pl, w, pool, P, stream)
+    comp = kernel_times(pl, w, pool, P, stream, flush, policy_pass=policy_pass if policy else None,
+                        policy_step=policy_step if policy else None)
+    comp["pass_ms"] = statistics.mean(pass_ms)
+    comp["sum_vs_pass"] = comp["sum_ms"] / comp["pass_ms"]
 
     # ---------------------------------------------------------- e2e
     e2e = None if args.no_e2e else run_e2e(args, pl, w, dev, stream, world,
@@ -431,8 +434,11 @@ def run_backbone(args, rank, world, local_rank):
         torch.cuda.synchronize()
         te = allreduce_max(s0.elapsed_time(s1) / 1e3, world, dev)
         h2d = sum(f.numel() * 2 for f in pf) + sum(p.numel() * 2 for p in pp)
-        e2e = {"value": round(w.T * n * world / te, 3), "unit": "denoising steps/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(w.total_resp * 4), "passes": n}
+        d2h = w.total_resp * 4
+        e2e = {"value": round(w.T * n * world / te, 3), "unit": "denoising steps/s",
+               "h2d_bytes_per_step": int(round(h2d / w.T)), "d2h_bytes_per_step": int(round(d2h / w.T)),
+               "h2d_bytes_per_pass": int(h2d), "d2h_bytes_per_pass": int(d2h), "passes": n,
+               "bytes_note": "per denoising step = per pass / T (inputs and tokens cross once per pass)"}
 
     if rank != 0:
         return None
@@ -538,69 +544,77 @@ def build_launches(w, realizer: str, fused: bool) -> int:
     return n
 
 
-def kernel_times(pl, w, pool, P, stream, reps=3):
-    """Average device time per call of each kernel.
+def kernel_times(pl, w, pool, P, stream, flush, reps=3, policy_pass=None, policy_step=None):
+    """Average device time of each kind of kernel over one pass.
 
-    The pass is captured once more into a CUDA graph with an event record
-    node before and after every library call, so each interval is the
-    kernel(s) of that call plus graph scheduling, without host launch
-    overhead; the graph is replayed `reps` times and the intervals summed.
-    Falls back to eager events when the event type cannot be captured."""
+    Every kind's calls of one pass are captured into a CUDA graph of their
+    own, in pass order and with nothing between them (so the kernels chain
+    with programmatic dependent launch as they do in the pass): the view
+    construction; the T step attentions (or gathers and attentions); the
+    answer-state reset followed by the T unmaskings; the allocation policy's
+    steps when it runs.  Each graph is replayed `reps` times between CUDA
+    events on the launching stream, L2 evicted before every replay as before
+    every timed pass.  The answer-state reset (three fills) is timed alone
+    and taken out of the unmasking.  `sum_ms` against the pass time shows
+    how well the parts add up."""
     import torch
 
-    def mk():
-        try:
-            return torch.cuda.Event(enable_timing=True, external=True)
-        except TypeError:
-            return None
+    def graph_of(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        return g
 
-    probe = mk()
-    calls = []  # (kind, start, end)
-    ev = []
+    def time_graph(g):
+        t = 0.0
+        with torch.cuda.stream(stream):
+            for i in range(reps):
+                flush.fill_(i & 0xFF)
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                g.replay()
+                b.record(stream)
+                b.synchronize()
+                t += a.elapsed_time(b)
+        return t / reps
 
-    def timed(kind, fn):
-        a, b = mk(), mk()
-        a.record(stream)
-        fn()
-        b.record(stream)
-        calls.append((kind, a, b))
-
-    def instrumented_pass():
-        pl.reset_state()
-        timed("pyramid", pl.build_pyramids)
+    def attn_all():
         for t in range(w.T):
             if pl.fused:
-                timed("view_attention", lambda t=t: pl.view_attention(t))
+                pl.view_attention(t)
             else:
-                timed("gather", lambda t=t: pl.gather(t))
-                timed("attention", pl.attention)
-            timed("unmask", lambda t=t: pl.unmask(t, pool[t % P]))
+                pl.gather(t)
+                pl.attention()
 
-    totals = {"pyramid": 0.0, "gather": 0.0, "attention": 0.0, "unmask": 0.0, "view_attention": 0.0}
-    mode = "graph"
-    if probe is not None:
-        try:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                instrumented_pass()
-            for _ in range(reps):
-                g.replay()
-                torch.cuda.synchronize()
-                for kind, a, b in calls:
-                    totals[kind] += a.elapsed_time(b) / reps
-        except Exception:
-            probe = None
-            totals = {k: 0.0 for k in totals}
-            calls.clear()
-    if probe is None:
-        mode = "eager"
-        with torch.cuda.stream(stream):
-            def mk():  # noqa: F811
-                return torch.cuda.Event(enable_timing=True)
-            instrumented_pass()
-        torch.cuda.synchronize()
-        for kind, a, b in calls:
-            totals[kind] += a.elapsed_time(b)
+    def gather_all():
+        for t in range(w.T):
+            pl.gather(t)
+
+    def unmask_all():
+        pl.reset_state()
+        for t in range(w.T):
+            pl.unmask(t, pool[t % P])
+
+    def policy_all():
+        policy_pass()
+        for t in range(w.T):
+            policy_step(t)
+
+    graphs = {"pyramid": graph_of(pl.build_pyramids), "reset": graph_of(pl.reset_state),
+              "unmask": graph_of(unmask_all)}
+    if pl.fused:
+        graphs["view_attention"] = graph_of(attn_all)
+    else:
+        graphs["gather"] = graph_of(gather_all)
+        graphs["gather+attention"] = graph_of(attn_all)
+    if policy_pass is not None:
+        graphs["policy"] = graph_of(policy_all)
+    torch.cuda.synchronize()
+    totals = {k: time_graph(g) for k, g in graphs.items()}
+    totals["unmask"] = max(totals["unmask"] - totals["reset"], 0.0)
+    if not pl.fused:
+        totals["attention"] = max(totals.pop("gather+attention") - totals["gather"], 0.0)
+    mode = "per-kind CUDA graphs (the pass's calls of one kind, chained as in the pass)"
     ms = totals
     flops = sum(w.attention_flops(t) for t in range(w.T))
     gbytes = sum(w.gather_bytes(t) for t in range(w.T))
@@ -632,6 +646,10 @@ def kernel_times(pl, w, pool, P, stream, reps=3):
                             "TFLOPs": flops / (ms["attention"] * 1e-3) / 1e12}
     out["unmask"] = {"launches": 2 * w.T, "ms": ms["unmask"], "bytes": ubytes,
                      "GBps": ubytes / (ms["unmask"] * 1e-3) / 1e9}
+    out["reset"] = {"launches": 3, "ms": ms["reset"], "what": "answer-state reset (torch fills)"}
+    if "policy" in ms:
+        out["policy"] = {"launches": 1 + w.T, "ms": ms["policy"]}
+    out["sum_ms"] = sum(v for k, v in ms.items())
     return out
 
 
@@ -769,8 +787,9 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
         e.record(stream)
     torch.cuda.synchronize()
     t = allreduce_max(s.elapsed_time(e) / 1e3, world, dev)
-    return {"value": round(w.T * n * world / t, 3), "unit": "denoising steps/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "passes": n, "mode": mode,
+    return {"value": round(w.T * n * world / t, 3), "unit": "denoising steps/s",
+            "h2d_bytes_per_step": int(round(h2d / w.T)), "d2h_bytes_per_step": int(round(d2h / w.T)),
+            "h2d_bytes_per_pass": int(h2d), "d2h_bytes_per_pass": int(d2h), "passes": n, "mode": mode,
             "h2d_GBps": round(h2d * n / t / 1e9, 1)}
 
 

@@ -477,17 +477,29 @@ davet_status davet_stage_masked_rows(const void* src, int V, const uint8_t* mask
  * call cudaMalloc because it can synchronize the device and stall the
  * pipeline.
  *
- * Computes exactly what davet_unmask_topk computes, with the same arguments
- * except the workspace.  Instead of a caller workspace it uses one scratch
- * array of DAVET_NOALLOC_SCRATCH_BYTES (1 MiB) that the library places in
- * device global memory; every device that loads the library holds that array
- * until the process exits.  The call allocates nothing.
- *   - Limit: sizes whose workspace (davet_unmask_topk_workspace) exceeds
- *     DAVET_NOALLOC_SCRATCH_BYTES are rejected with DAVET_ERR_UNSUPPORTED
- *     before anything is enqueued (about 43,000 answer rows).
- *   - Set-up: the first call on each device looks up the array's device
- *     address (cudaGetSymbolAddress) with that device current and caches it;
- *     make that first call before any stream capture.
+ * Computes what davet_unmask_topk computes, with the same arguments except
+ * the workspace.  Instead of a caller workspace it uses one scratch array of
+ * DAVET_NOALLOC_SCRATCH_BYTES (1 MiB) that the library places in device
+ * global memory; every device that loads the library holds that array until
+ * the process exits.  The call allocates nothing.
+ *   - Layout and limit: the scratch holds, per answer row, one 16-byte
+ *     (max, sum, first index) record per vocabulary chunk, then a 4-byte
+ *     confidence and a 4-byte index; each of these three arrays starts on a
+ *     256-byte boundary.  When the chunk count that davet_unmask_topk uses
+ *     (8 KB of logits per chunk, at most 64 chunks) does not fit, this call
+ *     cuts each row into fewer, longer chunks until it fits.  The argmax,
+ *     the tokens and the committed rows are the same as davet_unmask_topk's;
+ *     the confidences and statistics agree to fp32 rounding (the chunk sums
+ *     are added in a different grouping).  At V = 126464 the standard 31
+ *     chunks fit up to 2,080 answer rows.  Only a size that does not fit
+ *     even with one chunk per row (24 bytes per row: above 43,680 rows) is
+ *     rejected, with DAVET_ERR_UNSUPPORTED, before anything is enqueued.
+ *   - Set-up: the array's device address is looked up with
+ *     cudaGetSymbolAddress, with the device current, at the first call in
+ *     each CUDA context (a device's primary context, or another context the
+ *     caller made current) and kept for that context; a context created
+ *     later (for example after cudaDeviceReset) gets its own look-up.  Make
+ *     the first call in a context before any stream capture.
  *   - Sharing: every call on a device uses the same array, and the array keeps
  *     whatever the last call left in it.  Nothing in it needs clearing: a call
  *     writes every scratch entry it later reads.  Calls whose kernels overlap
@@ -539,8 +551,9 @@ davet_status davet_unmask_topk_noalloc(const void* logits, int V, const int32_t*
  *            time.
  *   rows_dev device int32, nullable: the row count to compute, read on the
  *            device when the kernels start (after the previous work on
- *            `stream`), clamped to [0, M]; rows from there on are neither read
- *            for the epilogue nor written.  M is then the capacity: A, out
+ *            `stream`), clamped to [0, M] (a count above M flags
+ *            DAVET_DEV_CAPACITY, a negative one DAVET_DEV_ARG); rows from
+ *            there on are neither read for the epilogue nor written.  M is then the capacity: A, out
  *            and the residual hold M rows, and the tiling and workspace are
  *            chosen for M.  Lets a captured step run a row count that
  *            earlier kernels decide (the allocation policy's views).

@@ -109,13 +109,21 @@ __device__ __forceinline__ float row_scale(const Params& p, long long row, bool 
   return rsqrtf(t / static_cast<float>(p.K) + p.rss_eps);
 }
 
+// A device row count clamped to [0, M]; a count outside that range sets a
+// bit of the device error word (capacity above M, argument below 0), raised
+// by one thread per block.
+__device__ __forceinline__ long long clamp_rows(const int32_t* rows_dev, long long M, unsigned* err) {
+  const long long m = *rows_dev;
+  if ((m < 0 || m > M) && threadIdx.x == 0) raise_error(err, m < 0 ? DEV_ERR_ARG : DEV_ERR_CAPACITY);
+  return m < 0 ? 0 : (m < M ? m : M);
+}
+
 // The launch's row count: M, or the smaller count on the device.  Kernels
 // keep it in a scalar of their own rather than in their copy of the
 // parameters.
 __device__ __forceinline__ long long rows_now(const Params& p) {
   if (!p.rows_dev) return p.M;
-  const long long m = *p.rows_dev;
-  return m < 0 ? 0 : (m < p.M ? m : p.M);
+  return clamp_rows(p.rows_dev, p.M, p.err);
 }
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0, int c1) {
@@ -896,13 +904,10 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const uint16_t* __restrict
                                                       const uint16_t* __restrict__ gamma, float eps,
                                                       uint16_t* __restrict__ out, const int32_t* cu,
                                                       const int32_t* cu_resp, int batch,
-                                                      const int32_t* __restrict__ rows_dev) {
+                                                      const int32_t* __restrict__ rows_dev, unsigned* err) {
   pdl_launch_dependents();
   pdl_wait();
-  if (rows_dev) {
-    const long long m = *rows_dev;
-    M = m < 0 ? 0 : (m < M ? m : M);
-  }
+  if (rows_dev) M = clamp_rows(rows_dev, M, err);
   const int lane = threadIdx.x & 31;
   const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
@@ -947,13 +952,11 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const uint16_t* __restrict
 // Sum of squares of each row's bf16 values (fp32, one warp per row, lanes in
 // a shuffle tree): the normalization input of the first projection.
 __global__ void __launch_bounds__(256) row_sumsq_kernel(const uint16_t* __restrict__ x, long long M, int C,
-                                                        float* __restrict__ ss, const int32_t* __restrict__ rows_dev) {
+                                                        float* __restrict__ ss, const int32_t* __restrict__ rows_dev,
+                                                        unsigned* err) {
   pdl_launch_dependents();
   pdl_wait();
-  if (rows_dev) {
-    const long long m = *rows_dev;
-    M = m < 0 ? 0 : (m < M ? m : M);
-  }
+  if (rows_dev) M = clamp_rows(rows_dev, M, err);
   const int lane = threadIdx.x & 31;
   const long long w0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long nw = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
@@ -1231,6 +1234,8 @@ extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const voi
   if (!x || !gamma || !out || !aligned16(x) || !aligned16(gamma) || !aligned16(out)) return DAVET_ERR_INVALID_ARG;
   const bool answers = cu_resp != nullptr;
   if (answers && (!cu_seqlens || batch < 1)) return DAVET_ERR_INVALID_ARG;
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
   const int blocks = static_cast<int>(std::min<long long>((M + 7) / 8, 152LL * 16));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const uint16_t* xs = static_cast<const uint16_t*>(x);
@@ -1238,9 +1243,9 @@ extern "C" davet_status davet_rmsnorm(const void* x, int64_t M, int C, const voi
   uint16_t* os = static_cast<uint16_t*>(out);
   const cudaError_t e =
       answers ? launch(rmsnorm_kernel<true>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs, eps,
-                       os, cu_seqlens, cu_resp, batch, rows_dev)
+                       os, cu_seqlens, cu_resp, batch, rows_dev, err)
               : launch(rmsnorm_kernel<false>, dim3(blocks), dim3(256), 0, st, xs, static_cast<long long>(M), C, gs,
-                       eps, os, cu_seqlens, cu_resp, batch, rows_dev);
+                       eps, os, cu_seqlens, cu_resp, batch, rows_dev, err);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }
@@ -1250,9 +1255,11 @@ extern "C" davet_status davet_row_sumsq(const void* x, int64_t M, int C, float* 
   if (M < 0 || C < 8 || C % 8 != 0) return DAVET_ERR_INVALID_ARG;
   if (M == 0) return DAVET_OK;
   if (!x || !ss_out || !aligned16(x)) return DAVET_ERR_INVALID_ARG;
+  unsigned* err = device_error_word();
+  if (!err) return DAVET_ERR_CUDA;
   const int blocks = static_cast<int>(std::min<long long>((M + 7) / 8, 152LL * 16));
   const cudaError_t e = launch(row_sumsq_kernel, dim3(blocks), dim3(256), 0, static_cast<cudaStream_t>(stream),
-                               static_cast<const uint16_t*>(x), static_cast<long long>(M), C, ss_out, rows_dev);
+                               static_cast<const uint16_t*>(x), static_cast<long long>(M), C, ss_out, rows_dev, err);
   if (e != cudaSuccess) return cuda_fail(e);
   return check_launch();
 }

@@ -554,12 +554,46 @@ constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;  // DAVET_NOALLOC_SCRAT
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 constexpr int kNoAllocMaxDevices = 64;
-static uint8_t* g_noalloc_addr[kNoAllocMaxDevices] = {};
+
+// The array's device address, kept per device together with the unique id
+// of the CUDA context it was looked up in (0: none yet).
+struct NoAllocAddr {
+  unsigned long long ctx_id;
+  uint8_t* ptr;
+};
+static NoAllocAddr g_noalloc_addr[kNoAllocMaxDevices] = {};
 static std::mutex g_noalloc_mu;
 
-// Device address of g_noalloc_scratch on the current device.  Host code only
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Unique id of the calling thread's current context, 0 when there is none
+// yet (the runtime creates the primary context at its first device call).
+static unsigned long long current_ctx_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx) return 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of g_noalloc_scratch in the current context.  Host code only
 // sees a host-side stand-in for the array under its name, so the address is
-// asked for once per device, with that device current, and cached.
+// asked for with the device current, once per context, and kept.
 static uint8_t* noalloc_scratch(davet_status* st) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -572,16 +606,20 @@ static uint8_t* noalloc_scratch(davet_status* st) {
     return nullptr;
   }
   std::lock_guard<std::mutex> g(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
+  NoAllocAddr& a = g_noalloc_addr[dev];
+  const unsigned long long id = current_ctx_id();
+  if (id == 0 || a.ctx_id != id || !a.ptr) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) {
       *st = cuda_fail(e);
       return nullptr;
     }
-    g_noalloc_addr[dev] = static_cast<uint8_t*>(p);
+    a.ptr = static_cast<uint8_t*>(p);
+    // the look-up made the context current if there was none
+    a.ctx_id = current_ctx_id();
   }
-  return g_noalloc_addr[dev];
+  return a.ptr;
 }
 
 }  // namespace unm

@@ -529,3 +529,45 @@ def test_row_sumsq_device_row_count(davet):
     torch.cuda.synchronize()
     assert torch.isnan(ss[m:]).all()
     assert np.allclose(ss[:m, 0].cpu().numpy(), (f64(x[:m]) ** 2).sum(1), rtol=1e-5)
+
+
+@pytest.mark.parametrize("m,flag", [(-3, 0x4), (250, 0x2)])
+def test_device_row_count_out_of_range_is_flagged(davet, m, flag):
+    """A device row count outside [0, M] is clamped (to 0 or M) and sets a bit
+    of the device error word: capacity above M, argument below 0.  Covers the
+    one-CTA and pair products, the RMS normalization and the sums of squares."""
+    K, N = 256, 512
+    rows_dev = torch.tensor([m], dtype=torch.int32, device="cuda")
+    mm = min(max(m, 0), 200)
+    for M in (100, 200):  # one-CTA tiles, CTA pairs
+        mc = min(max(m, 0), M)
+        A = rand_bf16((M, K), 150 + M).cuda()
+        W = rand_bf16((N, K), 151, K ** -0.5).cuda()
+        out = torch.full((M, N), -7.0, dtype=torch.bfloat16, device="cuda")
+        ws = torch.empty(max(davet.davet_linear_workspace_bytes(M, K, N), 256), dtype=torch.uint8, device="cuda")
+        davet.davet_device_status(clear=True)
+        davet.davet_linear(A, M, K, W, N, out, workspace=ws, rows_dev=rows_dev)
+        torch.cuda.synchronize()
+        st, flags = davet.davet_device_status(clear=True)
+        assert flags & flag, (M, m, flags)
+        assert (out[mc:].float() == -7.0).all()
+        if mc:
+            check_close(out[:mc], f64(A[:mc]) @ f64(W[:]).T, "clamped rows_dev")
+    M, C = 200, 1024
+    x = rand_bf16((M, C), 152).cuda()
+    g = torch.ones(C, dtype=torch.bfloat16, device="cuda")
+    y = torch.full((M, C), -7.0, dtype=torch.bfloat16, device="cuda")
+    davet.davet_rmsnorm(x, M, C, g, 1e-5, y, rows_dev=rows_dev)
+    torch.cuda.synchronize()
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags & flag
+    assert (y[mm:].float() == -7.0).all()
+    ss = torch.full((M, 1), float("nan"), dtype=torch.float32, device="cuda")
+    davet.davet_row_sumsq(x, M, C, ss, rows_dev=rows_dev)
+    torch.cuda.synchronize()
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags & flag
+    assert torch.isnan(ss[mm:]).all()
+    if mm:
+        assert np.allclose(ss[:mm, 0].cpu().numpy(), (f64(x[:mm]) ** 2).sum(1), rtol=1e-5)
+    assert davet.davet_device_status() == (0, 0)

@@ -1,7 +1,10 @@
-"""End-to-end parity of the step sequence (pyramid once, then per step
-gather -> attention -> unmask) against the oracle chain, on the tiny workload
-for every step and on the 8B-class workloads for sampled steps, in the same
-launch configuration the benchmark times (the Pipeline class)."""
+"""End-to-end parity of the step sequence against the oracle chain, on the
+tiny workload for every step and on the 8B-class workloads for sampled
+steps, through the Pipeline class the benchmark times, in both layouts:
+fused (the benchmark's default: view blocks built once, then per step the
+view attention, which reads each request's sequence from its view block,
+and the unmasking) and unfused (pyramid once, then per step gather ->
+attention -> unmask)."""
 import numpy as np
 import pytest
 import torch
@@ -14,7 +17,7 @@ from paper_2608_01821_gb300.pipeline import Pipeline
 pytestmark = pytest.mark.gpu
 
 
-def make_pipeline(davet, w, fused=False):
+def make_pipeline(davet, w, fused=True):
     pl = Pipeline(w, "cuda", davet, fused=fused)
     feats = [workloads.features(w, b) for b in range(w.batch)]
     text = workloads.text_rows(w)
@@ -98,13 +101,38 @@ def test_tiny_workload_every_step(davet, name, fused):
     assert masked.sum() == 0
 
 
+def sampled_views(w):
+    """The step views a full-size check covers: up to four distinct scheduled
+    ones (per-request view vectors), then every request on the high view
+    (level 0) and every request on the coarsest pooled level the schedule
+    uses."""
+    views, seen = [], set()
+    for t in range(w.T):
+        key = tuple(int(x) for x in w.schedule[t])
+        if key not in seen:
+            seen.add(key)
+            views.append(key)
+    views = views[:4]
+    pooled = [int(x) for x in np.unique(w.schedule) if x < w.n_levels]
+    for lvl in (0, max(pooled)):
+        key = (lvl,) * w.batch
+        if key not in seen:
+            seen.add(key)
+            views.append(key)
+    return [np.array(v, np.int32) for v in views]
+
+
+@pytest.mark.parametrize("fused", [True, False])
 @pytest.mark.parametrize("name", ["single", "anyres", "highres", "ragged", "single_mixed"])
-def test_workload_sampled_steps(davet, name):
-    """Full-size inputs in the benchmark's launch configuration: the gather is
-    compared bit for bit at one step per distinct level, attention on sampled
-    (row, head) outputs, and the first step's commits exactly."""
+def test_workload_sampled_steps(davet, name, fused):
+    """Full-size inputs in the benchmark's launch configuration (the fused
+    layout is the benchmark's default step): for every sampled view, the
+    step's cu_seqlens exactly, the packed rows bit for bit (unfused), and
+    sampled (row, head) attention outputs against the oracle's attention
+    over the oracle's gather of its own pyramid; the first view's commits
+    exactly (near-tie rule)."""
     w = workloads.make(name)
-    pl, feats, text = make_pipeline(davet, w)
+    pl, feats, text = make_pipeline(davet, w, fused)
     gpu_pyr = [pl.pyramid_cpu(b) for b in range(w.batch)]
     oracle_pyr, mrows = oracle_gather_inputs(w, oracle_pyramids(w, feats))
     # pyramid: one request, first tile, all levels against the oracle
@@ -116,34 +144,35 @@ def test_workload_sampled_steps(davet, name):
         mine = bf16_to_f64(gpu_pyr[0][off[lvl]: off[lvl] + g * g])
         assert np.abs(mine - ref[ref_off[lvl]:ref_off[lvl + 1]]).max() <= 2 ** -6
     rng = np.random.default_rng(1)
-    seen = set()
-    steps = []
-    for t in range(w.T):
-        key = tuple(w.schedule[t])
-        if key not in seen:
-            seen.add(key)
-            steps.append(t)
-    steps = steps[:4]
     masked = np.ones(w.total_resp, np.uint8)
     tokens = np.full(w.total_resp, -1, np.int32)
     argmax = np.full(w.total_resp, -1, np.int32)
     lg = workloads.logits(w, 0)
     lg_dev = lg.cuda()
-    for i, t in enumerate(steps):
-        pl.gather(t)
-        pl.attention()
+    for i, view in enumerate(sampled_views(w)):
+        # the step runs the view vector written into schedule slot 0
+        pl.schedule[0].copy_(torch.from_numpy(view))
+        if fused:
+            pl.view_attention(0)
+        else:
+            pl.gather(0)
+            pl.attention()
         if i == 0:
-            pl.unmask(t, lg_dev)
+            pl.unmask(0, lg_dev)
         torch.cuda.synchronize()
         assert davet.davet_device_status() == (0, 0)
         packed_ref, cu_ref = oracle.gather(oracle_pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp,
-                                           w.schedule[t], w.grid, w.n_levels, w.C, mixed_rows_per_tile=mrows)
+                                           view, w.grid, w.n_levels, w.C, mixed_rows_per_tile=mrows)
         N = int(cu_ref[-1])
-        assert list(pl.cu.cpu().numpy()) == list(cu_ref)
-        check_packed(pl.packed[:N], packed_ref)
+        assert list(pl.cu.cpu().numpy()) == list(cu_ref), (name, list(view))
+        if not fused:
+            check_packed(pl.packed[:N], packed_ref)
         rows, heads = [], []
         for b in range(w.batch):
-            rows += list(rng.integers(cu_ref[b], cu_ref[b + 1], size=16))
+            if cu_ref[b + 1] == cu_ref[b]:
+                continue
+            # random rows, plus the request's first and last row (tile edges)
+            rows += [cu_ref[b], cu_ref[b + 1] - 1] + list(rng.integers(cu_ref[b], cu_ref[b + 1], size=14))
             heads += list(rng.integers(0, w.H, size=16))
         rows = np.array(rows, np.int64)
         heads = np.array(heads, np.int32)
@@ -151,11 +180,11 @@ def test_workload_sampled_steps(davet, name):
         got = bf16_to_f64(pl.attn_out[torch.as_tensor(rows, device="cuda"),
                                       torch.as_tensor(heads, device="cuda").long()])
         max_abs, rel = attn_errors(got, att_ref)
-        assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (name, t, max_abs, rel)
+        assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (name, list(view), max_abs, rel)
         if i == 0:
             cu_resp = w.cu_resp()
             conf_ref, _, st_ref = oracle.unmask(lg, w.V, cu_resp, w.k, masked, tokens, argmax)
-            g_com = pl.committed[t].cpu().numpy()
+            g_com = pl.committed[0].cpu().numpy()
             for b in range(w.batch):
                 cref = {int(j - cu_resp[b]): conf_ref[j] for j in range(cu_resp[b], cu_resp[b + 1])}
                 check_topk([int(x) for x in g_com[b] if x >= 0], cref, w.k)

@@ -193,7 +193,7 @@ def test_fused_pipeline_tiny_against_oracle(davet):
             assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (name, t, max_abs, rel)
 
 
-@pytest.mark.parametrize("name", ["single", "ragged", "single_mixed"])
+@pytest.mark.parametrize("name", ["single", "anyres", "highres", "ragged", "single_mixed"])
 def test_fused_pipeline_full_size_matches_unfused(davet, name):
     """Full-size inputs in the benchmark's launch configuration: one step per
     distinct view schedule, fused and unfused pipelines bit-identical."""
