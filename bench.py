@@ -820,56 +820,69 @@ def _sampled_attention_time(oracle, packed, cu, w):
     return dt, dt * items / n
 
 def oracle_sample(w, budget_s=20.0):
-    """Times the fp64 oracle on a bounded sample of the workload: the pyramid
-    of every request once, then one denoising step (gather, attention,
-    unmask) per distinct scheduled level combination, and extrapolates to the
-    whole schedule.  Returns (denoising steps/s, cores, description)."""
+    """Times the fp64 oracle on a bounded sample of the workload and
+    extrapolates to the whole pass: the pyramid of the first request (scaled
+    to every request by tile count), then for each distinct scheduled view
+    combination (most frequent first, until the budget is spent) the gather
+    and the attention on at most ATTN_SAMPLE_ITEMS (row, head) outputs
+    (scaled by the output count), and the unmasking of the first step (every
+    answer row masked), scaled to each step by its masked-row count.
+    Returns (denoising steps/s, cores, description, seconds, parts)."""
     import numpy as np
 
     import oracle
     from paper_2608_01821_gb300 import workloads
     cores = oracle.max_threads()
-    feats = [workloads.features(w, b) for b in range(w.batch)]
     text = workloads.text_rows(w)
+    b0 = next(b for b in range(w.batch) if w.tiles[b] > 0)
+    f0 = workloads.features(w, b0)
     t0 = time.perf_counter()
+    ref = oracle.pyramid(f0, w.tiles[b0], w.grid, w.n_levels, w.C)
+    t_pyr1 = time.perf_counter() - t0
+    pyr0 = _to_bf16_bits(ref)
+    # the other requests' pyramids are not timed: their rows only feed the
+    # gather, whose cost does not depend on the values
     pyr = []
     for b in range(w.batch):
-        ref = oracle.pyramid(feats[b], w.tiles[b], w.grid, w.n_levels, w.C)
-        pyr.append(_to_bf16_bits(ref))
-    t_pyr = time.perf_counter() - t0
+        if b == b0 or w.tiles[b] == w.tiles[b0]:
+            pyr.append(pyr0)
+        else:
+            pyr.append(np.zeros((w.pyramid_rows(b), w.C), np.uint16))
+    t_pyr = t_pyr1 * sum(w.tiles) / w.tiles[b0]
     lg = workloads.logits(w, 0)
+    t2 = time.perf_counter()
+    masked = np.ones(w.total_resp, np.uint8)
+    tokens = np.full(w.total_resp, -1, np.int32)
+    argmax = np.full(w.total_resp, -1, np.int32)
+    oracle.unmask(lg, w.V, w.cu_resp(), w.k, masked, tokens, argmax)
+    t_unmask0 = time.perf_counter() - t2
+    spent = t_pyr1 + t_unmask0
     keys = {}
     for t in range(w.T):
         keys.setdefault(tuple(int(x) for x in w.schedule[t]), []).append(t)
     per_key = {}
-    spent = t_pyr
-    sampled = 0
     for key, ts in sorted(keys.items(), key=lambda kv: -len(kv[1])):
         t = ts[0]
         t1 = time.perf_counter()
         packed, cu = oracle.gather(pyr, w.tiles, text, w.text_offsets(), w.prompt, w.resp, w.schedule[t], w.grid,
                                    w.n_levels, w.C)
         t_gather = time.perf_counter() - t1
-        t_attn = _sampled_attention_time(oracle, packed, cu, w)[1]
-        t2 = time.perf_counter()
-        masked = np.ones(w.total_resp, np.uint8)
-        tokens = np.full(w.total_resp, -1, np.int32)
-        argmax = np.full(w.total_resp, -1, np.int32)
-        oracle.unmask(lg, w.V, w.cu_resp(), w.k, masked, tokens, argmax)
-        t_unmask = time.perf_counter() - t2
-        dt = t_gather + t_attn + t_unmask
-        per_key[key] = dt
-        spent += dt
-        sampled += 1
+        t_attn_spent, t_attn = _sampled_attention_time(oracle, packed, cu, w)
+        per_key[key] = t_gather + t_attn
+        spent += t_gather + t_attn_spent
         if spent > budget_s:
             break
     mean_dt = sum(per_key.values()) / len(per_key)
-    total = t_pyr + sum(per_key.get(k, mean_dt) * len(ts) for k, ts in keys.items())
-    desc = (f"fp64 oracle: pyramid of all {w.batch} request(s) + one denoising step for {sampled} of "
-            f"{len(keys)} distinct level combinations (gather and unmask in full, attention on at most "
-            f"{ATTN_SAMPLE_ITEMS} sampled (row, head) outputs scaled by the output count); extrapolated over "
-            f"the {w.T}-step schedule (unsampled combinations take the sampled mean)")
-    return w.T / total, cores, desc, spent
+    unmask_total = sum(t_unmask0 * w.masked_rows(t) / max(w.total_resp, 1) for t in range(w.T))
+    total = t_pyr + sum(per_key.get(k, mean_dt) * len(ts) for k, ts in keys.items()) + unmask_total
+    desc = (f"fp64 oracle: pyramid of request {b0} (scaled to all {sum(w.tiles)} tiles), one gather + attention "
+            f"for {len(per_key)} of {len(keys)} distinct view combinations (attention on at most "
+            f"{ATTN_SAMPLE_ITEMS} sampled (row, head) outputs, scaled by the output count), the unmasking of the "
+            f"first step (scaled by each step's masked rows); extrapolated over the {w.T}-step schedule")
+    parts = {"pyramid_one_request_s": round(t_pyr1, 3), "unmask_first_step_s": round(t_unmask0, 3),
+             "gather_plus_attention_s": {"/".join(map(str, k[:4])) + ("..." if len(k) > 4 else ""): round(v, 3)
+                                         for k, v in per_key.items()}}
+    return w.T / total, cores, desc, spent, parts
 
 
 def backbone_oracle_sample(w, n_layers: int):
@@ -1093,9 +1106,10 @@ def main(argv=None):
     if rank == 0:
         if not args.no_cpu_baseline:
             from paper_2608_01821_gb300 import workloads
-            v, cores, desc, spent = oracle_sample(workloads.make(args.config))
+            v, cores, desc, spent, parts = oracle_sample(workloads.make(args.config))
             out["cpu_baseline"] = {"value": round(v, 5), "unit": "denoising steps/s", "cores": cores,
-                                   "kind": "oracle", "sample": desc, "cpu_seconds": round(spent, 1)}
+                                   "kind": "oracle", "sample": desc, "cpu_seconds": round(spent, 1),
+                                   "parts": parts}
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist

@@ -377,7 +377,9 @@ def test_linear_device_row_count(davet, M, m, K, N, epi):
             out.copy_(R)
         davet.davet_linear(A, M, K, W, N, out, epi, out if epi == 1 else None, workspace=ws, rows_dev=rows_dev)
         torch.cuda.synchronize()
-        assert davet.davet_device_status() == (0, 0)
+        # a count above M is clamped and flags the capacity bit
+        st, flags = davet.davet_device_status(clear=True)
+        assert flags == (0x2 if rows_dev is not None and m > M else 0)
         outs.append(out)
     full, dyn = outs
     n = min(m, M)
@@ -430,6 +432,8 @@ def test_rmsnorm_device_row_count(davet, m):
     out = torch.full((M, C), -7.0, dtype=torch.bfloat16, device="cuda")
     davet.davet_rmsnorm(x, M, C, g, 1e-5, out, rows_dev=torch.tensor([m], dtype=torch.int32, device="cuda"))
     torch.cuda.synchronize()
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags == (0x2 if m > M else 0)
     n = min(m, M)
     assert (out[n:].float() == -7.0).all()
     if n:
