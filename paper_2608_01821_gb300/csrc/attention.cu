@@ -334,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // rows of the item's request: packed input (cu) or its view block
     if (lane == 0) {
       ATTN_TRACE_DECL;
-      uint32_t it = 0, wi = 0;
+      uint32_t it = 0, wi = 0, nq = 0, nk = 0, nv = 0;  // loads issued (query tiles, K, V)
       bool ok = true;
       for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x, ++wi) {
         const Item w = decode(s, item, H, qtiles);
@@ -345,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < w.ntile; ++t)
           for (int c = 0; c < KC; ++c)
             tma_load_3d(s.q[t][c], &tmap, &s.q_full, 64 * c, h_coord(0, w.h, H), src0 + w.q0 + t * BM);
+        ++nq;
         for (int j = 0; j < w.nkv; ++j, ++it) {
           const int st = it % NS;
           const int row = static_cast<int>(src0 + w.key_tile(j) * BN);
@@ -354,20 +355,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           ATTN_TRACE(0, 2, it);
           mbar_arrive_expect_tx(&s.k_full[st], KC * kChunkBytes);
           for (int c = 0; c < KC; ++c) tma_load_3d(s.k[st][c], &tmap, &s.k_full[st], 64 * c, h_coord(1, w.h, H), row);
+          ++nk;
           // V of stage st is free once the PV MMAs of that tile completed
           if (it >= NS) ok = mbar_wait(&s.v_empty[st], ((it / NS) - 1) & 1, prm.err, abort_flag);
           if (!ok) break;
           mbar_arrive_expect_tx(&s.v_full[st], KC * kChunkBytes);
           for (int c = 0; c < KC; ++c) tma_load_3d(s.v[st][c], &tmap, &s.v_full[st], 64 * c, h_coord(2, w.h, H), row);
+          ++nv;
           ATTN_TRACE(0, 1, it);
         }
       }
       if (!ok) {
-        // let copies already in flight land before the CTA exits
-        for (uint32_t i = (it > NS ? it - NS : 0); i < it; ++i) {
-          mbar_wait(&s.k_full[i % NS], (i / NS) & 1, nullptr, nullptr);
-          mbar_wait(&s.v_full[i % NS], (i / NS) & 1, nullptr, nullptr);
-        }
+        // let copies already in flight land before the CTA exits: the last
+        // query tiles (the MMA warp may not have waited for them) and the
+        // last NS key and NS value tiles issued
+        if (nq > 0) mbar_wait(&s.q_full, (nq - 1) & 1, nullptr, nullptr);
+        for (uint32_t i = (nk > NS ? nk - NS : 0); i < nk; ++i) mbar_wait(&s.k_full[i % NS], (i / NS) & 1, nullptr, nullptr);
+        for (uint32_t i = (nv > NS ? nv - NS : 0); i < nv; ++i) mbar_wait(&s.v_full[i % NS], (i / NS) & 1, nullptr, nullptr);
       }
     }
   } else if (warp == kWarpMma) {
