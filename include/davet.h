@@ -486,14 +486,17 @@ davet_status davet_stage_masked_rows(const void* src, int V, const uint8_t* mask
  *     (max, sum, first index) record per vocabulary chunk, then a 4-byte
  *     confidence and a 4-byte index; each of these three arrays starts on a
  *     256-byte boundary.  When the chunk count that davet_unmask_topk uses
- *     (8 KB of logits per chunk, at most 64 chunks) does not fit, this call
- *     cuts each row into fewer, longer chunks until it fits.  The argmax,
- *     the tokens and the committed rows are the same as davet_unmask_topk's;
- *     the confidences and statistics agree to fp32 rounding (the chunk sums
- *     are added in a different grouping).  At V = 126464 the standard 31
- *     chunks fit up to 2,080 answer rows.  Only a size that does not fit
- *     even with one chunk per row (24 bytes per row: above 43,680 rows) is
- *     rejected, with DAVET_ERR_UNSUPPORTED, before anything is enqueued.
+ *     (16 KB of logits per chunk when the call has at least 8,192 (row,
+ *     16 KB chunk) units, else 8 KB; at most 64 chunks) does not fit, this
+ *     call cuts each row into fewer, longer chunks until it fits.  The
+ *     argmax, the tokens and the committed rows are the same as
+ *     davet_unmask_topk's; the confidences and statistics agree to fp32
+ *     rounding (the chunk sums are added in a different grouping).  At
+ *     V = 126464 the standard layout (31 chunks per row below 512 answer
+ *     rows, 16 from 512 on) fits up to 3,970 answer rows.  Only a size that
+ *     does not fit even with one chunk per row (24 bytes per row: above
+ *     43,680 rows) is rejected, with DAVET_ERR_UNSUPPORTED, before anything
+ *     is enqueued.
  *   - Set-up: the array's device address is looked up with
  *     cudaGetSymbolAddress, with the device current, at the first call in
  *     each CUDA context (a device's primary context, or another context the

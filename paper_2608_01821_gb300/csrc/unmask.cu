@@ -2,7 +2,8 @@
 // Eq. 1-2) and the step statistics that feed the trajectory risk (Eq. 7).
 //
 // Two kernels:
-//  1. row kernel: every (answer row, 8 KB vocabulary chunk) is one warp.
+//  1. row kernel: every (answer row, vocabulary chunk of 8 or 16 KB) is one
+//     warp.
 //     A warp of a masked row streams its chunk of bf16 logits once with 128-bit
 //     loads (eight in flight per lane) and keeps, per lane, an online
 //     (max, sum of 2^(x*log2e - max*log2e), first argmax) triple, merged by
@@ -48,16 +49,23 @@ struct Layout {
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Chunks of 512 slices (8 KB: two rounds of loads per lane), at most
-// kMaxChunks per row; when `max_bytes` is given (the allocation-free path),
-// fewer and longer chunks so that the layout fits.  The conf / argmax
-// arrays serve requests longer than kSelSmemRows rows.
+// Chunks of 1024 slices (16 KB: four rounds of loads per lane) when the
+// call has at least kWideUnits such (row, chunk) units, which is enough to
+// keep every SM streaming, else of 512 slices (8 KB), so that few answer rows
+// still spread over many warps; at most kMaxChunks per row.  Longer chunks
+// mean fewer blocks per call (a late step, with few rows still masked, pays
+// for launching the blocks of every row) and fewer records for the select to
+// combine.  When `max_bytes` is given (the allocation-free path), fewer and
+// longer chunks so that the layout fits.  The conf / argmax arrays serve
+// requests longer than kSelSmemRows rows.
+constexpr int64_t kWideUnits = 8192;
 inline Layout layout_for(int64_t total_rows, int V, size_t max_bytes = ~size_t(0)) {
   Layout L;
   const int64_t v8 = V / 8;
   const size_t rows = static_cast<size_t>(total_rows);
   const size_t fixed = align256(rows * sizeof(float)) + align256(rows * sizeof(int32_t));
-  int64_t nchunk = std::max<int64_t>(1, std::min<int64_t>(kMaxChunks, (v8 + 511) / 512));
+  const int64_t slices = total_rows * ((v8 + 1023) / 1024) >= kWideUnits ? 1024 : 512;
+  int64_t nchunk = std::max<int64_t>(1, std::min<int64_t>(kMaxChunks, (v8 + slices - 1) / slices));
   while (nchunk > 1 && align256(rows * nchunk * sizeof(Partial)) + fixed > max_bytes) --nchunk;
   L.nchunk = static_cast<int>(nchunk);
   L.off_partial = 0;
@@ -526,7 +534,7 @@ extern "C" davet_status davet_stage_masked_rows(const void* src, int V, const ui
   if (total_rows > (int64_t(1) << 31) / 64) return DAVET_ERR_UNSUPPORTED;
   const int V8 = V / 8;
   // 16 KB per warp: over the host link fewer, longer streams do better
-  // than the unmasking's 8 KB chunks (4, 8, 16, 32, 64 KB and whole rows measured)
+  // than 8 KB chunks (4, 8, 16, 32, 64 KB and whole rows measured)
   const int nchunk = std::max(1, std::min(kMaxChunks, (V8 + 1023) / 1024));
   const int chunk = (V8 + nchunk - 1) / nchunk;
   const long long warps = total_rows * nchunk;

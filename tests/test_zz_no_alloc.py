@@ -82,8 +82,9 @@ def _logits(R, V, seed, dev):
     ([128], workloads.VOCAB_8B, 2),          # one 8B-class request (vocabulary split path)
     ([300, 0, 57, 512, 9], 4096, 3),         # ragged batch with an empty request
     ([32], 1024, 4),                         # tiny workload shape
-    # the standard 31 chunks per row do not fit: fewer, longer chunks
-    ([3000], workloads.VOCAB_8B, 2),         # 21 chunks per row
+    # the standard layout (16 chunks of 16 KB per row from 512 rows on) does
+    # not fit: fewer, longer chunks
+    ([5000], workloads.VOCAB_8B, 2),         # 12 chunks per row
     ([20000, 9000], workloads.VOCAB_8B, 2),  # one chunk per row; requests above the select's shared-memory rows
     ([_noalloc_max_rows()], 1024, 2),        # exactly the largest size the array holds
 ])
@@ -94,7 +95,7 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls(davet, resp, V, k):
     ref = _state(resp, k)
     new = _state(resp, k)
     ws_bytes = davet.davet_unmask_topk_workspace(R, V, B)
-    if V == workloads.VOCAB_8B and R > 2080:
+    if V == workloads.VOCAB_8B and R > 3970:
         # the workspace entry point's layout does not fit in the array, so the
         # allocation-free call runs on fewer vocabulary chunks per row
         assert ws_bytes > SCRATCH_BYTES
