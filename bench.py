@@ -794,7 +794,7 @@ def run_e2e(args, pl, w, dev, stream, world, policy_pass=None, policy_step=None)
 
 
 # ----------------------------------------------------------- CPU oracle
-ATTN_SAMPLE_ITEMS = 4096
+ATTN_SAMPLE_ITEMS = 32768
 
 
 def _to_bf16_bits(x):

@@ -21,8 +21,9 @@
 // head-major, so CTAs running together share a head's K/V in L2.  Keys past
 // the end of a request are masked to -inf and their V rows zeroed in shared
 // memory, so key tiles may straddle request boundaries and the buffer end.
-// With few items (short sequences) the host selects one query tile per item
-// so that more SMs get work.
+// With few items (short sequences) one query tile per item is chosen so that
+// more SMs get work; when the last of several rounds of two-tile items fills
+// at most half of the grid, those items are split into their two tiles.
 //
 // Fused variant (davet_view_attention, FUSED = true): the step input is never
 // packed.  Each request keeps every evidence view as a contiguous block
@@ -71,6 +72,7 @@ struct Smem {
   int abort;
   int n_req;   // requests with at least one row
   int n_items;
+  int n_whole;  // items run with all their query tiles; later ones are halves of two-tile items
   int qtiles;
   int32_t req_start[kMaxBatch];
   int32_t req_len[kMaxBatch];
@@ -151,6 +153,14 @@ __device__ __forceinline__ int h_coord(int slot, int h, int H) { return slot * H
 
 template <typename S>
 __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) {
+  // items from n_whole on are the two halves (one query tile each) of the
+  // last round's two-tile items
+  int half = -1;
+  if (item >= s.n_whole) {
+    const int k = item - s.n_whole;
+    item = s.n_whole + (k >> 1);
+    half = k & 1;
+  }
   // largest i with cum[i] <= item
   int lo = 0, hi = s.n_req - 1;
   while (lo < hi) {
@@ -174,6 +184,11 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
   const int qb = local - it.h * nq;
   it.kv0 = static_cast<int>((static_cast<long long>(qb) * it.nkv) / nq);
   it.ntile = (qtiles == 2 && it.q0 + BM < len) ? 2 : 1;
+  if (half >= 0) {
+    // a half whose tile lies past the request end computes rows it never stores
+    it.q0 += half * BM;
+    it.ntile = 1;
+  }
   return it;
 }
 
@@ -320,7 +335,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       acc += ((s.req_len[s.order[i]] + rows_per_item - 1) / rows_per_item) * H;
     }
     s.cum[s.n_req] = acc;
-    s.n_items = acc;
+    // when the last of several rounds of two-tile items fills at most half of
+    // the grid, its items run as two one-tile items each (on twice as many
+    // CTAs), so the launch ends after a one-tile item rather than a two-tile one
+    int split = 0;
+    const int g = static_cast<int>(gridDim.x);
+    if (qt == 2 && acc > g) {
+      const int r = acc % g;
+      if (r > 0 && 2 * r <= g) split = r;
+    }
+    s.n_whole = acc - split;
+    s.n_items = acc + split;
   }
   tc_fence_before();
   __syncthreads();
