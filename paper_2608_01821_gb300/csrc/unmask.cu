@@ -31,7 +31,12 @@ namespace unm {
 constexpr int kRowThreads = 256;  // 8 warps, one (row, chunk) unit each
 constexpr int kMaxChunks = 64;
 constexpr int kLoads = 8;         // 16-byte loads in flight per lane
-constexpr int kSelThreads = 256;  // one answer row per thread and pass
+// The select runs 512 threads combining records in rounds of 16 when a row
+// has at most 16 chunks (one round of loads each; a 512-row request in one
+// pass), else 256 threads with rounds of 32 (the register budget of a
+// 32-record round allows 256 threads).
+constexpr int kSelThreadsNarrow = 512, kSelGroupNarrow = 16;
+constexpr int kSelThreadsWide = 256, kSelGroupWide = 32;
 constexpr int kSelSmemRows = 4096;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -262,15 +267,16 @@ __device__ __forceinline__ void warp_best(float& c, long long& pos) {
   }
 }
 
-// Combination of chunks [c0, min(c0 + 32, nc)) of one row's triples in two
+// Combination of chunks [c0, min(c0 + G, nc)) of one row's triples in two
 // passes: the max M, then the sum of s * 2^((m - M)log2e) and the smallest
 // index among chunks at M.
+template <int G>
 __device__ __forceinline__ Partial combine_group(const Partial* __restrict__ part, long long rows, long long i, int c0,
                                                  int nc) {
-  float m[32], sv[32];
-  int ix[32];
+  float m[G], sv[G];
+  int ix[G];
 #pragma unroll
-  for (int c = 0; c < 32; ++c) {
+  for (int c = 0; c < G; ++c) {
     const bool ok = c0 + c < nc;
     const Partial v = part[static_cast<long long>(ok ? c0 + c : 0) * rows + i];
     m[c] = ok ? v.m : -INFINITY;
@@ -279,14 +285,14 @@ __device__ __forceinline__ Partial combine_group(const Partial* __restrict__ par
   }
   float mx = m[0];
 #pragma unroll
-  for (int c = 1; c < 32; ++c) mx = fmaxf(mx, m[c]);
+  for (int c = 1; c < G; ++c) mx = fmaxf(mx, m[c]);
   Partial r;
   r.m = mx;
   r.s = 0.f;
   r.idx = INT_MAX;
   r.pad = 0;
 #pragma unroll
-  for (int c = 0; c < 32; ++c) {
+  for (int c = 0; c < G; ++c) {
     if (sv[c] > 0.f) r.s += sv[c] * sfu_ex2((m[c] - mx) * kLog2e);
     if (m[c] == mx) r.idx = min(r.idx, ix[c]);
   }
@@ -294,11 +300,12 @@ __device__ __forceinline__ Partial combine_group(const Partial* __restrict__ par
 }
 
 // (argmax, conf) of one row from all its chunk triples.
+template <int G>
 __device__ __forceinline__ void combine_row(const Partial* __restrict__ part, long long rows, long long i, int nc,
                                             float& conf, int& idx) {
-  Partial p = combine_group(part, rows, i, 0, nc);
-  for (int c0 = 32; c0 < nc; c0 += 32) {
-    const Partial q = combine_group(part, rows, i, c0, nc);
+  Partial p = combine_group<G>(part, rows, i, 0, nc);
+  for (int c0 = G; c0 < nc; c0 += G) {
+    const Partial q = combine_group<G>(part, rows, i, c0, nc);
     const float mx = fmaxf(p.m, q.m);
     const float sp = p.s > 0.f ? p.s * sfu_ex2((p.m - mx) * kLog2e) : 0.f;
     const float sq = q.s > 0.f ? q.s * sfu_ex2((q.m - mx) * kLog2e) : 0.f;
@@ -314,6 +321,7 @@ __device__ __forceinline__ void combine_row(const Partial* __restrict__ part, lo
 // pass (one round of coalesced loads); after one barrier, warp 0 forms the
 // statistics and takes the top-k with k rounds of a warp arg-max over the
 // rows' confidences in shared memory.
+template <int kSelThreads, int kGroup>
 __global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
   __shared__ float s_conf_buf[kSelSmemRows];
   __shared__ int32_t s_idx_buf[kSelSmemRows];
@@ -344,7 +352,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
     const int prev = a.argmax ? a.argmax[i] : -1;
     float conf;
     int idx;
-    combine_row(a.partial, a.total_rows, i, a.nchunk, conf, idx);
+    combine_row<kGroup>(a.partial, a.total_rows, i, a.nchunk, conf, idx);
     if (!m8) {
       cbuf[r] = -3.f;
       continue;
@@ -455,7 +463,10 @@ inline davet_status enqueue(const void* logits, int V, const int32_t* cu, int ba
   a.row_conf = reinterpret_cast<float*>(ws + L.off_conf);
   a.row_idx = reinterpret_cast<int32_t*>(ws + L.off_idx);
   a.err = err;
-  const cudaError_t e = launch(select_kernel, dim3(batch), dim3(kSelThreads), 0, stream, a);
+  const cudaError_t e =
+      L.nchunk <= kSelGroupNarrow
+          ? launch(select_kernel<kSelThreadsNarrow, kSelGroupNarrow>, dim3(batch), dim3(kSelThreadsNarrow), 0, stream, a)
+          : launch(select_kernel<kSelThreadsWide, kSelGroupWide>, dim3(batch), dim3(kSelThreadsWide), 0, stream, a);
   return e == cudaSuccess ? DAVET_OK : cuda_fail(e);
 }
 
