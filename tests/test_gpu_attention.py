@@ -124,3 +124,28 @@ def test_full_size_sampled(davet, name):
         got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
         max_abs, rel = attn_errors(got, ref)
         assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (name, level, max_abs, rel)
+
+
+@pytest.mark.parametrize("L,H,nreq", [(5120, 16, 1), (2600, 16, 2)])
+def test_last_round_split_into_one_tile_items(davet, L, H, nreq):
+    """Work items of two 128-row query tiles run in rounds of one item per
+    SM; when the last of several rounds fills at most half of the grid its
+    items run as two one-tile items (on a 152-SM GPU: 5,120 rows x 16 heads
+    = 320 items, the last 16 split; 2 x 2,600 rows x 16 heads = 352 items,
+    the last 48 split).  Those items are the last heads' last query blocks in the
+    schedule (longest request first, head-major), so every row of the last
+    head is compared with the oracle, plus sampled rows of the others."""
+    lens = [L] * nreq
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    D = 128
+    qkv = workloads.qkv_rows(N, H, D, seed=L + H + nreq)
+    out = run(davet, qkv, cu, H, D)
+    rng = np.random.default_rng(L)
+    last = cu[-2]  # the last request in the schedule (equal lengths: the highest index)
+    rows = np.concatenate([np.arange(last, N), rng.integers(0, N, size=256)]).astype(np.int64)
+    heads = np.concatenate([np.full(N - last, H - 1), rng.integers(0, H, size=256)]).astype(np.int32)
+    ref = oracle.attention_rows(qkv, cu, H, D, 1.0 / math.sqrt(D), rows, heads)
+    got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
+    max_abs, rel = attn_errors(got, ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
