@@ -278,16 +278,7 @@ def run_ours(args, rank, world, local_rank):
             "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) features/text, N(0,2) logits; no weights)",
             "config": {
-                "workload": w.name,
-                "batch": w.batch,
-                "heads": w.H,
-                "head_dim": w.D,
-                "grid": w.grid,
-                "levels": w.n_levels,
-                "tiles": w.tiles if w.batch <= 16 else sum(w.tiles),
-                "denoising_steps_per_pass": w.T,
-                "vocab": w.V,
-                "k": w.k,
+                **workload_config(w),
                 "parallelism": f"replicas x{world} (independent requests)",
                 "timing": "CUDA events per pass on the launching stream; one CUDA graph per pass",
                 "l2": f"{L2_FLUSH_BYTES >> 20} MiB write between timed passes (not timed)",
@@ -524,6 +515,13 @@ def merge_round_count(grid: int, n_levels: int) -> int:
             n -= min(n - g * g, (n + 1) // 2)
             rounds += 1
     return rounds
+
+
+def workload_config(w) -> dict:
+    """The workload's defining sizes, reported by both arms."""
+    return {"workload": w.name, "batch": w.batch, "heads": w.H, "head_dim": w.D, "grid": w.grid,
+            "levels": w.n_levels, "tiles": w.tiles if w.batch <= 16 else sum(w.tiles),
+            "denoising_steps_per_pass": w.T, "vocab": w.V, "k": w.k}
 
 
 def build_launches(w, realizer: str, fused: bool) -> int:
@@ -969,7 +967,8 @@ def run_reference(args, rank, world):
     return {"metric": METRIC, "value": round(value, 5), "unit": "denoising steps/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": w.name}, "impl": "reference",
+            "data": "synthetic (seeded N(0,1) features/text, N(0,2) logits; no weights)",
+            "config": workload_config(w), "impl": "reference",
             "cpu_baseline": {"value": round(value, 5), "unit": "denoising steps/s", "cores": cores,
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 5), "unit": "denoising steps/s", "h2d_bytes_per_step": 0,
