@@ -17,6 +17,12 @@
 //                keep the same stale max, so the result is unchanged) and,
 //                after the last key tile, normalizes O and stores it as bf16.
 // TMEM: S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
+// The one-tile items of a launch with one tile per item, and the split
+// halves, use both score regions in turn: the MMA warp issues S(0), S(1),
+// then per key tile j PV(j), S(j+2), so the QK^T of the next key tile is done
+// before the softmax of the current one ends; warpgroup A alone runs the
+// softmax (warpgroup B idles in that item).  The odd last tile of a request
+// in a two-tile launch keeps one score region (S after the previous PV).
 // Items are ordered longest request first and, within a request,
 // head-major, so CTAs running together share a head's K/V in L2.  Keys past
 // the end of a request are masked to -inf and their V rows zeroed in shared
@@ -36,6 +42,7 @@
 #include <cstdio>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -139,6 +146,7 @@ struct Item {
   int b;                              // request
   int start, len, q0, h, nkv, ntile;  // q0: first query row of the item within the request
   int kv0;  // key tile the item starts from (key tiles are visited cyclically)
+  bool alt;  // one query tile whose scores alternate between both score regions
 
   // key tile visited at loop step j
   __device__ __forceinline__ int key_tile(int j) const {
@@ -189,6 +197,11 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
     it.q0 += half * BM;
     it.ntile = 1;
   }
+  // one-tile items of a one-tile launch and the split halves of the last
+  // round alternate their score regions; the odd last tile of a request in a
+  // two-tile launch runs one region in series (running it ahead among
+  // two-tile items costs those items more than it saves)
+  it.alt = it.ntile == 1 && (qtiles == 1 || half >= 0);
   return it;
 }
 
@@ -415,27 +428,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t v_desc0 = sw128_desc(smem_u32(s.v[0][0]), kChunkBytes, 1024);
       constexpr uint32_t kTile16 = (KC * kChunkBytes) >> 4;  // one Q tile / K or V stage
       uint32_t it = 0, wi = 0;
-      uint32_t np[2] = {0, 0};  // P tiles consumed per query tile
+      uint32_t np0 = 0, np1 = 0;  // phases of p_full[0], p_full[1] consumed
       bool ok = true;
 
-      // S_t = Q_t K^T for the K tile in stage st
-      auto issue_s = [&](int t, int st) {
+      // S = Q_t K^T into score region r for the K tile in stage st
+      auto issue_s = [&](int t, int r, int st) {
         const uint64_t a0 = q_desc0 + t * kTile16;
         const uint64_t b0 = k_desc0 + st * kTile16;
-        const uint32_t d = tmem + col_s(t);
+        const uint32_t d = tmem + col_s(r);
         umma_ss_imm<false>(d, a0, b0, kIdescQK);
 #pragma unroll
         for (int kk = 1; kk < D / 16; ++kk) {
           const uint32_t off = ((kk >> 2) * kChunkBytes + (kk & 3) * 32) >> 4;
           umma_ss_imm<true>(d, a0 + off, b0 + off, kIdescQK);
         }
-        umma_commit(&s.s_full[t]);
+        umma_commit(&s.s_full[r]);
       };
-      // O_t (+)= P_t V for the V tile in stage st, P read from TMEM
-      auto issue_pv = [&](int t, int st, bool first) {
+      // O_t (+)= P V for the V tile in stage st, P read from score region r
+      auto issue_pv = [&](int t, int r, int st, bool first) {
         const uint64_t b0 = v_desc0 + st * kTile16;
         const uint32_t d = tmem + col_o(t);
-        const uint32_t a = tmem + col_s(t);
+        const uint32_t a = tmem + col_s(r);
         if (first)
           umma_ts_imm<false>(d, a, b0, kIdescPV);
         else
@@ -448,12 +461,57 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Item w = decode(s, item, H, qtiles);
         ok = mbar_wait(&s.q_full, wi & 1, prm.err, abort_flag);
         if (!ok) break;
-        // prologue: S for key tile 0
+        if (w.alt) {
+          // One query tile: its scores alternate between the two score
+          // regions, so the QK^T of key tile j+1 runs during the softmax of
+          // key tile j.  Order: S(0), S(1), then per j: PV(j), S(j+2).
+          ok = mbar_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          tc_fence_after();
+          issue_s(0, 0, it % NS);
+          umma_commit(&s.k_empty[it % NS]);
+          if (w.nkv > 1) {
+            ok = mbar_wait(&s.k_full[(it + 1) % NS], ((it + 1) / NS) & 1, prm.err, abort_flag);
+            if (!ok) break;
+            tc_fence_after();
+            issue_s(0, 1, (it + 1) % NS);
+            umma_commit(&s.k_empty[(it + 1) % NS]);
+          }
+          if (w.nkv <= 2) umma_commit(&s.q_empty);
+          for (int j = 0; j < w.nkv; ++j, ++it) {
+            const int st = it % NS;
+            const int r = j & 1;
+            ok = mbar_wait(&s.v_full[st], (it / NS) & 1, prm.err, abort_flag);
+            if (!ok) break;
+            const uint32_t npr = r ? np1++ : np0++;
+            ok = mbar_wait(&s.p_full[r], npr & 1, prm.err, abort_flag);
+            if (!ok) break;
+            tc_fence_after();
+            issue_pv(0, r, st, j == 0);
+            umma_commit(&s.v_empty[st]);
+            if (j + 2 < w.nkv) {
+              // S(j+2) overwrites the P that PV(j) reads: the tensor pipe
+              // runs the two in issue order
+              const int st2 = (it + 2) % NS;
+              ok = mbar_wait(&s.k_full[st2], ((it + 2) / NS) & 1, prm.err, abort_flag);
+              if (!ok) break;
+              tc_fence_after();
+              issue_s(0, r, st2);
+              umma_commit(&s.k_empty[st2]);
+              if (j + 2 == w.nkv - 1) umma_commit(&s.q_empty);
+            } else if (j == w.nkv - 1) {
+              umma_commit(&s.o_full[0]);
+            }
+          }
+          continue;
+        }
+        // one or two query tiles, one score region each: prologue, S of key
+        // tile 0
         ok = mbar_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        issue_s(0, it % NS);
-        if (w.ntile == 2) issue_s(1, it % NS);
+        issue_s(0, 0, it % NS);
+        if (w.ntile == 2) issue_s(1, 1, it % NS);
         umma_commit(&s.k_empty[it % NS]);
         if (w.nkv == 1) umma_commit(&s.q_empty);
         for (int j = 0; j < w.nkv; ++j, ++it) {
@@ -464,19 +522,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           ATTN_TRACE(1, 10, it);
           // tile A: PV, then S of the next key tile
-          ok = mbar_wait(&s.p_full[0], np[0] & 1, prm.err, abort_flag);
+          ok = mbar_wait(&s.p_full[0], np0 & 1, prm.err, abort_flag);
           if (!ok) break;
           ATTN_TRACE(1, 12, it);
-          ++np[0];
+          ++np0;
           tc_fence_after();
-          issue_pv(0, st, j == 0);
+          issue_pv(0, 0, st, j == 0);
           if (w.ntile == 1) umma_commit(&s.v_empty[st]);
           if (more) {
             ok = mbar_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
             if (!ok) break;
-              ATTN_TRACE(1, 11, it);
+            ATTN_TRACE(1, 11, it);
             tc_fence_after();
-            issue_s(0, st1);
+            issue_s(0, 0, st1);
             if (w.ntile == 1) {
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
@@ -486,15 +544,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (w.ntile == 2) {
             // tile B: PV, then S of the next key tile
-            ok = mbar_wait(&s.p_full[1], np[1] & 1, prm.err, abort_flag);
+            ok = mbar_wait(&s.p_full[1], np1 & 1, prm.err, abort_flag);
             if (!ok) break;
             ATTN_TRACE(1, 13, it);
-            ++np[1];
+            ++np1;
             tc_fence_after();
-            issue_pv(1, st, j == 0);
+            issue_pv(1, 1, st, j == 0);
             umma_commit(&s.v_empty[st]);
             if (more) {
-              issue_s(1, st1);
+              issue_s(1, 1, st1);
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
             } else {
@@ -512,123 +570,152 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t = warp >> 2;             // query tile of this warpgroup
     const int r = tid & 127;             // query row within the tile == TMEM lane
     const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    const uint32_t s_addr = tmem + lane_base + col_s(t);
     const uint32_t o_addr = tmem + lane_base + col_o(t);
     ATTN_TRACE_DECL;
     const float c = prm.scale_log2;
-    uint32_t ns = 0, no = 0;
+    // ns_t: completions of s_full[t] so far; warpgroup A also counts those
+    // of s_full[1] (ns_b: its alternating items wait for them) and the key
+    // tiles of the CTA (kt: they name the K/V stage and its phase); no:
+    // epilogues of this warpgroup.  A warpgroup counts every completion of
+    // the barriers it waits for, also in items where it does not wait.
+    uint32_t ns_t = 0, ns_b = 0, kt = 0, no = 0;
     bool ok = true;
+    float m = -INFINITY;  // running max of c * score (log2 domain)
+    float l = 0.f;        // running sum of the bf16-rounded 2^(c*score - m)
+    // Softmax of key tile j of item w, its scores in region sr (the ns-th
+    // completion of s_full[sr]); alt: the item alternates its score regions.
+    auto key_tile = [&](auto alt, const Item& w, int j, int sr, uint32_t ns) __attribute__((always_inline)) -> bool {
+      if (!warp_wait(&s.s_full[sr], ns & 1, prm.err, abort_flag)) return false;
+      const uint32_t s_addr = tmem + lane_base + col_s(sr);
+      if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
+      tc_fence_after();
+      // all four TMEM loads in flight before one wait
+      // the row in two halves: the second half's TMEM load is in flight
+      // while the first half's max is taken
+      uint32_t raw[BN];
+      tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&raw[0]));
+      tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&raw[32]));
+      tmem_wait_ld_regs(&raw[0]);
+      tmem_ld32(s_addr + 64, *reinterpret_cast<uint32_t(*)[32]>(&raw[64]));
+      tmem_ld32(s_addr + 96, *reinterpret_cast<uint32_t(*)[32]>(&raw[96]));
+      if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
+      float* x = reinterpret_cast<float*>(raw);
+      const int valid = min(BN, w.len - w.key_tile(j) * BN);
+      if (t == 0 && valid < BN) {
+        // keys past the request end: zero their V rows before PV reads them
+        // (P is 0 there, but the rows may hold anything, including
+        // non-finite values).  Warpgroup A sees every key tile of the CTA,
+        // so kt names the V stage and phase.
+        if (!warp_wait(&s.v_full[kt % NS], (kt / NS) & 1, prm.err, abort_flag)) return false;
+        if (r >= valid) {
+#pragma unroll
+          for (int cc = 0; cc < KC; ++cc) {
+            uint4* row = reinterpret_cast<uint4*>(s.v[kt % NS][cc] + r * 128);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) row[u] = make_uint4(0, 0, 0, 0);
+          }
+        }
+        fence_proxy_async_smem();
+      }
+      if (valid < BN / 2) {
+#pragma unroll
+        for (int i = 0; i < BN / 2; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+      }
+      // row max: eight independent chains of three-input max, then a tree
+      float mp[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
+#pragma unroll
+      for (int i = 16; i < BN / 2; i += 16)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+      tmem_wait_ld_regs(&raw[64]);
+      if (valid < BN) {
+#pragma unroll
+        for (int i = BN / 2; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+      }
+#pragma unroll
+      for (int i = BN / 2; i < BN; i += 16)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+      const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
+      if (r == 0) ATTN_TRACE(2 + t, 26 + t, ns);
+      const float mt = mx * c;
+      float factor = 1.f;
+      bool need = false;
+      if (j == 0) {
+        m = mt;
+      } else if (mt > m + kRescaleThreshold) {
+        factor = ex2(m - mt);
+        m = mt;
+        need = true;
+      }
+      const float neg_m = -m;
+      // p = 2^(c*s - m): packed FMA for two scores, two SFU exponentials,
+      // rounded to bf16.  The row sum adds the rounded weights, the values
+      // the PV MMA multiplies V by, so the weights applied to V sum to one
+      // after the final division (four accumulators).
+      float rsum[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int q = 0; q < BN / 32; ++q) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float a0, a1;
+          ffma2(a0, a1, x[32 * q + 2 * i], x[32 * q + 2 * i + 1], c, c, neg_m, neg_m);
+          pk[i] = pack_bf16x2(ex2(a0), ex2(a1));
+          const int h = (i & 1) * 2;
+          add_bf16x2_f32(rsum[h], rsum[h + 1], pk[i]);
+        }
+        tmem_st16(s_addr + 16 * q, pk);
+      }
+      const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
+      if (r == 0) ATTN_TRACE(2 + t, 28 + t, ns);
+      // no MMA touches O before P is published; with two query tiles O is
+      // settled here (S of this tile was issued after the previous PV of
+      // this tile), with one the previous PV may still run: wait for it
+      if (j > 0 && __any_sync(0xffffffffu, need)) {
+        if constexpr (decltype(alt)::value) {
+          if (!warp_wait(&s.v_empty[(kt - 1) % NS], ((kt - 1) / NS) & 1, prm.err, abort_flag)) return false;
+          tc_fence_after();
+        }
+        uint32_t o[32];
+#pragma unroll 1
+        for (int q = 0; q < D / 32; ++q) {
+          tmem_ld32(o_addr + 32 * q, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+          tmem_st32(o_addr + 32 * q, o);
+        }
+      }
+      l = (j == 0) ? rs : l * factor + rs;
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&s.p_full[sr]);
+      if (r == 0) ATTN_TRACE(2 + t, 24 + t, ns);
+      return true;
+    };
     for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x) {
       const Item w = decode(s, item, H, qtiles);
-      if (t >= w.ntile) continue;
-      float m = -INFINITY;  // running max of c * score (log2 domain)
-      float l = 0.f;        // running sum of 2^(c*score - m)
-      for (int j = 0; j < w.nkv; ++j, ++ns) {
-        ok = warp_wait(&s.s_full[t], ns & 1, prm.err, abort_flag);
-        if (!ok) break;
-        if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
-        tc_fence_after();
-        // all four TMEM loads in flight before one wait
-        // the row in two halves: the second half's TMEM load is in flight
-        // while the first half's max is taken
-        uint32_t raw[BN];
-        tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&raw[0]));
-        tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&raw[32]));
-        tmem_wait_ld_regs(&raw[0]);
-        tmem_ld32(s_addr + 64, *reinterpret_cast<uint32_t(*)[32]>(&raw[64]));
-        tmem_ld32(s_addr + 96, *reinterpret_cast<uint32_t(*)[32]>(&raw[96]));
-        if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
-        float* x = reinterpret_cast<float*>(raw);
-        const int valid = min(BN, w.len - w.key_tile(j) * BN);
-        if (t == 0 && valid < BN) {
-          // keys past the request end: zero their V rows before PV reads them
-          // (P is 0 there, but the rows may hold anything, including
-          // non-finite values).  Tile A's key-tile count equals the global
-          // key-tile counter, so ns names the V stage and phase.
-          ok = warp_wait(&s.v_full[ns % NS], (ns / NS) & 1, prm.err, abort_flag);
-          if (!ok) break;
-          if (r >= valid) {
-#pragma unroll
-            for (int cc = 0; cc < KC; ++cc) {
-              uint4* row = reinterpret_cast<uint4*>(s.v[ns % NS][cc] + r * 128);
-#pragma unroll
-              for (int u = 0; u < 8; ++u) row[u] = make_uint4(0, 0, 0, 0);
-            }
-          }
-          fence_proxy_async_smem();
+      if (w.alt) {
+        if (t == 1) {
+          // Warpgroup B has no tile here; tile A's scores use both regions.
+          // B still waits for each of the item's completions of s_full[1]
+          // in turn: a parity wait only tells phases apart when the phase
+          // before has completed, so B's next wait must not run ahead.
+          for (int i = 0; ok && i < w.nkv / 2; ++i, ++ns_t) ok = warp_wait(&s.s_full[1], ns_t & 1, prm.err, abort_flag);
+          continue;
         }
-        if (valid < BN / 2) {
-#pragma unroll
-          for (int i = 0; i < BN / 2; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+        for (int j = 0; ok && j < w.nkv; ++j, ++kt) {
+          const int sr = j & 1;
+          const uint32_t n = sr ? ns_b++ : ns_t++;
+          ok = key_tile(std::true_type{}, w, j, sr, n);
         }
-        // row max: eight independent chains of three-input max, then a tree
-        float mp[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
-#pragma unroll
-        for (int i = 16; i < BN / 2; i += 16)
-#pragma unroll
-          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
-        tmem_wait_ld_regs(&raw[64]);
-        if (valid < BN) {
-#pragma unroll
-          for (int i = BN / 2; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
-        }
-#pragma unroll
-        for (int i = BN / 2; i < BN; i += 16)
-#pragma unroll
-          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
-        const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
-        if (r == 0) ATTN_TRACE(2 + t, 26 + t, ns);
-        const float mt = mx * c;
-        float factor = 1.f;
-        bool need = false;
-        if (j == 0) {
-          m = mt;
-        } else if (mt > m + kRescaleThreshold) {
-          factor = ex2(m - mt);
-          m = mt;
-          need = true;
-        }
-        const float neg_m = -m;
-        // p = 2^(c*s - m): packed FMA for two scores, two SFU exponentials;
-        // the row sum runs in two packed accumulators (four lanes)
-        float rsum[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int q = 0; q < BN / 32; ++q) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            float a0, a1;
-            ffma2(a0, a1, x[32 * q + 2 * i], x[32 * q + 2 * i + 1], c, c, neg_m, neg_m);
-            const float p0 = ex2(a0);
-            const float p1 = ex2(a1);
-            const int h = (i & 1) * 2;
-            fadd2(rsum[h], rsum[h + 1], rsum[h], rsum[h + 1], p0, p1);
-            pk[i] = pack_bf16x2(p0, p1);
-          }
-          tmem_st16(s_addr + 16 * q, pk);
-        }
-        const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
-        if (r == 0) ATTN_TRACE(2 + t, 28 + t, ns);
-        // O is settled here (S of this tile was issued after the previous
-        // PV of this tile) and no MMA touches it before P is published
-        if (j > 0 && __any_sync(0xffffffffu, need)) {
-          uint32_t o[32];
-#pragma unroll 1
-          for (int q = 0; q < D / 32; ++q) {
-            tmem_ld32(o_addr + 32 * q, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
-            tmem_st32(o_addr + 32 * q, o);
-          }
-        }
-        l = (j == 0) ? rs : l * factor + rs;
-        tmem_wait_st();
-        tc_fence_before();
-        mbar_arrive(&s.p_full[t]);
-        if (r == 0) ATTN_TRACE(2 + t, 24 + t, ns);
+      } else {
+        if (t >= w.ntile) continue;  // B: a one-tile item completes no s_full[1]
+        for (int j = 0; ok && j < w.nkv; ++j, ++kt, ++ns_t) ok = key_tile(std::false_type{}, w, j, t, ns_t);
+        if (t == 0 && w.ntile == 2) ns_b += w.nkv;
       }
       if (!ok) break;
       // ------------------------------------------------------- epilogue
@@ -750,7 +837,7 @@ davet_status launch(const void* qkv, const int32_t* cu, const attn::FusedView& f
   prm.H = H;
   prm.max_rows = static_cast<int>(max_rows);
   prm.qtiles = 0;
-  prm.qt2_cost = 26;
+  prm.qt2_cost = 24;
   if (const char* e = std::getenv("DAVET_ATTN_QTILES")) prm.qtiles = std::atoi(e) == 1 ? 1 : (std::atoi(e) == 2 ? 2 : 0);
   prm.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
   prm.out = static_cast<uint16_t*>(out);

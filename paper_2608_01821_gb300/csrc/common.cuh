@@ -126,6 +126,17 @@ __device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1, 
       : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
+// (s0, s1) += the two bf16 halves of x (low half to s0), each widened
+// exactly to fp32: two mixed-precision adds (round to nearest)
+__device__ __forceinline__ void add_bf16x2_f32(float& s0, float& s1, uint32_t x) {
+  asm("{\n\t.reg .b16 lo, hi;\n\t"
+      "mov.b32 {lo, hi}, %2;\n\t"
+      "add.rn.f32.bf16 %0, lo, %0;\n\t"
+      "add.rn.f32.bf16 %1, hi, %1;\n\t}"
+      : "+f"(s0), "+f"(s1)
+      : "r"(x));
+}
+
 // ------------------------------------------------------------- smem, sync
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

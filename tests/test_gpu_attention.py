@@ -5,6 +5,11 @@ Tolerance for bf16 inputs: max |gpu - oracle| <= 1e-2 and relative L2 error
 ragged tails, empty and one-row requests, both head dimensions, garbage
 (non-finite) rows past the last request, and the full packed shapes of the
 8B-class workloads, checked on sampled (row, head) pairs.
+
+Work items hold one or two 128-row query tiles; the launch picks the count
+(DAVET_ATTN_QTILES forces 1 or 2).  One-tile items run their scores through
+both TMEM score regions in turn, two-tile items one region per tile, so the
+small cases run under each choice.
 """
 import math
 
@@ -17,6 +22,18 @@ from helpers import ATTN_MAX_ABS, ATTN_REL_L2, attn_errors, bf16_to_f64
 from paper_2608_01821_gb300 import workloads
 
 pytestmark = pytest.mark.gpu
+
+QTILES = ["auto", "1", "2"]
+
+
+@pytest.fixture(params=QTILES)
+def qtiles(request, monkeypatch):
+    """Query tiles per work item: chosen by the launch, or forced."""
+    if request.param == "auto":
+        monkeypatch.delenv("DAVET_ATTN_QTILES", raising=False)
+    else:
+        monkeypatch.setenv("DAVET_ATTN_QTILES", request.param)
+    return request.param
 
 
 def run(davet, qkv_cpu, cu, H, D, max_rows=None, garbage_tail=False):
@@ -45,7 +62,7 @@ def run(davet, qkv_cpu, cu, H, D, max_rows=None, garbage_tail=False):
     ([513, 64], 2, 64),
     ([1000], 1, 128),
 ])
-def test_dense_parity(davet, lens, H, D):
+def test_dense_parity(davet, qtiles, lens, H, D):
     cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
     N = int(cu[-1])
     qkv = workloads.qkv_rows(N, H, D, seed=sum(lens) + H + D)
@@ -57,7 +74,7 @@ def test_dense_parity(davet, lens, H, D):
     assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
 
 
-def test_rows_past_the_last_request_do_not_leak(davet):
+def test_rows_past_the_last_request_do_not_leak(davet, qtiles):
     H, D = 2, 128
     lens = [200, 77]
     cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
@@ -83,7 +100,7 @@ def test_identical_keys_give_mean_of_values(davet):
     assert np.abs(got - mean_v[None]).max() <= ATTN_MAX_ABS
 
 
-def test_growing_scores_force_the_rescale_path(davet):
+def test_growing_scores_force_the_rescale_path(davet, qtiles):
     # key norms grow along the sequence, so later key tiles carry maxima far
     # above the first tile's (by much more than 2^8 in the log2 domain) and
     # the running max must be raised and O rescaled; values are halved to
@@ -145,6 +162,31 @@ def test_last_round_split_into_one_tile_items(davet, L, H, nreq):
     last = cu[-2]  # the last request in the schedule (equal lengths: the highest index)
     rows = np.concatenate([np.arange(last, N), rng.integers(0, N, size=256)]).astype(np.int64)
     heads = np.concatenate([np.full(N - last, H - 1), rng.integers(0, H, size=256)]).astype(np.int32)
+    ref = oracle.attention_rows(qkv, cu, H, D, 1.0 / math.sqrt(D), rows, heads)
+    got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
+    max_abs, rel = attn_errors(got, ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
+
+
+@pytest.mark.parametrize("qt", ["1", "2"])
+def test_many_items_per_cta(davet, monkeypatch, qt):
+    """More work items than SMs, so every CTA runs several items in turn and
+    its barrier phases carry over between them: 2 requests (1,900 and 731
+    rows, ragged last tiles) x 40 heads; under one-tile items ~5.5 per CTA,
+    under two-tile items ~3, with a one-tile item for the 1,900-row
+    request's odd last tile in each head.
+    Three heads are compared in full, the others on sampled rows."""
+    monkeypatch.setenv("DAVET_ATTN_QTILES", qt)
+    H, D = 40, 128
+    lens = [1900, 731]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    qkv = workloads.qkv_rows(N, H, D, seed=11)
+    out = run(davet, qkv, cu, H, D)
+    rng = np.random.default_rng(12)
+    full = [0, 17, H - 1]
+    rows = np.concatenate([np.tile(np.arange(N), len(full)), rng.integers(0, N, size=512)]).astype(np.int64)
+    heads = np.concatenate([np.repeat(full, N), rng.integers(0, H, size=512)]).astype(np.int32)
     ref = oracle.attention_rows(qkv, cu, H, D, 1.0 / math.sqrt(D), rows, heads)
     got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
     max_abs, rel = attn_errors(got, ref)
