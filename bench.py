@@ -977,7 +977,11 @@ def run_reference(args, rank, world):
 
 def run_profile(args):
     """Minimal launch sequence for profilers: the workload's inputs for one
-    step and `--steps` launches of one kernel (after `--warmup` launches)."""
+    step and `--steps` launches of one kernel (after `--warmup` launches).
+    `--profile-view V` runs the step at view V for every request.  With
+    `--profile-time`, the `--steps` launches are then captured as one CUDA
+    graph and replayed three times (an L2 flush before each replay, not
+    timed); the line reports the best replay's time per launch."""
     import torch
 
     from paper_2608_01821_gb300 import davet, workloads
@@ -990,6 +994,10 @@ def run_profile(args):
     pl.load_inputs([workloads.features(w, b) for b in range(w.batch)], workloads.text_rows(w),
                    scores=[workloads.token_scores(w, b) for b in range(w.batch)] if realizer == "prune" else None)
     t = args.profile_step
+    if args.profile_view is not None:
+        if not 0 <= args.profile_view < w.n_levels + (1 if w.mixed else 0):
+            raise SystemExit(f"--profile-view {args.profile_view}: no such view in workload {w.name}")
+        pl.schedule[t].fill_(args.profile_view)
     lg = workloads.logits_device(w, t, dev)
     pl.build_pyramids()
     pl.gather(t)
@@ -999,8 +1007,33 @@ def run_profile(args):
     for _ in range(args.warmup + args.steps):
         fn()
     torch.cuda.synchronize()
+    us = None
+    if args.profile_time and args.profile != "unmask":
+        stream = torch.cuda.Stream(device=dev)
+        flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            fn()  # first use on this stream, outside the capture
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, stream=stream):
+            for _ in range(args.steps):
+                fn()
+        best = None
+        for rep in range(3):
+            with torch.cuda.stream(stream):
+                flush.fill_(rep)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                graph.replay()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        us = round(best * 1000.0 / max(args.steps, 1), 2)
     st, flags = lib.davet_device_status()
-    print(json.dumps({"profile": args.profile, "workload": w.name, "step": t, "status": st, "flags": flags}))
+    views = sorted(set(int(v) for v in pl.schedule[t].cpu().tolist()))
+    print(json.dumps({"profile": args.profile, "workload": w.name, "step": t, "views": views, "status": st,
+                      "flags": flags, "us_per_launch": us}))
     return 0 if st == 0 else 1
 
 
@@ -1062,6 +1095,10 @@ def main(argv=None):
     ap.add_argument("--profile", choices=["pyramid", "gather", "attention", "view_attention", "unmask"], default=None,
                     help="only set up one step and launch this kernel --steps times (for ncu captures)")
     ap.add_argument("--profile-step", type=int, default=0)
+    ap.add_argument("--profile-view", type=int, default=None,
+                    help="with --profile: run the step at this view for every request")
+    ap.add_argument("--profile-time", action="store_true",
+                    help="with --profile: time the --steps launches as one CUDA graph (best of 3 replays)")
     ap.add_argument("--policy", action="store_true",
                     help="choose every step's view with the closed-loop allocation policy on the device")
     ap.add_argument("--schedule", choices=["workload", "high", "mid", "low"], default="workload",
