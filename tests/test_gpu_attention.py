@@ -191,3 +191,42 @@ def test_many_items_per_cta(davet, monkeypatch, qt):
     got = bf16_to_f64(out[torch.as_tensor(rows, device="cuda"), torch.as_tensor(heads, device="cuda").long()])
     max_abs, rel = attn_errors(got, ref)
     assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
+
+
+def test_decreasing_boundaries_are_flagged_and_clamped(davet):
+    """cu_seqlens that go backwards: the call flags an argument error and
+    runs each request from the previous request's end (clamped), so
+    [0, 300, 200, 500] computes the requests [0, 300), [300, 300) and
+    [300, 500)."""
+    H, D = 2, 64
+    N = 500
+    qkv = workloads.qkv_rows(N, H, D, seed=23)
+    davet.davet_device_status(clear=True)
+    dev = torch.device("cuda")
+    qkv_d = qkv.to(dev)
+    out = torch.full((N, H, D), 3.0, dtype=torch.bfloat16, device=dev)
+    cu_d = torch.tensor([0, 300, 200, 500], dtype=torch.int32, device=dev)
+    davet.davet_step_attention(qkv_d, cu_d, 3, N, H, D, 1.0 / math.sqrt(D), out)
+    torch.cuda.synchronize()
+    st, flags = davet.davet_device_status(clear=True)
+    assert flags & 0x4 and st != 0
+    ref = oracle.attention(qkv, np.array([0, 300, 300, 500], np.int32), H, D, 1.0 / math.sqrt(D))
+    max_abs, rel = attn_errors(bf16_to_f64(out), ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)
+
+
+@pytest.mark.parametrize("nreq", [33, 70])
+def test_more_than_32_requests(davet, nreq):
+    """More than 32 requests (ragged, some empty): laid out 32 at a time and
+    ordered longest first by the whole CTA."""
+    H, D = 2, 64
+    rng = np.random.default_rng(nreq)
+    lens = [int(x) for x in rng.integers(0, 260, size=nreq)]
+    lens[3] = 0
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    N = int(cu[-1])
+    qkv = workloads.qkv_rows(N, H, D, seed=nreq + 1)
+    out = run(davet, qkv, cu, H, D)
+    ref = oracle.attention(qkv, cu, H, D, 1.0 / math.sqrt(D))
+    max_abs, rel = attn_errors(bf16_to_f64(out[:N]), ref)
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, (max_abs, rel)

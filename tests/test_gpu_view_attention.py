@@ -222,3 +222,23 @@ def test_fused_pipeline_full_size_matches_unfused(davet, name):
         assert torch.equal(pu.cu, pf.cu)
         n = int(pu.cu[-1])
         assert torch.equal(pu.attn_out[:n].view(torch.int16), pf.attn_out[:n].view(torch.int16)), (name, t)
+
+
+def test_fused_matches_unfused_more_than_32_requests(davet):
+    """40 requests (some empty, views mixed): the schedule lays out requests
+    32 at a time and orders more than 32 with the whole CTA."""
+    grid, levels, H, D = 12, 3, 2, 64
+    rng = np.random.default_rng(40)
+    B = 40
+    tiles = [int(x) for x in rng.integers(0, 3, size=B)]
+    prompt = [int(x) for x in rng.integers(0, 40, size=B)]
+    resp = [int(x) for x in rng.integers(0, 90, size=B)]
+    tiles[5], prompt[5], resp[5] = 0, 0, 0  # an empty request
+    view = [int(x) for x in rng.integers(0, levels, size=B)]
+    d = build_both(davet, tiles, prompt, resp, grid, levels, H, D, 41, (0, 0))
+    cap = sum(t * 144 + p + r for t, p, r in zip(tiles, prompt, resp))
+    out_a, cu_a, out_b, cu_b, _ = run_both(davet, d, tiles, prompt, resp, view, grid, levels, H, D, cap, (0, 0))
+    assert davet.davet_device_status() == (0, 0)
+    assert torch.equal(cu_a, cu_b)
+    n = int(cu_a[-1])
+    assert np.array_equal(bits(out_a[:n]), bits(out_b[:n]))
