@@ -17,14 +17,6 @@
 //                keep the same stale max, so the result is unchanged) and,
 //                after the last key tile, normalizes O and stores it as bf16.
 // TMEM: S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
-// The one-tile items of a launch with one tile per item, and the split
-// halves, run their key tiles as two streams: even key tiles through S_A
-// into O_A (warpgroup A), odd ones through S_B into O_B (warpgroup B), each
-// stream with its own running max and row sum; the MMA order is the same as
-// for two query tiles.  The epilogue merges the two (each warpgroup writes
-// half of the columns, reading both O).  A short sequence then runs half as
-// many serial key-tile steps.  The odd last tile of a request in a two-tile
-// launch runs as one stream (warpgroup B idles).
 // Items are ordered longest request first and, within a request,
 // head-major, so CTAs running together share a head's K/V in L2.  Keys past
 // the end of a request are masked to -inf and their V rows zeroed in shared
@@ -44,7 +36,6 @@
 #include <cstdio>
 #include <cstring>
 #include <mutex>
-#include <type_traits>
 
 #include "common.cuh"
 
@@ -77,8 +68,6 @@ struct Smem {
   uint64_t q_full, q_empty, fin;
   uint64_t k_full[NS], v_full[NS], k_empty[NS], v_empty[NS];
   uint64_t s_full[2], p_full[2], o_full[2];
-  uint64_t ml_full, ml_done;  // one-tile items: both streams' (m, l) written / both O read
-  float2 ml[2][BM];           // one-tile items: (running max, row sum) of each stream
   uint32_t tmem;
   int abort;
   int n_req;   // requests with at least one row
@@ -150,7 +139,6 @@ struct Item {
   int b;                              // request
   int start, len, q0, h, nkv, ntile;  // q0: first query row of the item within the request
   int kv0;  // key tile the item starts from (key tiles are visited cyclically)
-  bool alt;  // one query tile whose key tiles run as two streams, merged at the end
 
   // key tile visited at loop step j
   __device__ __forceinline__ int key_tile(int j) const {
@@ -194,21 +182,13 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
   // query blocks of one head start at evenly spread key tiles, so CTAs that
   // run together on the same head read different K/V lines at any moment
   const int qb = local - it.h * nq;
-  // (32-bit division when the product fits: a 64-bit one is a long
-  // subroutine, and every role decodes every item)
-  it.kv0 = (it.nkv < 65536 && qb < 65536)
-               ? static_cast<int>((static_cast<unsigned>(qb) * static_cast<unsigned>(it.nkv)) / static_cast<unsigned>(nq))
-               : static_cast<int>((static_cast<long long>(qb) * it.nkv) / nq);
+  it.kv0 = static_cast<int>((static_cast<long long>(qb) * it.nkv) / nq);
   it.ntile = (qtiles == 2 && it.q0 + BM < len) ? 2 : 1;
   if (half >= 0) {
     // a half whose tile lies past the request end computes rows it never stores
     it.q0 += half * BM;
     it.ntile = 1;
   }
-  // one-tile items of a one-tile launch and the split halves of the last
-  // round run as two key streams; the odd last tile of a request in a
-  // two-tile launch runs as one
-  it.alt = it.ntile == 1 && (qtiles == 1 || half >= 0);
   return it;
 }
 
@@ -216,254 +196,6 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned* err, volatile int* abort_flag) {
   const bool ok = mbar_wait(bar, parity, err, abort_flag);
   return __all_sync(0xffffffffu, ok);
-}
-
-// Per-thread constants of a softmax warpgroup thread.
-struct SoftmaxCtx {
-  int t;              // warpgroup: query tile of a two-tile item, or key stream
-  int r;              // query row within the tile == TMEM lane
-  uint32_t tmem_row;  // TMEM address of this thread's lane, column 0
-  float c;            // scale * log2(e)
-  int H;
-  uint16_t* out;
-  unsigned* err;
-  volatile int* abort_flag;
-};
-
-#ifdef DAVET_ATTN_TRACE
-#define ATTN_TRACE_PARAM , unsigned long long *trace_buf, unsigned &trace_n
-#define ATTN_TRACE_ARG , trace_buf, trace_n
-#else
-#define ATTN_TRACE_PARAM
-#define ATTN_TRACE_ARG
-#endif
-
-// Softmax of key tile j of item w: this thread's S row from TMEM region t,
-// running max m and row sum l, P (bf16) written back into the region, P
-// published on p_full[t].  ns: this completion of s_full[t]; kj: the CTA's
-// key-tile count, naming the V stage and phase.  TWO: one-tile item whose
-// key tiles run as two streams (this warpgroup's first key tile is t, and it
-// owns its ragged tiles); otherwise both tiles of an item read each key tile
-// and warpgroup A zeroes the ragged tile's V rows.
-template <int D, bool TWO, typename SM>
-__device__ __forceinline__ bool softmax_tile(SM& s, const SoftmaxCtx& cx, const Item& w, int j, uint32_t ns, uint32_t kj,
-                                             float& m, float& l ATTN_TRACE_PARAM) {
-  constexpr int KC = D / 64;
-  const int t = cx.t, r = cx.r;
-  const int t0 = TWO ? t : 0;
-  const bool zero_v = TWO || t == 0;
-  const float c = cx.c;
-  const uint32_t s_addr = cx.tmem_row + col_s(t);
-  const uint32_t o_addr = cx.tmem_row + col_o(t);
-  if (!warp_wait(&s.s_full[t], ns & 1, cx.err, cx.abort_flag)) return false;
-  if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
-  tc_fence_after();
-  // the row in two halves: the second half's TMEM load is in flight while
-  // the first half's max is taken
-  uint32_t raw[BN];
-  tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&raw[0]));
-  tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&raw[32]));
-  tmem_wait_ld_regs(&raw[0]);
-  tmem_ld32(s_addr + 64, *reinterpret_cast<uint32_t(*)[32]>(&raw[64]));
-  tmem_ld32(s_addr + 96, *reinterpret_cast<uint32_t(*)[32]>(&raw[96]));
-  if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
-  float* x = reinterpret_cast<float*>(raw);
-  const int valid = min(BN, w.len - w.key_tile(j) * BN);
-  if (zero_v && valid < BN) {
-    // keys past the request end: zero their V rows before PV reads them
-    // (P is 0 there, but the rows may hold anything, including non-finite
-    // values)
-    if (!warp_wait(&s.v_full[kj % NS], (kj / NS) & 1, cx.err, cx.abort_flag)) return false;
-    if (r >= valid) {
-#pragma unroll
-      for (int cc = 0; cc < KC; ++cc) {
-        uint4* row = reinterpret_cast<uint4*>(s.v[kj % NS][cc] + r * 128);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) row[u] = make_uint4(0, 0, 0, 0);
-      }
-    }
-    fence_proxy_async_smem();
-  }
-  if (valid < BN / 2) {
-#pragma unroll
-    for (int i = 0; i < BN / 2; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
-  }
-  // row max: eight independent chains of three-input max, then a tree
-  float mp[8];
-#pragma unroll
-  for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
-#pragma unroll
-  for (int i = 16; i < BN / 2; i += 16)
-#pragma unroll
-    for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
-  tmem_wait_ld_regs(&raw[64]);
-  if (valid < BN) {
-#pragma unroll
-    for (int i = BN / 2; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
-  }
-#pragma unroll
-  for (int i = BN / 2; i < BN; i += 16)
-#pragma unroll
-    for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
-  const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
-  if (r == 0) ATTN_TRACE(2 + t, 26 + t, ns);
-  const float mt = mx * c;
-  float factor = 1.f;
-  bool need = false;
-  if (j == t0) {
-    m = mt;
-  } else if (mt > m + kRescaleThreshold) {
-    factor = ex2(m - mt);
-    m = mt;
-    need = true;
-  }
-  const float neg_m = -m;
-  // p = 2^(c*s - m): packed FMA for two scores, two SFU exponentials,
-  // rounded to bf16.  The row sum adds the rounded weights, the values the PV
-  // MMA multiplies V by, so the weights applied to V sum to one after the
-  // final division (four accumulators).
-  float rsum[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-  for (int q = 0; q < BN / 32; ++q) {
-    uint32_t pk[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      float a0, a1;
-      ffma2(a0, a1, x[32 * q + 2 * i], x[32 * q + 2 * i + 1], c, c, neg_m, neg_m);
-      pk[i] = pack_bf16x2(ex2(a0), ex2(a1));
-      const int h = (i & 1) * 2;
-      add_bf16x2_f32(rsum[h], rsum[h + 1], pk[i]);
-    }
-    tmem_st16(s_addr + 16 * q, pk);
-  }
-  const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
-  if (r == 0) ATTN_TRACE(2 + t, 28 + t, ns);
-  // O is settled here (S of this key tile was issued after this stream's
-  // previous PV) and no MMA touches it before P is published
-  if (j > t0 && __any_sync(0xffffffffu, need)) {
-    uint32_t o[32];
-#pragma unroll 1
-    for (int q = 0; q < D / 32; ++q) {
-      tmem_ld32(o_addr + 32 * q, o);
-      tmem_wait_ld();
-#pragma unroll
-      for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
-      tmem_st32(o_addr + 32 * q, o);
-    }
-  }
-  l = (j == t0) ? rs : l * factor + rs;
-  tmem_wait_st();
-  tc_fence_before();
-  mbar_arrive(&s.p_full[t]);
-  if (r == 0) ATTN_TRACE(2 + t, 24 + t, ns);
-  return true;
-}
-
-// Stores query row `row0 + r` of item w: the accumulator at TMEM column
-// o_col, scaled by g, as bf16.
-template <int D>
-__device__ __forceinline__ void store_tile(const SoftmaxCtx& cx, const Item& w, int row0, uint32_t o_col, float g) {
-  const int qrow = w.q0 + row0 + cx.r;
-  const bool row_ok = qrow < w.len;
-  uint16_t* dst = cx.out + (static_cast<int64_t>(w.start + qrow) * cx.H + w.h) * D;
-#pragma unroll
-  for (int q = 0; q < D / 32; ++q) {
-    uint32_t o[32];
-    tmem_ld32(cx.tmem_row + o_col + 32 * q, o);
-    tmem_wait_ld();
-    if (row_ok) {
-      uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * q);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        uint4 v;
-        v.x = pack_bf16x2(__uint_as_float(o[8 * u + 0]) * g, __uint_as_float(o[8 * u + 1]) * g);
-        v.y = pack_bf16x2(__uint_as_float(o[8 * u + 2]) * g, __uint_as_float(o[8 * u + 3]) * g);
-        v.z = pack_bf16x2(__uint_as_float(o[8 * u + 4]) * g, __uint_as_float(o[8 * u + 5]) * g);
-        v.w = pack_bf16x2(__uint_as_float(o[8 * u + 6]) * g, __uint_as_float(o[8 * u + 7]) * g);
-        d4[u] = v;
-      }
-    }
-  }
-}
-
-struct StreamCounts {
-  uint32_t ns, kt, no, nm;  // completions of s_full[t]; key tiles; epilogues; merges
-  bool ok;
-};
-
-// A one-tile item whose key tiles run as two streams: warpgroup t runs key
-// tiles t, t+2, ... (its own running max m_t and row sum l_t, accumulator
-// O_t).  Epilogue, with m = max(m_A, m_B):
-//   O = (O_A 2^(m_A - m) + O_B 2^(m_B - m)) / (l_A 2^(m_A - m) + l_B 2^(m_B - m)),
-// warpgroup t writing columns [t D/2, (t+1) D/2) of each row from both
-// accumulators.  Two handshakes (bounded mbarrier waits): both (m, l)
-// written; both accumulators read before either warpgroup lets the next item
-// overwrite them.  With one key tile, stream B is empty and A stores alone.
-template <int D, typename SM>
-__device__ __noinline__ StreamCounts two_stream_item(SM& s, const SoftmaxCtx cx, const Item w,
-                                                     StreamCounts n ATTN_TRACE_PARAM) {
-  const int t = cx.t, r = cx.r;
-  float m = -INFINITY, l = 0.f;
-  for (int j = t; j < w.nkv; j += 2, ++n.ns)
-    if (!softmax_tile<D, true>(s, cx, w, j, n.ns, n.kt + j, m, l ATTN_TRACE_ARG)) {
-      n.ok = false;
-      return n;
-    }
-  if (t >= w.nkv) return n;  // one key tile: stream B is empty
-  n.ok = warp_wait(&s.o_full[t], n.no & 1, cx.err, cx.abort_flag);
-  ++n.no;
-  if (!n.ok) return n;
-  tc_fence_after();
-  if (w.nkv == 1) {
-    store_tile<D>(cx, w, 0, col_o(0), 1.f / l);
-    tc_fence_before();
-    return n;
-  }
-  s.ml[t][r] = make_float2(m, l);
-  tc_fence_before();
-  mbar_arrive(&s.ml_full);
-  n.ok = warp_wait(&s.ml_full, n.nm & 1, cx.err, cx.abort_flag);
-  if (!n.ok) return n;
-  tc_fence_after();
-  const float2 ma = s.ml[0][r], mb = s.ml[1][r];
-  const float mm = fmaxf(ma.x, mb.x);
-  const float fa = ex2(ma.x - mm), fb = ex2(mb.x - mm);
-  const float inv_l = 1.f / (ma.y * fa + mb.y * fb);
-  const float ga = fa * inv_l, gb = fb * inv_l;
-  constexpr int kHalf = D / 2;
-  const int qrow = w.q0 + r;
-  uint16_t* dst = cx.out + (static_cast<int64_t>(w.start + qrow) * cx.H + w.h) * D + t * kHalf;
-  const uint32_t base = cx.tmem_row + t * kHalf;
-#pragma unroll 1
-  for (int q = 0; q < kHalf / 32; ++q) {
-    uint32_t oa[32], ob[32];
-    tmem_ld32(base + col_o(0) + 32 * q, oa);
-    tmem_ld32(base + col_o(1) + 32 * q, ob);
-    tmem_wait_ld();
-    if (q == kHalf / 32 - 1) {
-      tc_fence_before();
-      mbar_arrive(&s.ml_done);  // both accumulators read
-    }
-    if (qrow < w.len) {
-      uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * q);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int i = 8 * u + 2 * e;
-          pk[e] = pack_bf16x2(__uint_as_float(oa[i]) * ga + __uint_as_float(ob[i]) * gb,
-                              __uint_as_float(oa[i + 1]) * ga + __uint_as_float(ob[i + 1]) * gb);
-        }
-        d4[u] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-      }
-    }
-  }
-  n.ok = warp_wait(&s.ml_done, n.nm & 1, cx.err, cx.abort_flag);
-  ++n.nm;
-  if (!n.ok) return n;
-  tc_fence_after();
-  return n;
 }
 
 template <int D, bool FUSED>
@@ -497,8 +229,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&s.p_full[t], 128);
       mbar_init(&s.o_full[t], 1);
     }
-    mbar_init(&s.ml_full, 256);
-    mbar_init(&s.ml_done, 256);
     fence_mbar_init();
   }
   if (warp == kWarpMma) {
@@ -592,15 +322,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         i1 += (L + BM - 1) / BM;
         i2 += (L + 2 * BM - 1) / (2 * BM);
       }
-      // rounds of items over the grid (32-bit division when the count fits:
-      // a 64-bit one is a long subroutine on the path every CTA waits for)
-      const unsigned g = gridDim.x;
-      auto rounds = [g](long long n) -> long long {
-        return n < 0x7fffffffLL ? static_cast<long long>((static_cast<unsigned>(n) + g - 1u) / g)
-                                : (n + g - 1) / static_cast<long long>(g);
-      };
-      const long long c1 = rounds(i1 * H) * 16;
-      const long long c2 = rounds(i2 * H) * prm.qt2_cost;
+      const long long g = gridDim.x;
+      const long long c1 = ((i1 * H + g - 1) / g) * 16;
+      const long long c2 = ((i2 * H + g - 1) / g) * prm.qt2_cost;
       qt = c2 <= c1 ? 2 : 1;
     }
     s.qtiles = qt;
@@ -691,27 +415,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t v_desc0 = sw128_desc(smem_u32(s.v[0][0]), kChunkBytes, 1024);
       constexpr uint32_t kTile16 = (KC * kChunkBytes) >> 4;  // one Q tile / K or V stage
       uint32_t it = 0, wi = 0;
-      uint32_t np0 = 0, np1 = 0;  // phases of p_full[0], p_full[1] consumed
+      uint32_t np[2] = {0, 0};  // P tiles consumed per query tile
       bool ok = true;
 
-      // S = Q_t K^T into score region r for the K tile in stage st
-      auto issue_s = [&](int t, int r, int st) {
+      // S_t = Q_t K^T for the K tile in stage st
+      auto issue_s = [&](int t, int st) {
         const uint64_t a0 = q_desc0 + t * kTile16;
         const uint64_t b0 = k_desc0 + st * kTile16;
-        const uint32_t d = tmem + col_s(r);
+        const uint32_t d = tmem + col_s(t);
         umma_ss_imm<false>(d, a0, b0, kIdescQK);
 #pragma unroll
         for (int kk = 1; kk < D / 16; ++kk) {
           const uint32_t off = ((kk >> 2) * kChunkBytes + (kk & 3) * 32) >> 4;
           umma_ss_imm<true>(d, a0 + off, b0 + off, kIdescQK);
         }
-        umma_commit(&s.s_full[r]);
+        umma_commit(&s.s_full[t]);
       };
-      // O_t (+)= P V for the V tile in stage st, P read from score region r
-      auto issue_pv = [&](int t, int r, int st, bool first) {
+      // O_t (+)= P_t V for the V tile in stage st, P read from TMEM
+      auto issue_pv = [&](int t, int st, bool first) {
         const uint64_t b0 = v_desc0 + st * kTile16;
         const uint32_t d = tmem + col_o(t);
-        const uint32_t a = tmem + col_s(r);
+        const uint32_t a = tmem + col_s(t);
         if (first)
           umma_ts_imm<false>(d, a, b0, kIdescPV);
         else
@@ -724,59 +448,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Item w = decode(s, item, H, qtiles);
         ok = mbar_wait(&s.q_full, wi & 1, prm.err, abort_flag);
         if (!ok) break;
-        if (w.alt) {
-          // One query tile whose key tiles form two streams: even key tiles
-          // through score region 0 into O_A (softmax warpgroup A), odd ones
-          // through region 1 into O_B (warpgroup B); the epilogue merges the
-          // two.  The order is that of two query tiles: S(0), S(1), then per
-          // key tile j PV(j) and S(j+2) of the same stream.
-          ok = mbar_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
-          if (!ok) break;
-          tc_fence_after();
-          issue_s(0, 0, it % NS);
-          umma_commit(&s.k_empty[it % NS]);
-          if (w.nkv > 1) {
-            ok = mbar_wait(&s.k_full[(it + 1) % NS], ((it + 1) / NS) & 1, prm.err, abort_flag);
-            if (!ok) break;
-            tc_fence_after();
-            issue_s(0, 1, (it + 1) % NS);
-            umma_commit(&s.k_empty[(it + 1) % NS]);
-          }
-          if (w.nkv <= 2) umma_commit(&s.q_empty);
-          for (int j = 0; j < w.nkv; ++j, ++it) {
-            const int st = it % NS;
-            const int r = j & 1;
-            ok = mbar_wait(&s.v_full[st], (it / NS) & 1, prm.err, abort_flag);
-            if (!ok) break;
-            const uint32_t npr = r ? np1++ : np0++;
-            ok = mbar_wait(&s.p_full[r], npr & 1, prm.err, abort_flag);
-            if (!ok) break;
-            tc_fence_after();
-            issue_pv(r, r, st, j < 2);
-            umma_commit(&s.v_empty[st]);
-            if (j + 2 < w.nkv) {
-              // S(j+2) overwrites the P that PV(j) reads: the tensor pipe
-              // runs the two in issue order
-              const int st2 = (it + 2) % NS;
-              ok = mbar_wait(&s.k_full[st2], ((it + 2) / NS) & 1, prm.err, abort_flag);
-              if (!ok) break;
-              tc_fence_after();
-              issue_s(0, r, st2);
-              umma_commit(&s.k_empty[st2]);
-              if (j + 2 == w.nkv - 1) umma_commit(&s.q_empty);
-            } else {
-              umma_commit(&s.o_full[r]);  // the stream's last PV
-            }
-          }
-          continue;
-        }
-        // one or two query tiles, one score region each: prologue, S of key
-        // tile 0
+        // prologue: S for key tile 0
         ok = mbar_wait(&s.k_full[it % NS], (it / NS) & 1, prm.err, abort_flag);
         if (!ok) break;
         tc_fence_after();
-        issue_s(0, 0, it % NS);
-        if (w.ntile == 2) issue_s(1, 1, it % NS);
+        issue_s(0, it % NS);
+        if (w.ntile == 2) issue_s(1, it % NS);
         umma_commit(&s.k_empty[it % NS]);
         if (w.nkv == 1) umma_commit(&s.q_empty);
         for (int j = 0; j < w.nkv; ++j, ++it) {
@@ -787,19 +464,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           ATTN_TRACE(1, 10, it);
           // tile A: PV, then S of the next key tile
-          ok = mbar_wait(&s.p_full[0], np0 & 1, prm.err, abort_flag);
+          ok = mbar_wait(&s.p_full[0], np[0] & 1, prm.err, abort_flag);
           if (!ok) break;
           ATTN_TRACE(1, 12, it);
-          ++np0;
+          ++np[0];
           tc_fence_after();
-          issue_pv(0, 0, st, j == 0);
+          issue_pv(0, st, j == 0);
           if (w.ntile == 1) umma_commit(&s.v_empty[st]);
           if (more) {
             ok = mbar_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
             if (!ok) break;
-            ATTN_TRACE(1, 11, it);
+              ATTN_TRACE(1, 11, it);
             tc_fence_after();
-            issue_s(0, 0, st1);
+            issue_s(0, st1);
             if (w.ntile == 1) {
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
@@ -809,15 +486,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (w.ntile == 2) {
             // tile B: PV, then S of the next key tile
-            ok = mbar_wait(&s.p_full[1], np1 & 1, prm.err, abort_flag);
+            ok = mbar_wait(&s.p_full[1], np[1] & 1, prm.err, abort_flag);
             if (!ok) break;
             ATTN_TRACE(1, 13, it);
-            ++np1;
+            ++np[1];
             tc_fence_after();
-            issue_pv(1, 1, st, j == 0);
+            issue_pv(1, st, j == 0);
             umma_commit(&s.v_empty[st]);
             if (more) {
-              issue_s(1, 1, st1);
+              issue_s(1, st1);
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
             } else {
@@ -832,45 +509,155 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------- softmax + epilogue
-    const int t = warp >> 2;  // query tile (or key stream) of this warpgroup
-    const int r = tid & 127;  // query row within the tile == TMEM lane
+    const int t = warp >> 2;             // query tile of this warpgroup
+    const int r = tid & 127;             // query row within the tile == TMEM lane
     const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    const SoftmaxCtx cx{t, r, tmem + lane_base, prm.scale_log2, H, prm.out, prm.err, abort_flag};
+    const uint32_t s_addr = tmem + lane_base + col_s(t);
+    const uint32_t o_addr = tmem + lane_base + col_o(t);
     ATTN_TRACE_DECL;
-    // ns_t: completions of s_full[t] so far; kt: key tiles of this CTA so
-    // far (they name the K/V stage and its phase); no: epilogues of this
-    // warpgroup; nm: merged epilogues (one-tile items of two streams).  Each
-    // warpgroup waits for every completion of its own s_full and o_full.
-    uint32_t ns_t = 0, kt = 0, no = 0, nm = 0;
+    const float c = prm.scale_log2;
+    uint32_t ns = 0, no = 0;
     bool ok = true;
     for (int item = blockIdx.x; ok && item < s.n_items; item += gridDim.x) {
       const Item w = decode(s, item, H, qtiles);
-      if (w.alt) {
-        // one query tile, two key streams: out of line, so that its
-        // registers do not weigh on the loop below
-        const StreamCounts n = two_stream_item<D>(s, cx, w, StreamCounts{ns_t, kt, no, nm, true} ATTN_TRACE_ARG);
-        ns_t = n.ns;
-        no = n.no;
-        nm = n.nm;
-        kt += w.nkv;
-        ok = n.ok;
-        continue;
-      }
-      if (t >= w.ntile) {
-        kt += w.nkv;
-        continue;
-      }
+      if (t >= w.ntile) continue;
       float m = -INFINITY;  // running max of c * score (log2 domain)
-      float l = 0.f;        // running sum of the bf16-rounded 2^(c*score - m)
-      for (int j = 0; ok && j < w.nkv; ++j, ++ns_t, ++kt)
-        ok = softmax_tile<D, false>(s, cx, w, j, ns_t, kt, m, l ATTN_TRACE_ARG);
+      float l = 0.f;        // running sum of 2^(c*score - m)
+      for (int j = 0; j < w.nkv; ++j, ++ns) {
+        ok = warp_wait(&s.s_full[t], ns & 1, prm.err, abort_flag);
+        if (!ok) break;
+        if (r == 0) ATTN_TRACE(2 + t, 20 + t, ns);
+        tc_fence_after();
+        // all four TMEM loads in flight before one wait
+        // the row in two halves: the second half's TMEM load is in flight
+        // while the first half's max is taken
+        uint32_t raw[BN];
+        tmem_ld32(s_addr, *reinterpret_cast<uint32_t(*)[32]>(&raw[0]));
+        tmem_ld32(s_addr + 32, *reinterpret_cast<uint32_t(*)[32]>(&raw[32]));
+        tmem_wait_ld_regs(&raw[0]);
+        tmem_ld32(s_addr + 64, *reinterpret_cast<uint32_t(*)[32]>(&raw[64]));
+        tmem_ld32(s_addr + 96, *reinterpret_cast<uint32_t(*)[32]>(&raw[96]));
+        if (r == 0) ATTN_TRACE(2 + t, 22 + t, ns);
+        float* x = reinterpret_cast<float*>(raw);
+        const int valid = min(BN, w.len - w.key_tile(j) * BN);
+        if (t == 0 && valid < BN) {
+          // keys past the request end: zero their V rows before PV reads them
+          // (P is 0 there, but the rows may hold anything, including
+          // non-finite values).  Tile A's key-tile count equals the global
+          // key-tile counter, so ns names the V stage and phase.
+          ok = warp_wait(&s.v_full[ns % NS], (ns / NS) & 1, prm.err, abort_flag);
+          if (!ok) break;
+          if (r >= valid) {
+#pragma unroll
+            for (int cc = 0; cc < KC; ++cc) {
+              uint4* row = reinterpret_cast<uint4*>(s.v[ns % NS][cc] + r * 128);
+#pragma unroll
+              for (int u = 0; u < 8; ++u) row[u] = make_uint4(0, 0, 0, 0);
+            }
+          }
+          fence_proxy_async_smem();
+        }
+        if (valid < BN / 2) {
+#pragma unroll
+          for (int i = 0; i < BN / 2; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+        }
+        // row max: eight independent chains of three-input max, then a tree
+        float mp[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) mp[u] = fmaxf(x[u], x[u + 8]);
+#pragma unroll
+        for (int i = 16; i < BN / 2; i += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+        tmem_wait_ld_regs(&raw[64]);
+        if (valid < BN) {
+#pragma unroll
+          for (int i = BN / 2; i < BN; ++i) x[i] = (i < valid) ? x[i] : -INFINITY;
+        }
+#pragma unroll
+        for (int i = BN / 2; i < BN; i += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mp[u] = fmax3(mp[u], x[i + u], x[i + 8 + u]);
+        const float mx = fmax3(fmax3(mp[0], mp[1], mp[2]), fmax3(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
+        if (r == 0) ATTN_TRACE(2 + t, 26 + t, ns);
+        const float mt = mx * c;
+        float factor = 1.f;
+        bool need = false;
+        if (j == 0) {
+          m = mt;
+        } else if (mt > m + kRescaleThreshold) {
+          factor = ex2(m - mt);
+          m = mt;
+          need = true;
+        }
+        const float neg_m = -m;
+        // p = 2^(c*s - m): packed FMA for two scores, two SFU exponentials,
+        // rounded to bf16.  The row sum adds the rounded weights, the values
+        // the PV MMA multiplies V by, so the weights applied to V sum to one
+        // after the final division (four accumulators).
+        float rsum[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < BN / 32; ++q) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            float a0, a1;
+            ffma2(a0, a1, x[32 * q + 2 * i], x[32 * q + 2 * i + 1], c, c, neg_m, neg_m);
+            pk[i] = pack_bf16x2(ex2(a0), ex2(a1));
+            const int h = (i & 1) * 2;
+            add_bf16x2_f32(rsum[h], rsum[h + 1], pk[i]);
+          }
+          tmem_st16(s_addr + 16 * q, pk);
+        }
+        const float rs = (rsum[0] + rsum[1]) + (rsum[2] + rsum[3]);
+        if (r == 0) ATTN_TRACE(2 + t, 28 + t, ns);
+        // O is settled here (S of this tile was issued after the previous
+        // PV of this tile) and no MMA touches it before P is published
+        if (j > 0 && __any_sync(0xffffffffu, need)) {
+          uint32_t o[32];
+#pragma unroll 1
+          for (int q = 0; q < D / 32; ++q) {
+            tmem_ld32(o_addr + 32 * q, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+            tmem_st32(o_addr + 32 * q, o);
+          }
+        }
+        l = (j == 0) ? rs : l * factor + rs;
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&s.p_full[t]);
+        if (r == 0) ATTN_TRACE(2 + t, 24 + t, ns);
+      }
       if (!ok) break;
       // ------------------------------------------------------- epilogue
       ok = warp_wait(&s.o_full[t], no & 1, prm.err, abort_flag);
       ++no;
       if (!ok) break;
       tc_fence_after();
-      store_tile<D>(cx, w, t * BM, col_o(t), 1.f / l);
+      const float inv_l = 1.f / l;
+      const int qrow = w.q0 + t * BM + r;
+      const bool row_ok = qrow < w.len;
+      uint16_t* dst = prm.out + (static_cast<int64_t>(w.start + qrow) * H + w.h) * D;
+#pragma unroll
+      for (int q = 0; q < D / 32; ++q) {
+        uint32_t o[32];
+        tmem_ld32(o_addr + 32 * q, o);
+        tmem_wait_ld();
+        if (row_ok) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + 32 * q);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(o[8 * u + 0]) * inv_l, __uint_as_float(o[8 * u + 1]) * inv_l);
+            v.y = pack_bf16x2(__uint_as_float(o[8 * u + 2]) * inv_l, __uint_as_float(o[8 * u + 3]) * inv_l);
+            v.z = pack_bf16x2(__uint_as_float(o[8 * u + 4]) * inv_l, __uint_as_float(o[8 * u + 5]) * inv_l);
+            v.w = pack_bf16x2(__uint_as_float(o[8 * u + 6]) * inv_l, __uint_as_float(o[8 * u + 7]) * inv_l);
+            d4[u] = v;
+          }
+        }
+      }
       tc_fence_before();
     }
   }

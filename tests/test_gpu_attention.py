@@ -7,9 +7,9 @@ ragged tails, empty and one-row requests, both head dimensions, garbage
 8B-class workloads, checked on sampled (row, head) pairs.
 
 Work items hold one or two 128-row query tiles; the launch picks the count
-(DAVET_ATTN_QTILES forces 1 or 2).  One-tile items split their key tiles
-between two streams (two accumulators merged at the end), two-tile items run
-one stream per tile, so the small cases run under each choice.
+(DAVET_ATTN_QTILES forces 1 or 2); the two kinds of item take different
+paths through the MMA issuer and the softmax warpgroups, so the small cases
+run under each choice.
 """
 import math
 
