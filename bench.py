@@ -600,6 +600,24 @@ def kernel_times(pl, w, pool, P, stream, flush, reps=3, policy_pass=None, policy
 
     graphs = {"pyramid": graph_of(pl.build_pyramids), "reset": graph_of(pl.reset_state),
               "unmask": graph_of(unmask_all)}
+    scratch = []
+    if pl.fused and pl.realizer == "pool":
+        # the pyramid kernel alone (the view-block build also runs the text
+        # fill): each request's level 0 copied into a level-major scratch
+        # pyramid, pooled there with davet_build_pyramid (the same kernel and
+        # bytes as inside davet_build_views)
+        for b in range(w.batch):
+            if w.tiles[b] > 0:
+                buf = torch.empty((w.pyramid_rows(b), w.C), dtype=torch.bfloat16, device=pl.dev)
+                l0 = pl.level0(b)
+                buf[:l0.shape[0]].copy_(l0)
+                scratch.append((b, buf))
+
+        def pyramid_kernels():
+            for b, buf in scratch:
+                pl.lib.davet_build_pyramid(buf, buf, w.tiles[b], w.grid, w.n_levels, w.C, None, stream)
+
+        graphs["pyramid_kernel"] = graph_of(pyramid_kernels)
     if pl.fused:
         graphs["view_attention"] = graph_of(attn_all)
     else:
@@ -609,6 +627,8 @@ def kernel_times(pl, w, pool, P, stream, flush, reps=3, policy_pass=None, policy
         graphs["policy"] = graph_of(policy_all)
     torch.cuda.synchronize()
     totals = {k: time_graph(g) for k, g in graphs.items()}
+    pk_ms = totals.pop("pyramid_kernel", None)
+    del scratch
     totals["unmask"] = max(totals["unmask"] - totals["reset"], 0.0)
     if not pl.fused:
         totals["attention"] = max(totals.pop("gather+attention") - totals["gather"], 0.0)
@@ -628,6 +648,11 @@ def kernel_times(pl, w, pool, P, stream, flush, reps=3, policy_pass=None, policy
                         "bytes_with_fill": pbytes + w.view_fill_bytes(),
                         "GBps_with_fill": (pbytes + w.view_fill_bytes()) / (ms["pyramid"] * 1e-3) / 1e9},
         }
+        if pk_ms:
+            out["pyramid"]["pyramid_kernel"] = {
+                "launches": sum(1 for t in w.tiles if t > 0), "ms": pk_ms, "bytes": pbytes,
+                "GBps": pbytes / (pk_ms * 1e-3) / 1e9,
+                "what": "the pyramid kernel alone (davet_build_pyramid on a level-major copy of level 0)"}
     else:
         out = {
             "timing_mode": mode,

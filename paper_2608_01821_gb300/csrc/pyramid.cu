@@ -172,11 +172,13 @@ __device__ __forceinline__ bool subtree(const Ctx& c, const Geom& g, int y, int 
       for (int qq = 0; qq < 4; ++qq) {
         const int i = 2 * a + (qq >> 1), j = 2 * b + (qq & 1);
         if (y * S + i < g0 && x * S + j < g0) {
+          // each bf16 widened exactly and added in fp32: one mixed-precision
+          // add per value instead of a widening plus an add
           const uint4 u = leaf[i * S + j];
-          acc[0] += bf16lo(u.x); acc[1] += bf16hi(u.x);
-          acc[2] += bf16lo(u.y); acc[3] += bf16hi(u.y);
-          acc[4] += bf16lo(u.z); acc[5] += bf16hi(u.z);
-          acc[6] += bf16lo(u.w); acc[7] += bf16hi(u.w);
+          add_bf16x2_f32(acc[0], acc[1], u.x);
+          add_bf16x2_f32(acc[2], acc[3], u.y);
+          add_bf16x2_f32(acc[4], acc[5], u.z);
+          add_bf16x2_f32(acc[6], acc[7], u.w);
           ++n;
         }
       }
