@@ -323,9 +323,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         i2 += (L + 2 * BM - 1) / (2 * BM);
       }
       const long long g = gridDim.x;
-      const long long c1 = ((i1 * H + g - 1) / g) * 16;
-      const long long c2 = ((i2 * H + g - 1) / g) * prm.qt2_cost;
-      qt = c2 <= c1 ? 2 : 1;
+      if (i1 * H <= g) {
+        qt = 1;  // one round of one-tile items: two tiles cannot take fewer rounds
+      } else {
+        // rounds of items over the grid (32-bit division when the counts
+        // fit: a 64-bit one is a long subroutine on the path every CTA waits for)
+        auto rounds = [g](long long n) -> long long {
+          return n < 0x7fffffffLL ? static_cast<long long>((static_cast<unsigned>(n) + static_cast<unsigned>(g) - 1u) /
+                                                           static_cast<unsigned>(g))
+                                  : (n + g - 1) / g;
+        };
+        const long long c1 = rounds(i1 * H) * 16;
+        const long long c2 = rounds(i2 * H) * prm.qt2_cost;
+        qt = c2 <= c1 ? 2 : 1;
+      }
     }
     s.qtiles = qt;
     int acc = 0;
