@@ -170,8 +170,9 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
   const int b = s.order[lo];
   const int local = item - s.cum[lo];
   const int len = s.req_len[b];
-  const int rows_per_item = BM * qtiles;
-  const int nq = (len + rows_per_item - 1) / rows_per_item;
+  const int shift = qtiles == 2 ? 8 : 7;  // log2 of the rows per item
+  const int rows_per_item = 1 << shift;
+  const int nq = (len + rows_per_item - 1) >> shift;
   Item it;
   it.b = b;
   it.start = s.req_start[b];
@@ -182,7 +183,11 @@ __device__ __forceinline__ Item decode(const S& s, int item, int H, int qtiles) 
   // query blocks of one head start at evenly spread key tiles, so CTAs that
   // run together on the same head read different K/V lines at any moment
   const int qb = local - it.h * nq;
-  it.kv0 = static_cast<int>((static_cast<long long>(qb) * it.nkv) / nq);
+  // (32-bit division when the product fits: a 64-bit one is a long
+  // subroutine, and every role decodes every item)
+  const long long qk = static_cast<long long>(qb) * it.nkv;
+  it.kv0 = qk < 0x7fffffffLL ? static_cast<int>(static_cast<unsigned>(qk) / static_cast<unsigned>(nq))
+                             : static_cast<int>(qk / nq);
   it.ntile = (qtiles == 2 && it.q0 + BM < len) ? 2 : 1;
   if (half >= 0) {
     // a half whose tile lies past the request end computes rows it never stores
