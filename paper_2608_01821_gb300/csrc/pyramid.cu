@@ -254,14 +254,26 @@ __global__ void pyramid_kernel(const uint4* __restrict__ feat, uint4* __restrict
     const int chunks = (g.C8 + 63) / 64;
     const long long units = static_cast<long long>(g.n_tiles) * cells * chunks;
     for (long long u = blockIdx.x; u < units; u += gridDim.x) {
-      const int chunk = static_cast<int>(u % chunks);
-      const long long rest = u / chunks;
-      const int cellid = static_cast<int>(rest % cells);
+      // 32-bit divisions while the unit count fits (a 64-bit division is a
+      // long subroutine)
+      int chunk, cellid, tile;
+      if (units <= 0xffffffffLL) {
+        const unsigned u32 = static_cast<unsigned>(u);
+        const unsigned rest32 = u32 / static_cast<unsigned>(chunks);
+        chunk = static_cast<int>(u32 - rest32 * static_cast<unsigned>(chunks));
+        cellid = static_cast<int>(rest32 % static_cast<unsigned>(cells));
+        tile = static_cast<int>(rest32 / static_cast<unsigned>(cells));
+      } else {
+        chunk = static_cast<int>(u % chunks);
+        const long long rest = u / chunks;
+        cellid = static_cast<int>(rest % cells);
+        tile = static_cast<int>(rest / cells);
+      }
       Ctx c;
       c.feat = feat;
       c.pyr = pyr;
       c.pyr32 = pyr32;
-      c.tile = static_cast<int>(rest / cells);
+      c.tile = tile;
       c.cv = chunk * 64 + cv_local;
       const int Y = cellid / gt, X = cellid % gt;
       float v[8];

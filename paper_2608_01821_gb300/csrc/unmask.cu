@@ -215,9 +215,11 @@ __global__ void __launch_bounds__(kRowThreads) row_kernel(RowArgs a) {
   const long long unit = (static_cast<long long>(blockIdx.x) * kRowThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (unit >= a.total_rows * a.nchunk) return;
-  const long long row = unit / a.nchunk;
+  // unit < 2^31 (rows and chunks are bounded on the host): a 32-bit division
+  const unsigned u32 = static_cast<unsigned>(unit);
+  const long long row = u32 / static_cast<unsigned>(a.nchunk);
   if (!a.masked[row]) return;
-  const int ch = static_cast<int>(unit - row * a.nchunk);
+  const int ch = static_cast<int>(u32 - static_cast<unsigned>(row) * static_cast<unsigned>(a.nchunk));
   const int lo = ch * a.chunk, hi = min(a.V8, lo + a.chunk);
   const uint4* base = a.logits + row * static_cast<long long>(a.V8);
   Run run = empty_run();
@@ -514,9 +516,11 @@ __global__ void __launch_bounds__(kRowThreads) stage_kernel(const uint4* __restr
   const long long unit = (static_cast<long long>(blockIdx.x) * kRowThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (unit >= total_rows * nchunk) return;
-  const long long row = unit / nchunk;
+  // unit < 2^31 (rows and chunks are bounded on the host): a 32-bit division
+  const unsigned u32 = static_cast<unsigned>(unit);
+  const long long row = u32 / static_cast<unsigned>(nchunk);
   if (!masked[row]) return;
-  const int ch = static_cast<int>(unit - row * nchunk);
+  const int ch = static_cast<int>(u32 - static_cast<unsigned>(row) * static_cast<unsigned>(nchunk));
   const int lo = ch * chunk, hi = min(V8, lo + chunk);
   const uint4* s = src + row * static_cast<long long>(V8);
   uint4* d = dst + row * static_cast<long long>(V8);
