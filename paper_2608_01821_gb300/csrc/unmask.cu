@@ -257,11 +257,11 @@ struct SelArgs {
 };
 
 // Warp arg-max of (conf, -pos): the winning (conf, pos) on every lane.
-__device__ __forceinline__ void warp_best(float& c, long long& pos) {
+__device__ __forceinline__ void warp_best(float& c, int& pos) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float c2 = __shfl_xor_sync(0xffffffffu, c, o);
-    const long long p2 = __shfl_xor_sync(0xffffffffu, pos, o);
+    const int p2 = __shfl_xor_sync(0xffffffffu, pos, o);
     if (c2 > c || (c2 == c && p2 < pos)) {
       c = c2;
       pos = p2;
@@ -403,19 +403,21 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
   // top-k: k rounds of a warp arg-max over the rows still masked
   const int take = min(a.k, tot_masked);
   int j = 0;
+  // (positions in 32 bits: a request has fewer than 2^31 rows)
+  const int n32 = static_cast<int>(n);
   for (; j < take; ++j) {
     float best_c = -2.f;
-    long long best_pos = LLONG_MAX;
-    for (long long i = lane; i < n; i += 32) {
+    int best_pos = INT_MAX;
+    for (int i = lane; i < n32; i += 32) {
       const float c = cbuf[i];
       if (c > best_c || (c == best_c && i < best_pos)) {
         best_c = c;
         best_pos = i;
       }
     }
-    const long long mine = best_pos;
+    const int mine = best_pos;
     warp_best(best_c, best_pos);
-    if (best_pos == LLONG_MAX) break;  // only when confidences are not numbers
+    if (best_pos == INT_MAX) break;  // only when confidences are not numbers
     if (mine == best_pos) {
       a.tokens[s0 + best_pos] = ibuf[best_pos];
       a.masked[s0 + best_pos] = 0;
