@@ -298,8 +298,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     s.n_req = n;
   }
   __syncthreads();
-  // longest request first (stable); only for modest batches
-  if (s.n_req <= kLptMaxBatch) {
+  // longest request first (stable); only for modest batches (one request
+  // is already in order)
+  if (s.n_req > 1 && s.n_req <= kLptMaxBatch) {
     int my_b = -1, my_rank = 0;
     if (tid < s.n_req) {
       my_b = s.order[tid];
