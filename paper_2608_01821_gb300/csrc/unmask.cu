@@ -430,6 +430,112 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
     for (int q = j + lane; q < a.k; q += 32) a.committed[static_cast<long long>(b) * a.k + q] = -1;
 }
 
+// The row pass with bulk copies: each warp's (row, chunk) unit arrives in
+// 4 KB pieces through the copy engine of the SM (cp.async.bulk into shared
+// memory, two pieces in flight per warp), not through L1, then folds from
+// shared memory.  Each lane folds the same elements in the same order as in
+// row_kernel, so the results are bit-identical.
+constexpr int kPiece = 256;  // 16-byte slices per bulk piece (4 KB)
+
+struct RowStage {  // one warp's two pieces and their barriers
+  uint4 buf[2][kPiece];
+  uint64_t bar[2];
+};
+constexpr size_t kRowBulkSmem = sizeof(RowStage) * (kRowThreads / 32);
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__global__ void __launch_bounds__(kRowThreads) row_kernel_bulk(RowArgs a, unsigned* err) {
+  extern __shared__ __align__(128) uint8_t row_smem[];
+  RowStage* ws = reinterpret_cast<RowStage*>(row_smem) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (lane == 0) {
+    mbar_init(&ws->bar[0], 1);
+    mbar_init(&ws->bar[1], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  pdl_launch_dependents();
+  pdl_wait();
+  const long long unit = (static_cast<long long>(blockIdx.x) * kRowThreads + threadIdx.x) >> 5;
+  if (unit >= a.total_rows * a.nchunk) return;
+  // unit < 2^31 (rows and chunks are bounded on the host): a 32-bit division
+  const unsigned u32 = static_cast<unsigned>(unit);
+  const long long row = u32 / static_cast<unsigned>(a.nchunk);
+  if (!a.masked[row]) return;
+  const int ch = static_cast<int>(u32 - static_cast<unsigned>(row) * static_cast<unsigned>(a.nchunk));
+  const int lo = ch * a.chunk, hi = min(a.V8, lo + a.chunk);
+  const int n = hi - lo;
+  const int npieces = (n + kPiece - 1) / kPiece;
+  const uint4* src = a.logits + row * static_cast<long long>(a.V8) + lo;
+  auto issue = [&](int p) {  // lane 0
+    const int sl = p & 1;
+    const int cnt = min(kPiece, n - p * kPiece);
+    mbar_arrive_expect_tx(&ws->bar[sl], static_cast<uint32_t>(cnt) * 16u);
+    bulk_g2s(&ws->buf[sl][0], src + p * kPiece, static_cast<uint32_t>(cnt) * 16u, &ws->bar[sl]);
+  };
+  if (lane == 0) {
+    issue(0);
+    if (npieces > 1) issue(1);
+  }
+  Run run = empty_run();
+  int p = 0;
+  for (; p < npieces; ++p) {
+    const int sl = p & 1;
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&ws->bar[sl], (p >> 1) & 1, err, nullptr));
+    if (!ok) break;
+    const int cnt = min(kPiece, n - p * kPiece);
+    const int w0 = (lo + p * kPiece) * 8;
+    for (int k = lane; k < cnt; k += 32) fold(run, ws->buf[sl][k], w0 + k * 8);
+    __syncwarp();
+    if (lane == 0 && p + 2 < npieces) {
+      fence_proxy_async_smem();  // the warp's reads of this piece before the copy's writes
+      issue(p + 2);
+    }
+  }
+  if (p < npieces) {
+    // a wait gave up: let the copies still in flight land before the warp
+    // leaves (bounded), and write nothing
+    if (lane == 0)
+      for (int q = p; q < min(npieces, p + 2); ++q) mbar_wait(&ws->bar[q & 1], (q >> 1) & 1, nullptr, nullptr);
+    return;
+  }
+  const Partial pt = warp_combine(to_partial(run));
+  // chunk-major, so the select's row-per-thread loads are coalesced
+  if (lane == 0) a.partial[static_cast<long long>(ch) * a.total_rows + row] = pt;
+}
+
+// Whether p is device memory (the bulk row pass reads only device memory;
+// pinned host memory mapped for the device takes the plain-load pass).
+inline bool device_memory(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice;
+}
+
+// The bulk row pass's dynamic shared memory limit, once per device.
+inline cudaError_t set_row_bulk_smem() {
+  static std::mutex mu;
+  static bool done[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> g(mu);
+  if (done[dev]) return cudaSuccess;
+  e = cudaFuncSetAttribute(row_kernel_bulk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kRowBulkSmem));
+  if (e == cudaSuccess) done[dev] = true;
+  return e;
+}
+
 // Both kernels of one call on `stream`, over the workspace `ws` (layout L).
 inline davet_status enqueue(const void* logits, int V, const int32_t* cu, int batch, int64_t total_rows, int k,
                             uint8_t* masked, int32_t* tokens, int32_t* argmax, float* conf, int32_t* committed,
@@ -448,7 +554,16 @@ inline davet_status enqueue(const void* logits, int V, const int32_t* cu, int ba
     r.partial = partial;
     const long long warps = total_rows * L.nchunk;
     const long long blocks = (warps + kRowThreads / 32 - 1) / (kRowThreads / 32);
-    const cudaError_t e = launch(row_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kRowThreads), 0, stream, r);
+    cudaError_t e;
+    if (device_memory(logits)) {
+      e = set_row_bulk_smem();
+      if (e == cudaSuccess)
+        e = launch(row_kernel_bulk, dim3(static_cast<unsigned>(blocks)), dim3(kRowThreads), kRowBulkSmem, stream, r,
+                   err);
+    } else {
+      // host-mapped logits: plain loads
+      e = launch(row_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kRowThreads), 0, stream, r);
+    }
     if (e != cudaSuccess) return cuda_fail(e);
   }
   SelArgs a;
