@@ -101,7 +101,7 @@ __device__ __forceinline__ Partial warp_combine(Partial p) {
   float mx = p.m;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  float sm = p.s > 0.f ? p.s * sfu_ex2((p.m - mx) * kLog2e) : 0.f;
+  float sm = p.s > 0.f ? __fmul_rn(p.s, sfu_ex2((p.m - mx) * kLog2e)) : 0.f;
   int ix = p.m == mx ? p.idx : INT_MAX;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -167,8 +167,10 @@ __device__ __forceinline__ void fold(Run& r, uint4 u, int w0) {
       first = (xk == vm) ? k : first;
     }
     r.idx = w0 + first;
-    const float ml = vm * kLog2e;
-    const float f = r.s0 + r.s1 > 0.f ? sfu_ex2(r.ml - ml) : 0.f;
+    // explicit roundings: no contraction into an FMA, which could differ
+    // between the kernels this is inlined into
+    const float ml = __fmul_rn(vm, kLog2e);
+    const float f = r.s0 + r.s1 > 0.f ? sfu_ex2(__fsub_rn(r.ml, ml)) : 0.f;
     r.s0 *= f;
     r.s1 *= f;
     r.m = vm;
@@ -188,6 +190,71 @@ __device__ __forceinline__ void fold(Run& r, uint4 u, int w0) {
   fadd2(t2, t3, e[4], e[5], e[6], e[7]);
   fadd2(t0, t1, t0, t1, t2, t3);
   fadd2(r.s0, r.s1, r.s0, r.s1, t0, t1);
+}
+
+// Fold a lane's batch of kLoads slices: u[m] holds the 8 logits from
+// vocabulary index w0 + 256 m (the lane's slices of one piece, 32 slices
+// apart).  The batch's max is found first, by one tree of packed bf16 maxima,
+// so the running max, its first index and the rescale are updated at most
+// once per batch (first index: lowest m, then lowest position in the
+// slice); the terms of every slice are then summed as in fold, relative to
+// the batch's running max.
+__device__ __forceinline__ void fold_batch(Run& r, const uint4 (&u)[kLoads], int w0) {
+  uint32_t sm[kLoads];
+#pragma unroll
+  for (int m = 0; m < kLoads; ++m) sm[m] = max_bf16x2(max_bf16x2(u[m].x, u[m].y), max_bf16x2(u[m].z, u[m].w));
+  uint32_t t[kLoads / 2];
+#pragma unroll
+  for (int m = 0; m < kLoads / 2; ++m) t[m] = max_bf16x2(sm[2 * m], sm[2 * m + 1]);
+  const uint32_t bm = max_bf16x2(max_bf16x2(t[0], t[1]), max_bf16x2(t[2], t[3]));
+  const float vm = fmaxf(bf16lo(bm), bf16hi(bm));
+  if (vm > r.m) {
+    // the first slice holding vm, then its first position
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+    int fm = 0;
+#pragma unroll
+    for (int m = kLoads - 1; m >= 0; --m) {
+      if (fmaxf(bf16lo(sm[m]), bf16hi(sm[m])) == vm) {
+        fm = m;
+        w[0] = u[m].x;
+        w[1] = u[m].y;
+        w[2] = u[m].z;
+        w[3] = u[m].w;
+      }
+    }
+    int first = 7;
+#pragma unroll
+    for (int k = 7; k >= 0; --k) {
+      const float xk = (k & 1) ? bf16hi(w[k >> 1]) : bf16lo(w[k >> 1]);
+      first = (xk == vm) ? k : first;
+    }
+    r.idx = w0 + 256 * fm + first;
+    // explicit roundings: no contraction into an FMA, which could differ
+    // between the kernels this is inlined into
+    const float ml = __fmul_rn(vm, kLog2e);
+    const float f = r.s0 + r.s1 > 0.f ? sfu_ex2(__fsub_rn(r.ml, ml)) : 0.f;
+    r.s0 *= f;
+    r.s1 *= f;
+    r.m = vm;
+    r.ml = ml;
+  }
+  const float nm = -r.ml;
+#pragma unroll
+  for (int m = 0; m < kLoads; ++m) {
+    float a[8];
+    ffma2(a[0], a[1], bf16lo(u[m].x), bf16hi(u[m].x), kLog2e, kLog2e, nm, nm);
+    ffma2(a[2], a[3], bf16lo(u[m].y), bf16hi(u[m].y), kLog2e, kLog2e, nm, nm);
+    ffma2(a[4], a[5], bf16lo(u[m].z), bf16hi(u[m].z), kLog2e, kLog2e, nm, nm);
+    ffma2(a[6], a[7], bf16lo(u[m].w), bf16hi(u[m].w), kLog2e, kLog2e, nm, nm);
+    float e[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) e[k] = sfu_ex2(a[k]);
+    float t0, t1, t2, t3;
+    fadd2(t0, t1, e[0], e[1], e[2], e[3]);
+    fadd2(t2, t3, e[4], e[5], e[6], e[7]);
+    fadd2(t0, t1, t0, t1, t2, t3);
+    fadd2(r.s0, r.s1, r.s0, r.s1, t0, t1);
+  }
 }
 
 __device__ __forceinline__ Partial to_partial(const Run& r) {
@@ -229,9 +296,13 @@ __global__ void __launch_bounds__(kRowThreads) row_kernel(RowArgs a) {
 #pragma unroll
     for (int k = 0; k < kLoads; ++k)
       if (v + 32 * k < hi) u[k] = ld_stream(base + v + 32 * k);
+    if (v + 32 * (kLoads - 1) < hi) {
+      fold_batch(run, u, v * 8);
+    } else {
 #pragma unroll
-    for (int k = 0; k < kLoads; ++k)
-      if (v + 32 * k < hi) fold(run, u[k], (v + 32 * k) * 8);
+      for (int k = 0; k < kLoads; ++k)
+        if (v + 32 * k < hi) fold(run, u[k], (v + 32 * k) * 8);
+    }
   }
   const Partial p = warp_combine(to_partial(run));
   // chunk-major, so the select's row-per-thread loads are coalesced
@@ -436,6 +507,7 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(SelArgs a) {
 // shared memory.  Each lane folds the same elements in the same order as in
 // row_kernel, so the results are bit-identical.
 constexpr int kPiece = 256;  // 16-byte slices per bulk piece (4 KB)
+static_assert(kPiece == 32 * kLoads, "a lane's slices of a piece are one batch of row_kernel");
 
 struct RowStage {  // one warp's two pieces and their barriers
   uint4 buf[2][kPiece];
@@ -490,7 +562,16 @@ __global__ void __launch_bounds__(kRowThreads) row_kernel_bulk(RowArgs a, unsign
     if (!ok) break;
     const int cnt = min(kPiece, n - p * kPiece);
     const int w0 = (lo + p * kPiece) * 8;
-    for (int k = lane; k < cnt; k += 32) fold(run, ws->buf[sl][k], w0 + k * 8);
+    // the lane's slices of the piece are those of one plain-load iteration
+    // of row_kernel, folded the same way (bit-identical results)
+    if (lane + 32 * (kLoads - 1) < cnt) {
+      uint4 u[kLoads];
+#pragma unroll
+      for (int m = 0; m < kLoads; ++m) u[m] = ws->buf[sl][lane + 32 * m];
+      fold_batch(run, u, w0 + lane * 8);
+    } else {
+      for (int k = lane; k < cnt; k += 32) fold(run, ws->buf[sl][k], w0 + k * 8);
+    }
     __syncwarp();
     if (lane == 0 && p + 2 < npieces) {
       fence_proxy_async_smem();  // the warp's reads of this piece before the copy's writes
