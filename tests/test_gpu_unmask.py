@@ -117,6 +117,51 @@ def test_ties_resolve_to_lowest_index_and_position(davet):
     assert (s.d["argmax"].cpu().numpy() == 5).all()
 
 
+def test_argmax_ties_inside_one_lane_batch(davet):
+    """Equal maxima planted where the row pass must order them itself.
+
+    At V = 126464 and 8 rows a row has 31 vocabulary chunks of 510 16-byte
+    slices; a lane folds its 8 slices of a 256-slice piece (slices
+    lane + 32 m) as one batch when all 8 exist, else slice by slice.  The
+    maxima sit in two slices of one batch, twice in one slice, in two lanes,
+    in two chunks, in a partial piece after a full one, and as a later,
+    larger maximum (the rescale).  argmax must be the first index of the
+    maximum (Eq. 1 reads the arg-max token; ties take the lowest index, as in
+    the oracle), conf as in the oracle.  Should the chunking change, the
+    comparison with the oracle still holds."""
+    V, k, chunk = 126464, 2, 510
+
+    def el(ch, piece, lane, m, pos):
+        return (ch * chunk + piece * 256 + lane + 32 * m) * 8 + pos
+
+    plants = {
+        0: [(el(0, 0, 3, 5, 1), 8.0), (el(0, 0, 3, 2, 5), 8.0)],     # two slices of one batch
+        1: [(el(2, 0, 9, 4, 6), 8.0), (el(2, 0, 9, 4, 2), 8.0)],     # one slice, two positions
+        2: [(el(5, 0, 7, 0, 3), 8.0), (el(5, 0, 2, 1, 0), 8.0)],     # two lanes of one piece
+        3: [(el(3, 0, 0, 0, 0), 8.0), (el(1, 1, 4, 3, 7), 8.0)],     # two chunks
+        4: [(el(4, 1, 31, 6, 4), 8.0), (el(4, 0, 30, 7, 1), 8.0)],   # partial piece after a full one
+        5: [(el(6, 0, 5, 1, 1), 6.0), (el(6, 1, 5, 1, 1), 8.0)],     # a later, larger maximum
+        6: [(el(30, 1, 10, 6, 0), 8.0)],                              # the last chunk
+        7: [],
+    }
+    g = torch.Generator().manual_seed(11)
+    lg = torch.randn((8, V), generator=g) * 0.5
+    expect = {}
+    for r, pl in plants.items():
+        for pos, val in pl:
+            assert 0 <= pos < V
+            lg[r, pos] = val
+        if pl:
+            top = max(v for _, v in pl)
+            expect[r] = min(p for p, v in pl if v == top)
+    lg = lg.to(torch.bfloat16)
+    s = State([8], V, k)
+    s.step(davet, lg)
+    arg = s.d["argmax"].cpu().numpy()
+    for r, e in expect.items():
+        assert arg[r] == e, (r, int(arg[r]), e)
+
+
 def test_churn_and_mean_confidence(davet):
     V, k = 64, 1
     resp = [4]
