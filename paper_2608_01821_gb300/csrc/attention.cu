@@ -487,7 +487,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++np[0];
           tc_fence_after();
           issue_pv(0, st, j == 0);
-          if (w.ntile == 1) umma_commit(&s.v_empty[st]);
+          // the V stage is released with the next commits (after S, when
+          // there is a next key tile): a commit alone between two MMA groups
+          // leaves the tensor pipe idle for a while
           if (more) {
             ok = mbar_wait(&s.k_full[st1], ((it + 1) / NS) & 1, prm.err, abort_flag);
             if (!ok) break;
@@ -495,10 +497,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             issue_s(0, st1);
             if (w.ntile == 1) {
+              umma_commit(&s.v_empty[st]);
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
             }
           } else {
+            if (w.ntile == 1) umma_commit(&s.v_empty[st]);
             umma_commit(&s.o_full[0]);
           }
           if (w.ntile == 2) {
@@ -509,12 +513,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++np[1];
             tc_fence_after();
             issue_pv(1, st, j == 0);
-            umma_commit(&s.v_empty[st]);
             if (more) {
               issue_s(1, st1);
+              umma_commit(&s.v_empty[st]);
               umma_commit(&s.k_empty[st1]);
               if (j + 1 == w.nkv - 1) umma_commit(&s.q_empty);
             } else {
+              umma_commit(&s.v_empty[st]);
               umma_commit(&s.o_full[1]);
             }
           }
