@@ -182,6 +182,43 @@ def test_invalid_arguments_are_rejected_without_a_device(lib):
     assert lib.davet_policy_step(0, 16, p, p, null, 1, d(0.5), None, p, null, null) == INV
 
 
+def test_noalloc_validates_before_touching_the_device(lib):
+    """davet_unmask_topk_noalloc returns its argument and size statuses
+    before any device call, so they hold on a machine without a GPU.  Its
+    scratch array is DAVET_NOALLOC_SCRATCH_BYTES (1 MiB); with one vocabulary
+    chunk per row a row needs a 16-byte chunk record, a 4-byte confidence and
+    a 4-byte index, each array starting on a 256-byte boundary.  One row more
+    than that holds is rejected as unsupported; pointers are never read."""
+    OK, INV, UNS = 0, 1, 2
+    p = ctypes.c_void_p(1 << 20)
+    scratch = 1 << 20
+
+    def a256(x):
+        return (x + 255) & ~255
+
+    rows = scratch // 24
+    while a256(16 * rows) + 2 * a256(4 * rows) > scratch:
+        rows -= 1
+    for V in (1024, 126464):
+        assert lib.davet_unmask_topk_noalloc(p, V, p, 1, rows + 1, 2, p, p, None, None, None, None, None) == UNS
+    assert lib.davet_unmask_topk_noalloc(p, 126464, p, 1, 1 << 40, 2, p, p, None, None, None, None, None) == UNS
+    assert lib.davet_unmask_topk_noalloc(p, 126464, p, 70000, 100, 2, p, p, None, None, None, None, None) == UNS
+    # argument errors: V not a multiple of 8, k out of range, null state,
+    # logits off a 16-byte boundary, negative sizes
+    assert lib.davet_unmask_topk_noalloc(p, 1001, p, 1, 10, 2, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, 1, 10, 0, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, 1, 10, 1025, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, None, 1, 10, 2, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, 1, 10, 2, None, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(None, 1024, p, 1, 10, 2, p, p, None, None, None, None, None) == INV
+    odd = ctypes.c_void_p((1 << 20) + 8)
+    assert lib.davet_unmask_topk_noalloc(odd, 1024, p, 1, 10, 2, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, 1, -1, 2, p, p, None, None, None, None, None) == INV
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, -1, 10, 2, p, p, None, None, None, None, None) == INV
+    # no requests: nothing to do
+    assert lib.davet_unmask_topk_noalloc(p, 1024, p, 0, 0, 2, p, p, None, None, None, None, None) == OK
+
+
 def test_package_fails_loudly_without_library(tmp_path):
     from paper_2608_01821_gb300 import davet
     saved = davet._lib
